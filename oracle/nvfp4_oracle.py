@@ -1,0 +1,381 @@
+"""CPU oracle for the NVFP4 W4A4KV4 hot path -- TEST INFRASTRUCTURE ONLY.
+
+Only the test suite, ``__graft_entry__.smoke()`` and the ``cpu_baseline`` /
+``--impl reference`` legs of ``bench.py`` may import this module.  The product
+path (the CUDA library and its Python binding) never calls it, and this module
+imports nothing from the product package: the two share no code.
+
+Everything here is the plain definition of what the path computes, written for
+readability, not speed:
+
+* the NVFP4 format (Appendix A, table "Quantization configurations of MXFP4 and
+  NVFP4"): E2M1 elements, one FP8-E4M3 scale per block of 16 elements, one FP32
+  per-tensor scale;
+* the quantizer that maps a bf16 tensor onto that format (the paper fixes the
+  format but not the recipe; the reading used is spelled out in ``quantize``);
+* the linear layer on dequantized operands in fp64 (every linear of the decoder
+  is quantized, Appendix D.1);
+* decode attention over a quantized KV cache, ``z = softmax(Q K^T / sqrt(d)) V``
+  with quantized K and V (Sec. 2.1), in fp64;
+* the inference-time Q-FIT key shift ``K~ = R(K_pre / s) - m`` applied before
+  the KV cache is quantized (Eq. 2, Appendix D.3), and the RoPE / paired scaling
+  pieces needed to state its invariances (Sec. 2.1, Eq. 2).
+
+Floating-point conventions: the quantizer's arithmetic is IEEE fp32 with
+round-to-nearest-even (numpy float32 scalars/arrays, no fused multiply-add);
+everything downstream of dequantization is fp64.
+
+Parity status: every function here is pinned by ``tests/test_oracle_pins.py``
+(format tables, hand-worked ties in ``tests/golden/``, closed forms, library
+routines and brute force on tiny inputs); none is "parity unpinned".
+"""
+from __future__ import annotations
+
+import numpy as np
+
+# ---------------------------------------------------------------------------
+# E2M1 elements (Appendix A: FP4 with 2 exponent bits and 1 mantissa bit).
+# A 4-bit code is  s e1 e0 m : sign, exponent (bias 1), mantissa.
+#   e == 0 : subnormal, value = m * 0.5
+#   e >= 1 : value = 2**(e-1) * (1 + m/2)
+# The eight magnitudes are therefore 0, 0.5, 1, 1.5, 2, 3, 4, 6.
+# ---------------------------------------------------------------------------
+
+
+def e2m1_decode(code):
+    """Value of 4-bit E2M1 codes (array of ints 0..15) as float64."""
+    code = np.asarray(code, dtype=np.int64)
+    sign = np.where(code & 0x8, -1.0, 1.0)
+    e = (code >> 1) & 0x3
+    m = code & 0x1
+    mag = np.where(e == 0, m * 0.5, np.ldexp(1.0 + m / 2.0, e - 1))
+    return sign * mag
+
+
+E2M1_GRID = e2m1_decode(np.arange(8))  # non-negative magnitudes, index == code
+
+
+def e2m1_encode(v):
+    """Round float values onto E2M1, round-to-nearest-even, saturating at 6.
+
+    The nearest grid point is chosen by brute force over the eight magnitudes;
+    on an exact tie the code with an even index (even mantissa bit) wins.
+    Values beyond 6 saturate to 6 ("satfinite").  The sign bit is kept, also
+    when the magnitude rounds to zero (``-0.1 -> 0x8``).
+    Inputs must be finite.
+    """
+    v = np.asarray(v, dtype=np.float64)
+    flat = v.reshape(-1)
+    out = np.empty(flat.shape, dtype=np.uint8)
+    step = 1 << 20
+    for lo in range(0, flat.size, step):
+        x = flat[lo:lo + step]
+        mag = np.abs(x)
+        dist = np.abs(mag[:, None] - E2M1_GRID[None, :])          # (n, 8)
+        best = dist.min(axis=1, keepdims=True)
+        cand = dist == best                                          # ties: <= 2 adjacent
+        even = cand & ((np.arange(8) % 2) == 0)[None, :]
+        idx = np.where(even.any(axis=1), even.argmax(axis=1), cand.argmax(axis=1))
+        idx = np.where(mag >= 6.0, 7, idx)
+        out[lo:lo + step] = (idx | (np.signbit(x).astype(np.int64) << 3)).astype(np.uint8)
+    return out.reshape(v.shape)
+
+
+# ---------------------------------------------------------------------------
+# FP8 E4M3 block scales (Appendix A).  OCP E4M3 "FN": 1 sign, 4 exponent bits
+# (bias 7), 3 mantissa bits, no infinities, S.1111.111 is NaN, max 448.
+# NVFP4 block scales are non-negative, i.e. the unsigned view the tensor core
+# consumes; the encoder never produces the sign bit nor 0x7F.
+# ---------------------------------------------------------------------------
+
+E4M3_MAX = 448.0
+
+
+def e4m3_decode(code):
+    """Value of 8-bit E4M3 codes (array of ints 0..255) as float64 (NaN for 0x7F/0xFF)."""
+    code = np.asarray(code, dtype=np.int64)
+    sign = np.where(code & 0x80, -1.0, 1.0)
+    e = (code >> 3) & 0xF
+    m = code & 0x7
+    mag = np.where(e == 0, np.ldexp(m / 8.0, -6), np.ldexp(1.0 + m / 8.0, e - 7))
+    mag = np.where((e == 15) & (m == 7), np.nan, mag)
+    return sign * mag
+
+
+def e4m3_encode_nonneg(s):
+    """Round non-negative values onto E4M3 (RNE), saturating to 448 ("satfinite").
+
+    For s in binade [2**E, 2**(E+1)) with E >= -6 the representable values are
+    multiples of 2**(E-3); below 2**-6 (subnormals) they are multiples of 2**-9.
+    The value is rounded to the nearest multiple with ties to even (an even
+    multiple is an even mantissa), then clamped to 448.  +inf saturates too.
+    """
+    s = np.asarray(s, dtype=np.float64)
+    if np.any(np.isnan(s)) or np.any(s < 0):
+        raise ValueError("e4m3_encode_nonneg: inputs must be non-negative and not NaN")
+    finite = np.isfinite(s)
+    sf = np.where(finite, s, 0.0)
+    _, ex = np.frexp(sf)                    # sf = f * 2**ex, f in [0.5, 1)
+    binade = np.maximum(ex - 1, -6)         # floor(log2(sf)), clamped to the subnormal range
+    quantum = np.ldexp(1.0, binade - 3)
+    val = np.rint(sf / quantum) * quantum   # np.rint: round half to even; the division is exact
+    val = np.where(finite, np.minimum(val, E4M3_MAX), E4M3_MAX)
+    return _e4m3_code_of_value(val)
+
+
+def _e4m3_code_of_value(val):
+    """Code of exactly representable non-negative E4M3 values."""
+    val = np.asarray(val, dtype=np.float64)
+    code = np.zeros(val.shape, dtype=np.int64)
+    sub = (val > 0) & (val < 2.0 ** -6)
+    code = np.where(sub, np.rint(val / 2.0 ** -9).astype(np.int64), code)
+    nrm = val >= 2.0 ** -6
+    _, ex = np.frexp(np.where(nrm, val, 1.0))
+    E = ex - 1
+    mant = np.rint((np.ldexp(np.where(nrm, val, 1.0), -E) - 1.0) * 8).astype(np.int64)
+    code = np.where(nrm, ((E + 7) << 3) | mant, code)
+    return code.astype(np.uint8)
+
+
+# ---------------------------------------------------------------------------
+# NVFP4 tensor quantization.
+# ---------------------------------------------------------------------------
+
+BLOCK = 16                    # elements per E4M3 block scale (Appendix A)
+TENSOR_SCALE_DIV = np.float32(6.0 * 448.0)   # largest E2M1 magnitude x largest E4M3 scale
+
+
+def bf16_bits_to_f32(bits):
+    """bf16 bit patterns (uint16) -> exactly equal float32 values."""
+    bits = np.asarray(bits, dtype=np.uint16)
+    return (bits.astype(np.uint32) << 16).view(np.float32)
+
+
+def tensor_scale(x_f32):
+    """FP32 per-tensor scale g = amax(|x|) / (6 * 448), fp32 division.
+
+    With this g the largest element of the tensor maps onto the largest
+    representable NVFP4 value (E2M1 6 times E4M3 448).  An all-zero tensor gets
+    g = 1 (any positive g quantizes it to zero codes and zero scales).
+    """
+    amax = np.float32(np.max(np.abs(np.asarray(x_f32, dtype=np.float32)))) if np.size(x_f32) else np.float32(0)
+    if amax == 0:
+        return np.float32(1.0)
+    return np.float32(amax / TENSOR_SCALE_DIV)
+
+
+def quantize(x_f32, g):
+    """NVFP4-quantize a [rows, cols] tensor along its rows (cols % 16 == 0).
+
+    Reading of the format (the paper gives the format, not the recipe), per
+    block b of 16 consecutive elements of a row, all fp32 RNE:
+      1. amax_b = max |x_i|
+      2. s_f = amax_b / (6 * g)                       (product, then quotient)
+      3. S = E4M3_RNE_satfinite(s_f)                  (block scale code)
+      4. if S == 0: codes are the signs only (signed zeros)
+         else:      v_i = x_i * (1 / (S * g))          (product, reciprocal, product)
+                    code_i = E2M1_RNE_satfinite(v_i)  (sign kept)
+    Returns (codes uint8 [rows, cols/2] with element 2j in the low nibble of
+    byte j and element 2j+1 in the high nibble, scales uint8 [rows, cols/16]).
+    """
+    x = np.asarray(x_f32, dtype=np.float32)
+    rows, cols = x.shape
+    if cols % BLOCK:
+        raise ValueError("cols must be a multiple of 16")
+    g = np.float32(g)
+    if not (np.isfinite(g) and g > 0):
+        raise ValueError("tensor scale must be positive and finite")
+    xb = x.reshape(rows, cols // BLOCK, BLOCK)
+    amax = np.max(np.abs(xb), axis=2)                               # exact
+    six_g = np.float32(np.float32(6.0) * g)
+    with np.errstate(over="ignore", divide="ignore"):
+        s_f = (amax / six_g).astype(np.float32)
+    S = e4m3_encode_nonneg(s_f)                                      # uint8 [rows, cols/16]
+    S_val = e4m3_decode(S).astype(np.float32)                        # exact
+    d = (S_val * g).astype(np.float32)
+    zero_scale = S == 0
+    with np.errstate(divide="ignore", over="ignore"):
+        r = np.where(zero_scale, np.float32(0.0), np.float32(1.0) / np.where(zero_scale, np.float32(1.0), d))
+    r = r.astype(np.float32)
+    v = (xb * r[:, :, None]).astype(np.float32)                     # zero scale -> signed zeros
+    codes = e2m1_encode(v).reshape(rows, cols)
+    packed = (codes[:, 0::2] | (codes[:, 1::2] << 4)).astype(np.uint8)
+    return packed, S
+
+
+def unpack_codes(packed):
+    """uint8 [rows, cols/2] -> 4-bit codes [rows, cols] (low nibble first)."""
+    packed = np.asarray(packed, dtype=np.uint8)
+    out = np.empty(packed.shape[:-1] + (packed.shape[-1] * 2,), dtype=np.uint8)
+    out[..., 0::2] = packed & 0xF
+    out[..., 1::2] = packed >> 4
+    return out
+
+
+def dequantize(packed, scales, g):
+    """x_hat = e2m1(code) * e4m3(S) * g, evaluated in fp64 (exact)."""
+    codes = unpack_codes(packed)
+    vals = e2m1_decode(codes)
+    rows, cols = codes.shape[-2], codes.shape[-1]
+    s = e4m3_decode(scales).astype(np.float64)
+    s = np.repeat(s, BLOCK, axis=-1)
+    return vals * s * np.float64(np.float32(g))
+
+
+# ---------------------------------------------------------------------------
+# Block-scale storage order consumed by the tensor core ("MMA layout").
+# Rows are grouped in tiles of 128, K-blocks in groups of 4 (64 elements).
+# Each (row-tile, k-group) pair owns 512 contiguous bytes; pairs are stored
+# k-group-fastest.  Inside a 512-byte atom, row r and k-block kb sit at byte
+#     (r % 32) * 16 + ((r % 128) // 32) * 4 + (kb % 4).
+# Rows beyond the tensor (padding up to a multiple of 128) hold zero.
+# ---------------------------------------------------------------------------
+
+
+def mma_scale_bytes(rows, cols):
+    return ((rows + 127) // 128) * 128 * (cols // BLOCK)
+
+
+def scales_to_mma(scales):
+    """Row-major [rows, cols/16] scales -> flat MMA-layout byte array."""
+    scales = np.asarray(scales, dtype=np.uint8)
+    rows, kblocks = scales.shape
+    if kblocks % 4:
+        raise ValueError("cols must be a multiple of 64 for the MMA layout")
+    kgroups = kblocks // 4
+    out = np.zeros(mma_scale_bytes(rows, kblocks * BLOCK), dtype=np.uint8)
+    for r in range(rows):
+        for kb in range(kblocks):
+            atom = (r // 128) * kgroups + kb // 4
+            off = atom * 512 + (r % 32) * 16 + ((r % 128) // 32) * 4 + kb % 4
+            out[off] = scales[r, kb]
+    return out
+
+
+def scales_from_mma(flat, rows, cols):
+    """Inverse of ``scales_to_mma`` (drops padding rows)."""
+    flat = np.asarray(flat, dtype=np.uint8).reshape(-1)
+    kblocks = cols // BLOCK
+    kgroups = kblocks // 4
+    r = np.arange(rows)[:, None]
+    kb = np.arange(kblocks)[None, :]
+    off = ((r // 128) * kgroups + kb // 4) * 512 + (r % 32) * 16 + ((r % 128) // 32) * 4 + kb % 4
+    return flat[off]
+
+
+# ---------------------------------------------------------------------------
+# Linear layer on NVFP4 operands (every linear of the decoder, Appendix D.1).
+# D[m, n] = sum_k A_hat[m, k] * W_hat[n, k]  in fp64 on the dequantized inputs.
+# ---------------------------------------------------------------------------
+
+
+def linear(a_codes, a_scales, g_a, w_codes, w_scales, g_w):
+    """fp64 reference of the NVFP4 linear: dequantize both operands, multiply."""
+    a = dequantize(a_codes, a_scales, g_a)
+    w = dequantize(w_codes, w_scales, g_w)
+    return a @ w.T
+
+
+def linear_rows(a_codes, a_scales, g_a, w_codes, w_scales, g_w, rows):
+    """Same as ``linear`` for a subset of output rows (large shapes)."""
+    rows = np.asarray(rows)
+    a = dequantize(a_codes[rows], a_scales[rows], g_a)
+    w = dequantize(w_codes, w_scales, g_w)
+    return a @ w.T
+
+
+# ---------------------------------------------------------------------------
+# KV cache: per-token NVFP4 rows with a static per-layer tensor scale.
+# Cache arrays (one set for K, one for V):
+#     codes  uint8 [batch, kv_heads, capacity, head_dim/2]
+#     scales uint8 [batch, kv_heads, capacity, head_dim/16]
+# Blocks of 16 run along head_dim, so every appended token is self-contained.
+# ---------------------------------------------------------------------------
+
+
+def kv_append(k_codes, k_scales, v_codes, v_scales, k_new, v_new, seq_idx, pos, g_k, g_v, k_shift=None):
+    """Quantize and store new K/V rows in place.
+
+    k_new, v_new: float32 [n_new, kv_heads, head_dim] (bf16 values, post-RoPE K).
+    k_shift: optional float32 [kv_heads, head_dim]: the Q-FIT post-RoPE shift m,
+    subtracted in fp32 before quantization, K~ = R(K) - m (Eq. 2).
+    """
+    k = np.asarray(k_new, dtype=np.float32)
+    v = np.asarray(v_new, dtype=np.float32)
+    n_new, hkv, d = k.shape
+    if k_shift is not None:
+        k = (k - np.asarray(k_shift, dtype=np.float32)[None, :, :]).astype(np.float32)
+    kc, ks = quantize(k.reshape(n_new * hkv, d), g_k)
+    vc, vs = quantize(v.reshape(n_new * hkv, d), g_v)
+    kc = kc.reshape(n_new, hkv, d // 2); ks = ks.reshape(n_new, hkv, d // BLOCK)
+    vc = vc.reshape(n_new, hkv, d // 2); vs = vs.reshape(n_new, hkv, d // BLOCK)
+    for i in range(n_new):
+        b, p = int(seq_idx[i]), int(pos[i])
+        k_codes[b, :, p] = kc[i]; k_scales[b, :, p] = ks[i]
+        v_codes[b, :, p] = vc[i]; v_scales[b, :, p] = vs[i]
+
+
+def decode_attention(q_f32, k_codes, k_scales, v_codes, v_scales, seq_lens, g_k, g_v, softmax_scale,
+                     batches=None, heads=None):
+    """fp64 decode attention over the NVFP4 cache (Sec. 2.1).
+
+    For query head h of sequence b, with KV head kv = h // (H_q / H_kv)
+    (contiguous grouped-query replication):
+        s_t = softmax_scale * (q . K_hat_t),  t < seq_lens[b]
+        o   = sum_t softmax(s)_t * V_hat_t
+    q_f32: [batch, H_q, d].  Returns fp64 [len(batches), len(heads), d].
+    """
+    q = np.asarray(q_f32, dtype=np.float64)
+    B, Hq, d = q.shape
+    Hkv = k_codes.shape[1]
+    if Hq % Hkv:
+        raise ValueError("H_q must be a multiple of H_kv")
+    group = Hq // Hkv
+    batches = range(B) if batches is None else batches
+    heads = range(Hq) if heads is None else heads
+    scale = np.float64(np.float32(softmax_scale))
+    out = np.zeros((len(batches), len(heads), d))
+    for i, b in enumerate(batches):
+        T = int(seq_lens[b])
+        cache = {}
+        for j, h in enumerate(heads):
+            kv = h // group
+            if kv not in cache:
+                cache[kv] = (dequantize(k_codes[b, kv, :T], k_scales[b, kv, :T], g_k),
+                             dequantize(v_codes[b, kv, :T], v_scales[b, kv, :T], g_v))
+            K, V = cache[kv]
+            out[i, j] = attention_fp64(q[b, h], K, V, scale)
+    return out
+
+
+def attention_fp64(q, K, V, scale):
+    """softmax(scale * K q) V for one query vector, numerically stable, fp64."""
+    s = (K @ q) * scale
+    s = s - s.max()
+    p = np.exp(s)
+    p /= p.sum()
+    return p @ V
+
+
+# ---------------------------------------------------------------------------
+# RoPE and the Q-FIT transforms (Sec. 2.1, Eq. 2).  Used to state invariances.
+# RoPE rotates channel pairs (r, r + d/2) by angle pos * theta**(-2r/d).
+# ---------------------------------------------------------------------------
+
+
+def rope(x, positions, theta=1.0e6):
+    """Apply RoPE to x [..., T, d] at integer positions [T] (fp64)."""
+    x = np.asarray(x, dtype=np.float64)
+    d = x.shape[-1]
+    half = d // 2
+    inv = theta ** (-np.arange(half) * 2.0 / d)
+    ang = np.asarray(positions, dtype=np.float64)[:, None] * inv[None, :]
+    c, s = np.cos(ang), np.sin(ang)
+    x1, x2 = x[..., :half], x[..., half:]
+    return np.concatenate([x1 * c - x2 * s, x1 * s + x2 * c], axis=-1)
+
+
+def qfit_transform(q_pre, k_pre, s, m, positions, theta=1.0e6):
+    """Q~ = R(Q_pre * s), K~ = R(K_pre / s) - m  (Eq. 2), fp64."""
+    s = np.asarray(s, dtype=np.float64)
+    return rope(q_pre * s, positions, theta), rope(k_pre / s, positions, theta) - np.asarray(m, np.float64)

@@ -1,0 +1,340 @@
+"""Pins for the CPU oracle: each check ties it to something other than itself.
+
+Sources of truth used here: the NVFP4 format (Appendix A: E2M1 elements, E4M3
+block scale per 16 elements, FP32 tensor scale), hand-worked values in
+tests/golden/, closed forms, a library routine (torch's float8_e4m3fn cast),
+brute force on tiny inputs, and the exact invariances of attention stated in
+Sec. 2.1 / Eq. 2 (softmax shift invariance under the post-RoPE key shift,
+logit preservation under paired pre-RoPE scaling).
+"""
+import math
+import os
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import nvfp4_oracle as O
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def _golden_rows(name):
+    with open(os.path.join(GOLDEN, name)) as f:
+        for line in f:
+            line = line.split("#", 1)[0].strip()
+            if line:
+                yield line
+
+
+# ----------------------------------------------------------------- E2M1 ---
+
+def test_e2m1_decode_exhaustive_table():
+    # Appendix A: E2M1, the eight magnitudes 0, .5, 1, 1.5, 2, 3, 4, 6 and a sign bit.
+    expect = [0, .5, 1, 1.5, 2, 3, 4, 6, -0.0, -.5, -1, -1.5, -2, -3, -4, -6]
+    got = O.e2m1_decode(np.arange(16))
+    assert np.array_equal(got, np.array(expect))
+    assert np.signbit(got[8])
+
+
+def test_e2m1_roundtrip_all_codes():
+    for c in range(16):
+        assert O.e2m1_encode(O.e2m1_decode(c)) == c
+
+
+def test_e2m1_golden_ties_and_saturation():
+    for row in _golden_rows("e2m1_rne.txt"):
+        v, c = row.split()
+        assert O.e2m1_encode(np.float64(float(v))) == int(c, 16), row
+
+
+def test_e2m1_neighbours_of_midpoints():
+    # Just off a tie the nearest grid point decides, whatever the tie rule.
+    grid = O.E2M1_GRID
+    for i in range(7):
+        mid = np.float32((grid[i] + grid[i + 1]) / 2)
+        lo = np.nextafter(mid, np.float32(0)); hi = np.nextafter(mid, np.float32(10))
+        assert O.e2m1_encode(lo) == i and O.e2m1_encode(hi) == i + 1
+        assert O.e2m1_encode(-lo) == 8 | i and O.e2m1_encode(-hi) == 8 | (i + 1)
+
+
+def test_e2m1_is_nearest_point_dense_sweep():
+    # Independent check of "nearest": the decoded value is never farther from v
+    # than any other grid magnitude.
+    v = np.linspace(-7, 7, 20001)
+    c = O.e2m1_encode(v)
+    dec = np.abs(O.e2m1_decode(c))
+    dist = np.abs(np.abs(np.minimum(np.abs(v), 6.0))[:, None] - O.E2M1_GRID[None, :]).min(axis=1)
+    assert np.allclose(np.abs(np.minimum(np.abs(v), 6.0) - dec), dist, atol=0)
+
+
+# ----------------------------------------------------------------- E4M3 ---
+
+def test_e4m3_decode_matches_library_all_codes():
+    lib = torch.arange(256, dtype=torch.int32).to(torch.uint8).view(torch.float8_e4m3fn).double().numpy()
+    ours = O.e4m3_decode(np.arange(256))
+    assert np.array_equal(np.isnan(lib), np.isnan(ours))
+    fin = ~np.isnan(lib)
+    assert np.array_equal(lib[fin], ours[fin])
+
+
+def test_e4m3_encode_identity_on_all_finite_nonneg_codes():
+    codes = np.arange(0x7F)  # 0x00..0x7E: every finite non-negative value
+    assert np.array_equal(O.e4m3_encode_nonneg(O.e4m3_decode(codes)), codes.astype(np.uint8))
+
+
+def test_e4m3_encode_matches_library_rne_in_range():
+    rng = np.random.default_rng(7)
+    v = np.concatenate([rng.uniform(0, 448, 20000), np.exp(rng.uniform(-16, 6, 20000)),
+                        (O.e4m3_decode(np.arange(0x7E)) + O.e4m3_decode(np.arange(1, 0x7F))) / 2])
+    v = v.astype(np.float32)
+    lib = torch.from_numpy(v).to(torch.float8_e4m3fn).view(torch.uint8).numpy()
+    assert np.array_equal(O.e4m3_encode_nonneg(v), lib)
+
+
+def test_e4m3_golden_and_saturation():
+    for row in _golden_rows("e4m3_rne.txt"):
+        v, c = row.split()
+        assert O.e4m3_encode_nonneg(np.float64(float(v))) == int(c, 16), row
+    assert O.e4m3_encode_nonneg(np.inf) == 0x7E
+
+
+# ------------------------------------------------------------- quantize ---
+
+def _parse_block(row):
+    g, vals, sc, packed = [p.strip() for p in row.split("|")]
+    vals = [float(t) for t in vals.split()]
+    return np.float32(float(g)), np.array(vals, np.float32), int(sc, 16), [int(t, 16) for t in packed.split()]
+
+
+def test_quantize_golden_blocks():
+    n = 0
+    for row in _golden_rows("nvfp4_blocks.txt"):
+        g, x, sc, packed = _parse_block(row)
+        codes, scales = O.quantize(x[None, :], g)
+        assert scales[0, 0] == sc, row
+        assert list(codes[0]) == packed, row
+        n += 1
+    assert n == 6
+
+
+def test_quantize_scale_closed_form_and_error_bound():
+    rng = np.random.default_rng(1)
+    x = (rng.standard_normal((64, 256)) * np.exp(rng.uniform(-3, 3, (64, 1)))).astype(np.float32)
+    g = O.tensor_scale(x)
+    codes, S = O.quantize(x, g)
+    s_true = np.abs(x.reshape(64, 16, 16)).max(axis=2) / (6.0 * float(g))
+    s_val = O.e4m3_decode(S)
+    normal = s_true >= 2 ** -6
+    # RNE onto 3 mantissa bits: relative error at most 2**-4 in the normal range.
+    assert np.all(np.abs(s_val[normal] - s_true[normal]) <= 2 ** -4 * s_true[normal] * (1 + 1e-6))
+    # The block holding the tensor amax maps to the largest scale, 448.
+    r, b = np.unravel_index(np.argmax(np.abs(x)), x.shape)
+    assert S[r, b // 16] == 0x7E
+    # Element error: half the local grid spacing times S*g, plus saturation.
+    xh = O.dequantize(codes, S, g)
+    Sg = np.repeat(s_val, 16, axis=1) * float(g)
+    v = np.abs(x) / np.where(Sg > 0, Sg, 1)
+    gap = np.where(v < 2, 0.5, np.where(v < 4, 1.0, 2.0))
+    bound = 0.5 * gap * Sg + np.maximum(v - 6, 0) * Sg + 1e-6 * np.abs(x)
+    assert np.all(np.abs(x - xh) <= bound)
+
+
+def test_quantize_roundtrip_of_representable_blocks():
+    # Every code, both signs, in blocks whose amax pins S exactly: quantize(dequant) == id.
+    rng = np.random.default_rng(3)
+    for _ in range(20):
+        g = np.float32(2.0 ** rng.integers(-20, 5))
+        S = int(rng.integers(0x08, 0x7F))                  # normal E4M3 scale
+        codes = rng.integers(0, 16, 16).astype(np.uint8)
+        codes[0] = 7                                        # amax element = 6 * S * g
+        packed = (codes[0::2] | (codes[1::2] << 4)).astype(np.uint8)[None, :]
+        x = O.dequantize(packed, np.array([[S]], np.uint8), g).astype(np.float32)
+        c2, s2 = O.quantize(x, g)
+        assert s2[0, 0] == S and np.array_equal(c2, packed)
+
+
+def test_pack_order_low_nibble_first():
+    x = np.zeros((1, 16), np.float32)
+    x[0, 0] = 6.0  # code 7 in the low nibble of byte 0
+    x[0, 3] = -3.0  # code 0xD in the high nibble of byte 1
+    codes, _ = O.quantize(x, np.float32(1.0))
+    assert codes[0, 0] == 0x07 and codes[0, 1] == 0xD0
+
+
+def test_tensor_scale_closed_form():
+    x = np.array([[0.5, -2688.0, 3.0]], np.float32)
+    assert O.tensor_scale(x) == np.float32(1.0)
+    assert O.tensor_scale(np.zeros((2, 16), np.float32)) == np.float32(1.0)
+
+
+# ----------------------------------------------------------- MMA layout ---
+
+def test_mma_layout_golden_offsets():
+    rows, cols = 256, 128
+    S = np.zeros((rows, cols // 16), np.uint8)
+    for row in _golden_rows("mma_scale_layout.txt"):
+        r, kb, off = (int(t) for t in row.split())
+        S[:] = 0
+        S[r, kb] = 0xA5
+        flat = O.scales_to_mma(S)
+        assert flat.size == 2048 and np.flatnonzero(flat).tolist() == [off], row
+
+
+def test_mma_layout_roundtrip_and_padding():
+    rng = np.random.default_rng(5)
+    for rows, cols in [(1, 64), (130, 192), (256, 128), (17, 1536)]:
+        S = rng.integers(1, 255, (rows, cols // 16)).astype(np.uint8)
+        flat = O.scales_to_mma(S)
+        assert flat.size == ((rows + 127) // 128) * 128 * cols // 16
+        assert np.array_equal(O.scales_from_mma(flat, rows, cols), S)
+        assert np.count_nonzero(flat) == S.size  # padding rows are zero
+
+
+# ----------------------------------------------------------------- GEMM ---
+
+def _brute_linear(a, w):
+    M, K = a.shape
+    N = w.shape[0]
+    out = [[0.0] * N for _ in range(M)]
+    for m in range(M):
+        for n in range(N):
+            acc = 0.0
+            for k in range(K):
+                acc += float(a[m, k]) * float(w[n, k])
+            out[m][n] = acc
+    return np.array(out)
+
+
+@pytest.mark.parametrize("M,N,K", [(3, 5, 16), (7, 4, 32), (2, 9, 64), (5, 3, 256)])
+def test_linear_brute_force(M, N, K):
+    rng = np.random.default_rng(M * 100 + N)
+    a = rng.standard_normal((M, K)).astype(np.float32)
+    w = (rng.standard_normal((N, K)) * 0.02).astype(np.float32)
+    ga, gw = O.tensor_scale(a), O.tensor_scale(w)
+    ac, as_ = O.quantize(a, ga)
+    wc, ws = O.quantize(w, gw)
+    ref = O.linear(ac, as_, ga, wc, ws, gw)
+    brute = _brute_linear(O.dequantize(ac, as_, ga), O.dequantize(wc, ws, gw))
+    assert ref.shape == (M, N)
+    assert np.allclose(ref, brute, rtol=1e-12, atol=1e-300)
+    # Rows subset agrees with the full product.
+    assert np.allclose(O.linear_rows(ac, as_, ga, wc, ws, gw, [M - 1, 0]), ref[[M - 1, 0]], rtol=1e-13, atol=0)
+
+
+def test_linear_k16_is_outer_product_and_identity_codes():
+    a = np.array([[1, 2, 0, 0, 0, 0, 0, 0, 0, 0, 0, 0, 0, 0, 0, 0]], np.float32) * 3.0
+    w = np.zeros((16, 16), np.float32)
+    for i in range(16):
+        w[i, i] = 6.0                                       # W = 6 * I, exact in NVFP4 with S = 1, g = 1
+    ac, as_ = O.quantize(a, np.float32(1.0))
+    wc, ws = O.quantize(w, np.float32(1.0))
+    out = O.linear(ac, as_, 1.0, wc, ws, 1.0)
+    assert np.array_equal(out, 6.0 * O.dequantize(ac, as_, 1.0))
+    # K = 16, single block: the result is an outer product of (dequantized) vectors.
+    u = O.dequantize(*O.quantize(np.ones((4, 16), np.float32) * np.arange(1, 5, dtype=np.float32)[:, None], 1.0), 1.0)
+    v = O.dequantize(*O.quantize(np.ones((3, 16), np.float32) * np.float32(0.5), 1.0), 1.0)
+    assert np.array_equal(O.linear(*O.quantize(np.ones((4, 16), np.float32) * np.arange(1, 5, dtype=np.float32)[:, None], 1.0), 1.0,
+                                   *O.quantize(np.ones((3, 16), np.float32) * np.float32(0.5), 1.0), 1.0),
+                          16 * np.outer(u[:, 0], v[:, 0]))
+
+
+# ------------------------------------------------------------ attention ---
+
+def _cache(rng, B, Hkv, T, d=128, cap=None):
+    cap = cap or T
+    kc = np.zeros((B, Hkv, cap, d // 2), np.uint8); ks = np.zeros((B, Hkv, cap, d // 16), np.uint8)
+    vc = np.zeros_like(kc); vs = np.zeros_like(ks)
+    k = rng.standard_normal((B * T, Hkv, d)).astype(np.float32)
+    v = rng.standard_normal((B * T, Hkv, d)).astype(np.float32)
+    gk, gv = O.tensor_scale(k), O.tensor_scale(v)
+    seq = np.repeat(np.arange(B), T); pos = np.tile(np.arange(T), B)
+    O.kv_append(kc, ks, vc, vs, k, v, seq, pos, gk, gv)
+    return kc, ks, vc, vs, gk, gv
+
+
+def test_attention_single_token_returns_v():
+    rng = np.random.default_rng(11)
+    kc, ks, vc, vs, gk, gv = _cache(rng, 2, 2, 1)
+    q = rng.standard_normal((2, 6, 128)).astype(np.float32)
+    out = O.decode_attention(q, kc, ks, vc, vs, [1, 1], gk, gv, 1 / math.sqrt(128))
+    for b in range(2):
+        for h in range(6):
+            assert np.array_equal(out[b, h], O.dequantize(vc[b, h // 3, :1], vs[b, h // 3, :1], gv)[0])
+
+
+def test_attention_equal_keys_or_zero_query_is_mean_of_v():
+    rng = np.random.default_rng(12)
+    kc, ks, vc, vs, gk, gv = _cache(rng, 1, 1, 37)
+    V = O.dequantize(vc[0, 0], vs[0, 0], gv)
+    q0 = np.zeros((1, 2, 128), np.float32)
+    out = O.decode_attention(q0, kc, ks, vc, vs, [37], gk, gv, 0.1)
+    assert np.allclose(out[0, 0], V.mean(axis=0), rtol=1e-13, atol=1e-15)
+    kc[0, 0, :] = kc[0, 0, 5]; ks[0, 0, :] = ks[0, 0, 5]      # all keys equal
+    q = rng.standard_normal((1, 2, 128)).astype(np.float32)
+    out = O.decode_attention(q, kc, ks, vc, vs, [37], gk, gv, 0.1)
+    assert np.allclose(out[0, 1], V.mean(axis=0), rtol=1e-13, atol=1e-15)
+
+
+def test_attention_brute_force_and_gqa_map():
+    rng = np.random.default_rng(13)
+    kc, ks, vc, vs, gk, gv = _cache(rng, 2, 2, 9)
+    q = rng.standard_normal((2, 10, 128)).astype(np.float32)
+    out = O.decode_attention(q, kc, ks, vc, vs, [9, 4], gk, gv, 0.125)
+    for b, T in [(0, 9), (1, 4)]:
+        for h in range(10):
+            kv = h // 5                                       # contiguous groups of 5 query heads
+            K = O.dequantize(kc[b, kv, :T], ks[b, kv, :T], gk)
+            V = O.dequantize(vc[b, kv, :T], vs[b, kv, :T], gv)
+            logits = [0.125 * sum(float(q[b, h, i]) * K[t, i] for i in range(128)) for t in range(T)]
+            mx = max(logits)
+            e = [math.exp(l - mx) for l in logits]
+            ref = sum(e[t] / sum(e) * V[t] for t in range(T))
+            assert np.allclose(out[b, h], ref, rtol=1e-12, atol=1e-14)
+
+
+def test_attention_invariant_to_key_shift():
+    # Softmax shift invariance behind the post-RoPE shift K~ = R(K) - m (Sec. 2.1, Eq. 2):
+    # subtracting the same vector from every key changes all logits of a query by a constant.
+    rng = np.random.default_rng(14)
+    K = rng.standard_normal((50, 128)); V = rng.standard_normal((50, 128)); q = rng.standard_normal(128)
+    m = rng.standard_normal(128) * 3
+    a = O.attention_fp64(q, K, V, 0.09)
+    b = O.attention_fp64(q, K - m[None, :], V, 0.09)
+    assert np.allclose(a, b, rtol=1e-12, atol=1e-13)
+    assert not np.allclose(O.attention_fp64(q, K * 1.5, V, 0.09), a)  # the check can fail
+
+
+def test_paired_scaling_commutes_with_rope_and_preserves_logits():
+    # Eq. 2 / Sec. 2.1: with s_r = s_{r+d/2}, R(q*s) . R(k/s) == R(q) . R(k).
+    rng = np.random.default_rng(15)
+    d, T = 128, 20
+    q_pre = rng.standard_normal((T, d)); k_pre = rng.standard_normal((T, d))
+    half = np.exp(rng.standard_normal(d // 2))
+    s = np.concatenate([half, half])
+    pos = np.arange(T) * 37
+    qt, kt = O.qfit_transform(q_pre, k_pre, s, np.zeros(d), pos)
+    q0, k0 = O.rope(q_pre, pos), O.rope(k_pre, pos)
+    assert np.allclose(qt @ kt.T, q0 @ k0.T, rtol=1e-10, atol=1e-10)
+    # An unpaired scale breaks it (so the check can fail).
+    s_bad = np.exp(rng.standard_normal(d))
+    qb, kb = O.qfit_transform(q_pre, k_pre, s_bad, np.zeros(d), pos)
+    assert not np.allclose(qb @ kb.T, q0 @ k0.T, rtol=1e-6)
+    # RoPE preserves norms (a rotation of channel pairs).
+    assert np.allclose(np.linalg.norm(q0, axis=1), np.linalg.norm(q_pre, axis=1))
+
+
+def test_kv_append_shift_is_subtracted_before_quantization():
+    rng = np.random.default_rng(16)
+    B, Hkv, d = 1, 2, 128
+    k = rng.standard_normal((3, Hkv, d)).astype(np.float32) + 4.0
+    v = rng.standard_normal((3, Hkv, d)).astype(np.float32)
+    m = np.full((Hkv, d), 4.0, np.float32)
+    kc = np.zeros((B, Hkv, 8, 64), np.uint8); ks = np.zeros((B, Hkv, 8, 8), np.uint8)
+    vc = np.zeros_like(kc); vs = np.zeros_like(ks)
+    O.kv_append(kc, ks, vc, vs, k, v, [0, 0, 0], [5, 1, 2], np.float32(0.01), np.float32(0.02), k_shift=m)
+    c, s = O.quantize((k[0] - m).astype(np.float32), np.float32(0.01))
+    assert np.array_equal(kc[0, :, 5], c) and np.array_equal(ks[0, :, 5], s)
+    c, s = O.quantize(v[1], np.float32(0.02))
+    assert np.array_equal(vc[0, :, 1], c) and np.array_equal(vs[0, :, 1], s)
+    assert not kc[0, :, 0].any() and not kc[0, :, 3:5].any()
