@@ -1,0 +1,455 @@
+"""Benchmark of the NVFP4 W4A4KV4 hot path on GB300.
+
+One step = one pass of the path over one batch of synthetic inputs of the
+Qwen-1.5B-shaped prefill layer (M = 2048 tokens): for each linear (qkv, o,
+gate_up, down) the FP32 tensor scale of its bf16 activation, NVFP4
+quantization of the activation, and the block-scaled FP4 GEMM to bf16.
+Weights are quantized once, before timing.  The headline value is the GEMM
+FLOPs of the step divided by its device time (TFLOP/s).
+
+The decode-attention half of the metric is measured in the same run on the
+Qwen-14B-shaped decode workload (batch 64, 40/8 heads, 16384-token NVFP4
+cache): per step, quantize-and-append one new K/V token per sequence and run
+decode attention over the cache; reported as algorithmic HBM GB/s under
+"decode_attention".
+
+Timing: CUDA events on the launching stream around each step, L2 flushed
+(256 MiB write) between steps, steps replayed from a CUDA graph.  Clocks are
+sampled with nvidia-smi while the timed loops run.  `--impl reference` times
+the CPU oracle instead, on a bounded sample of the same workload.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+GEMM_WL = "qwen1.5b_prefill_linears_m2048"
+ATTN_WL = "qwen14b_decode_attention_b64_t16384"
+METRIC = "NVFP4 GEMM TFLOP/s & FP4-KV decode-attn HBM GB/s vs GB300 roofline"
+FP4_OVER_BF16 = 13.5 / 2.25  # nominal dense FP4 / BF16 tensor ratio of GB300
+
+
+def load_peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return {"hbm_gbs": float(p["hbm_gbs"]), "bf16_tflops": float(p["bf16_tflops"]),
+                "bf16_tflops_sustained": float(p.get("bf16_tflops_sustained", p["bf16_tflops"])), "src": "measured"}
+    except (OSError, KeyError, ValueError):
+        return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0, "src": "fallback"}
+
+
+# ------------------------------------------------------------ clocks ---
+
+class ClockSampler:
+    """nvidia-smi clock/throttle sampling in a background process."""
+
+    Q = ("timestamp,index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
+         "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+         "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, device_index):
+        self.dev = device_index
+        self.rows = []
+        self.proc = None
+        self.windows = []
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", f"--query-gpu={self.Q}", "--format=csv,noheader,nounits",
+                                          "-i", str(self.dev), "-lms", "50"], stdout=subprocess.PIPE,
+                                         stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+            return
+        def reader():
+            for line in self.proc.stdout:
+                self.rows.append((time.time(), line.strip()))
+        self.t = threading.Thread(target=reader, daemon=True)
+        self.t.start()
+
+    def mark(self, t0, t1):
+        self.windows.append((t0, t1))
+
+    def stop(self):
+        if self.proc:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+            self.t.join(timeout=2)
+
+    def summary(self):
+        parsed = []
+        for ts, line in self.rows:
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                parsed.append((ts, float(f[2]), float(f[3]), f[5:9]))
+            except ValueError:
+                continue
+        if not parsed:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"], "samples": 0}
+        inside = [p for p in parsed if any(a - 0.06 <= p[0] <= b + 0.06 for a, b in self.windows)]
+        use = inside or parsed
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for p in use for i, v in enumerate(p[3]) if v.lower() == "active"})
+        return {"sm_mhz": statistics.median(p[1] for p in use), "sm_max_mhz": max(p[2] for p in use),
+                "reasons": reasons, "samples": len(use), "in_timed_region": bool(inside)}
+
+
+# ---------------------------------------------------------- our arm ---
+
+def run_ours(args, rank, world):
+    import numpy as np
+    import torch
+
+    from paper_2606_15682_gb300 import build as B
+    B.build()
+    from paper_2606_15682_gb300 import nvfp4 as N
+    from paper_2606_15682_gb300 import synth
+
+    dev = torch.device("cuda", int(os.environ.get("LOCAL_RANK", 0)))
+    torch.cuda.set_device(dev)
+    stream = torch.cuda.Stream(device=dev)
+    peaks = load_peaks()
+    flush_buf = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    sampler = ClockSampler(dev.index)
+    sampler.start()
+
+    # ---------------- GEMM step: prefill linears with on-the-fly activation quantization
+    w = synth.WORKLOADS[GEMM_WL]
+    M = w["M"]
+    layers = []
+    flops = 0
+    for name, (Nn, K) in w["linears"].items():
+        a, W = synth.linear_inputs(GEMM_WL, name, device=dev)
+        gw = torch.empty(1, dtype=torch.float32, device=dev)
+        wc = torch.empty(Nn, K // 2, dtype=torch.uint8, device=dev)
+        ws = torch.empty(N.nvfp4_scales_bytes(Nn, K, N.SCALES_MMA), dtype=torch.uint8, device=dev)
+        N.nvfp4_tensor_scale(W, gw)
+        N.nvfp4_quantize(W, gw, wc, ws, N.SCALES_MMA)
+        del W
+        L = dict(name=name, N=Nn, K=K, a=a, wc=wc, ws=ws, gw=gw,
+                 ga=torch.empty(1, dtype=torch.float32, device=dev),
+                 ac=torch.empty(M, K // 2, dtype=torch.uint8, device=dev),
+                 asf=torch.empty(N.nvfp4_scales_bytes(M, K, N.SCALES_MMA), dtype=torch.uint8, device=dev),
+                 out=torch.empty(M, Nn, dtype=torch.bfloat16, device=dev),
+                 ev=[torch.cuda.Event(enable_timing=True) for _ in range(2)])
+        layers.append(L)
+        flops += 2 * M * Nn * K
+    torch.cuda.synchronize()
+
+    def gemm_step(record_gemm_events):
+        for L in layers:
+            N.nvfp4_tensor_scale(L["a"], L["ga"])
+            N.nvfp4_quantize(L["a"], L["ga"], L["ac"], L["asf"], N.SCALES_MMA)
+            if record_gemm_events:
+                L["ev"][0].record()
+            N.nvfp4_linear(L["ac"], L["asf"], L["ga"], L["wc"], L["ws"], L["gw"], L["out"], M, L["N"], L["K"])
+            if record_gemm_events:
+                L["ev"][1].record()
+
+    with torch.cuda.stream(stream):
+        gemm_step(False)
+        stream.synchronize()
+        graph = torch.cuda.CUDAGraph()
+        n0 = N.nvfp4_launch_count()
+        with torch.cuda.graph(graph, stream=stream):
+            gemm_step(False)
+        launches_per_step = N.nvfp4_launch_count() - n0
+    torch.cuda.synchronize()
+
+    def timed_loop(replay, steps, warmup, per_step_extra=None):
+        with torch.cuda.stream(stream):
+            for _ in range(warmup):
+                replay()
+                flush_buf.zero_()
+            stream.synchronize()
+            evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(steps)]
+            barrier()
+            t0 = time.time()
+            for i in range(steps):
+                evs[i][0].record(stream)
+                replay()
+                evs[i][1].record(stream)
+                if per_step_extra:
+                    per_step_extra(i)
+                flush_buf.zero_()
+            stream.synchronize()
+            t1 = time.time()
+            barrier()
+        sampler.mark(t0, t1)
+        return [a.elapsed_time(b) for a, b in evs]
+
+    def barrier():
+        if world > 1:
+            import torch.distributed as dist
+            dist.barrier()
+
+    step_ms = timed_loop(graph.replay, args.steps, args.warmup)
+    # GEMM-only kernel durations (same work, eager launches with events between kernels).
+    gemm_ms = {L["name"]: [] for L in layers}
+    with torch.cuda.stream(stream):
+        for _ in range(max(3, min(args.steps, 20))):
+            gemm_step(True)
+            stream.synchronize()
+            for L in layers:
+                gemm_ms[L["name"]].append(L["ev"][0].elapsed_time(L["ev"][1]))
+            flush_buf.zero_()
+    gemm_mean = {k: statistics.mean(v) for k, v in gemm_ms.items()}
+
+    # e2e: host activations (pinned) -> device, full path, outputs -> pinned host, every step.
+    host_a = [L["a"].cpu().pin_memory() for L in layers]
+    host_o = [torch.empty(L["out"].shape, dtype=torch.bfloat16).pin_memory() for L in layers]
+    h2d = sum(t.numel() * t.element_size() for t in host_a)
+    d2h = sum(t.numel() * t.element_size() for t in host_o)
+
+    def e2e_step():
+        for L, ha in zip(layers, host_a):
+            L["a"].copy_(ha, non_blocking=True)
+        gemm_step(False)
+        for L, ho in zip(layers, host_o):
+            ho.copy_(L["out"], non_blocking=True)
+
+    e2e_ms = timed_loop(e2e_step, max(3, min(args.steps, 50)), args.warmup)
+
+    # ---------------- decode attention over the NVFP4 cache
+    aw = synth.WORKLOADS[ATTN_WL]
+    Bq, hq, hkv, T = aw["batch"], aw["num_q_heads"], aw["num_kv_heads"], aw["context"]
+    rec = synth.kv_recipe(ATTN_WL, device=dev)
+    gk = torch.zeros(1, dtype=torch.float32, device=dev)
+    gv = torch.zeros(1, dtype=torch.float32, device=dev)
+    kv_chunks = []
+    for b in range(Bq):
+        k, v = rec.kv(T, seed=synth.seed_for(ATTN_WL, f"kv:{b}") % (1 << 62))
+        kv_chunks.append((k, v))
+    K_all = torch.stack([c[0] for c in kv_chunks]).view(-1, 128)
+    V_all = torch.stack([c[1] for c in kv_chunks]).view(-1, 128)
+    del kv_chunks
+    N.nvfp4_tensor_scale(K_all, gk)
+    N.nvfp4_tensor_scale(V_all, gv)
+    cache = N.KVCache(Bq, hkv, T, gk.item(), gv.item(), device=dev)
+    seq = torch.arange(Bq, dtype=torch.int32, device=dev).repeat_interleave(T)
+    pos = torch.arange(T, dtype=torch.int32, device=dev).repeat(Bq)
+    N.kv_append_nvfp4(cache, K_all.view(-1, hkv, 128), V_all.view(-1, hkv, 128), seq, pos)
+    del K_all, V_all, seq, pos
+    cache.seq_lens.fill_(T)
+    q = rec.queries(Bq, hq, seed=synth.seed_for(ATTN_WL, "q") % (1 << 62))
+    k_new, v_new = rec.kv(Bq, seed=synth.seed_for(ATTN_WL, "new") % (1 << 62))
+    seq_new = torch.arange(Bq, dtype=torch.int32, device=dev)
+    pos_new = torch.full((Bq,), T - 1, dtype=torch.int32, device=dev)
+    attn_ws = torch.empty(N.decode_attention_nvfp4_workspace_size(Bq, hq, T) // 4, dtype=torch.float32, device=dev)
+    attn_out = torch.empty(Bq, hq, 128, dtype=torch.bfloat16, device=dev)
+    scale = 1.0 / math.sqrt(128)
+    ev_a = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
+
+    def attn_step(record=False):
+        N.kv_append_nvfp4(cache, k_new, v_new, seq_new, pos_new)
+        if record:
+            ev_a[0].record()
+        N.decode_attention_nvfp4(cache, q, scale, attn_out, attn_ws)
+        if record:
+            ev_a[1].record()
+
+    with torch.cuda.stream(stream):
+        attn_step()
+        stream.synchronize()
+        agraph = torch.cuda.CUDAGraph()
+        n0 = N.nvfp4_launch_count()
+        with torch.cuda.graph(agraph, stream=stream):
+            attn_step()
+        attn_launches = N.nvfp4_launch_count() - n0
+    attn_step_ms = timed_loop(agraph.replay, args.steps, args.warmup)
+    attn_kernel_ms = []
+    with torch.cuda.stream(stream):
+        for _ in range(max(3, min(args.steps, 20))):
+            attn_step(True)
+            stream.synchronize()
+            attn_kernel_ms.append(ev_a[0].elapsed_time(ev_a[1]))
+    sampler.stop()
+    status = N.nvfp4_get_device_status()
+    if status != 0:
+        raise RuntimeError(f"device status {status} after the bench")
+
+    # ---------------- reduce over ranks (max time, summed work)
+    ms_step = statistics.mean(step_ms)
+    ms_e2e = statistics.mean(e2e_ms)
+    ms_attn_step = statistics.mean(attn_step_ms)
+    ms_attn_kernel = statistics.mean(attn_kernel_ms)
+    vals = torch.tensor([ms_step, ms_e2e, ms_attn_step, ms_attn_kernel], dtype=torch.float64)
+    if world > 1:
+        import torch.distributed as dist
+        dist.all_reduce(vals, op=dist.ReduceOp.MAX)
+    ms_step, ms_e2e, ms_attn_step, ms_attn_kernel = vals.tolist()
+
+    # Algorithmic bytes: codes 0.5 B/elem, scales 1/16 B/elem, bf16 output 2 B/elem, each operand once.
+    def gemm_bytes(Mm, Nn, K):
+        return Mm * K * (0.5 + 1 / 16) + Nn * K * (0.5 + 1 / 16) + Mm * Nn * 2
+    fp4_peak = peaks["bf16_tflops"] * FP4_OVER_BF16
+    dom = max(layers, key=lambda L: gemm_mean[L["name"]])
+    d_flops = 2 * M * dom["N"] * dom["K"]
+    d_bytes = gemm_bytes(M, dom["N"], dom["K"])
+    d_s = gemm_mean[dom["name"]] * 1e-3
+    t_mem, t_cmp = d_bytes / (peaks["hbm_gbs"] * 1e9), d_flops / (fp4_peak * 1e12)
+    if t_cmp >= t_mem:
+        roof = {"bound": "tensor", "achieved": d_flops / d_s / 1e12, "peak": fp4_peak, "unit": "TFLOP/s"}
+    else:
+        roof = {"bound": "hbm", "achieved": d_bytes / d_s / 1e9, "peak": peaks["hbm_gbs"], "unit": "GB/s"}
+    roof["frac"] = roof["achieved"] / roof["peak"]
+    roof["traffic"] = None
+    roof["kernel"] = f"nvfp4_gemm_kernel ({dom['name']}: {M}x{dom['N']}x{dom['K']})"
+    roof["peak_src"] = (f"{peaks['src']}: bf16 {peaks['bf16_tflops']} TFLOP/s x {FP4_OVER_BF16:g} nominal FP4/BF16"
+                        if roof["bound"] == "tensor" else f"{peaks['src']} HBM copy")
+    roof["also"] = {"tflops": d_flops / d_s / 1e12, "tflops_frac_of_fp4_peak": d_flops / d_s / 1e12 / fp4_peak,
+                    "gbs": d_bytes / d_s / 1e9, "gbs_frac": d_bytes / d_s / 1e9 / peaks["hbm_gbs"]}
+
+    kv_tokens = Bq * hkv * T
+    attn_bytes = kv_tokens * 2 * (64 + 8) + q.numel() * 2 + attn_out.numel() * 2
+    attn_gbs = attn_bytes / (ms_attn_kernel * 1e-3) / 1e9
+
+    result = {
+        "metric": METRIC,
+        "value": world * flops / (ms_step * 1e-3) / 1e12,
+        "unit": "TFLOP/s",
+        "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": ms_step,
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "e2m1 x e2m1 -> f32 accumulate -> bf16 (e4m3 block scales)",
+        "data": "synthetic (seeded; Qwen-shaped activations with outlier channels, N(0,0.02) weights)",
+        "config": {"workload": GEMM_WL, "M": M,
+                   "linears": {L["name"]: [L["N"], L["K"]] for L in layers},
+                   "step": "per linear: tensor scale + quantize activation + NVFP4 GEMM (weights pre-quantized)",
+                   "l2": "flushed between steps (256 MiB write)", "graph": "CUDA graph replay",
+                   "parallelism": f"replicas x{world}"},
+        "gemm_ms": gemm_mean,
+        "roofline": roof,
+        "e2e": {"value": world * flops / (ms_e2e * 1e-3) / 1e12, "unit": "TFLOP/s",
+                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": ms_e2e},
+        "gpu_launches": launches_per_step * args.steps,
+        "decode_attention": {
+            "workload": ATTN_WL, "value": world * attn_gbs, "unit": "GB/s",
+            "ms_attention": ms_attn_kernel, "ms_per_step": ms_attn_step,
+            "step": "append 1 token/sequence (kv_append_nvfp4) + decode_attention_nvfp4",
+            "algorithmic_bytes": attn_bytes,
+            "roofline": {"bound": "hbm", "achieved": attn_gbs, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                         "frac": attn_gbs / peaks["hbm_gbs"], "traffic": None,
+                         "kernel": "attn_partial_kernel + attn_combine_kernel (one decode_attention_nvfp4 call)"},
+            "gpu_launches": attn_launches * args.steps,
+        },
+        "clocks": sampler.summary(),
+    }
+    if rank == 0 and not args.no_cpu_baseline:
+        result["cpu_baseline"] = cpu_baseline(args.cpu_seconds)
+    return result
+
+
+# ------------------------------------------------------- oracle arm ---
+
+def oracle_sample(rows=64):
+    """One bounded oracle step: the workload's 4 linears on `rows` activation rows
+    (tensor scale + quantize the rows, dequantized fp64 GEMM); weights pre-quantized."""
+    import numpy as np
+
+    from oracle import nvfp4_oracle as O
+    from paper_2606_15682_gb300 import synth
+    w = synth.WORKLOADS[GEMM_WL]
+    prep = []
+    for name, (Nn, K) in w["linears"].items():
+        a, W = synth.linear_inputs(GEMM_WL, name)
+        Wf = W.float().numpy()
+        gw = O.tensor_scale(Wf)
+        wc, ws = O.quantize(Wf, gw)
+        prep.append((a.float().numpy(), wc, ws, gw, Nn, K))
+
+    def step():
+        fl = 0
+        for a, wc, ws, gw, Nn, K in prep:
+            ga = O.tensor_scale(a)
+            ac, as_ = O.quantize(a[:rows], ga)
+            O.linear(ac, as_, ga, wc, ws, gw)
+            fl += 2 * rows * Nn * K
+        return fl
+    return step
+
+
+def cpu_baseline(seconds=15.0):
+    step = oracle_sample()
+    t0 = time.perf_counter()
+    fl = 0
+    n = 0
+    while True:
+        fl += step()
+        n += 1
+        if time.perf_counter() - t0 > seconds:
+            break
+    dt = time.perf_counter() - t0
+    return {"value": fl / dt / 1e12, "unit": "TFLOP/s", "cores": os.cpu_count(), "kind": "oracle",
+            "sample": f"{n} oracle steps of 64 activation rows x all 4 linears of {GEMM_WL} "
+                      f"(quantize + fp64 dequantized GEMM), {dt:.1f} s"}
+
+
+def run_reference(args):
+    step = oracle_sample()
+    for _ in range(max(args.warmup, 1)):
+        step()
+    times = []
+    fl = 0
+    for _ in range(args.steps):
+        t0 = time.perf_counter()
+        fl = step()
+        times.append(time.perf_counter() - t0)
+    ms = statistics.mean(times) * 1e3
+    value = fl / (ms * 1e-3) / 1e12
+    return {"impl": "reference", "metric": METRIC, "value": value, "unit": "TFLOP/s", "n_gpus": 1,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64 (dequantized)", "data": "synthetic",
+            "config": {"workload": GEMM_WL, "sample_rows": 64},
+            "cpu_baseline": {"value": value, "unit": "TFLOP/s", "cores": os.cpu_count(), "kind": "oracle",
+                             "sample": f"64 activation rows x all 4 linears of {GEMM_WL} per step"},
+            "e2e": {"value": value, "unit": "TFLOP/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--cpu-seconds", type=float, default=15.0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    args.warmup = max(args.warmup, 3)
+    rank = int(os.environ.get("RANK", 0))
+    world = int(os.environ.get("WORLD_SIZE", 1))
+    if args.impl == "reference":
+        if rank == 0:
+            print(json.dumps(run_reference(args)))
+        return
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("gloo")
+    res = run_ours(args, rank, world)
+    if rank == 0:
+        print(json.dumps(res))
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,206 @@
+/*
+ * nvfp4.h -- C ABI of the GB300 (sm_103a) NVFP4 W4A4KV4 hot path.
+ *
+ * The library implements the data-parallel inference path behind the paper's
+ * deployment speedup: fully quantized NVFP4 execution of a transformer layer
+ * ("W4A4KV4": 4-bit weights, activations and KV cache; Sec. 2.1, Sec. 5.3,
+ * Appendix D.3).  NVFP4 is defined in Appendix A (table "Quantization
+ * configurations of MXFP4 and NVFP4"): E2M1 elements, one FP8-E4M3 scale per
+ * block of 16 elements, one FP32 scale per tensor.
+ *
+ * Conventions shared by every call
+ *   - All pointers are DEVICE pointers unless a parameter says "host".  The
+ *     caller owns every buffer; the library never allocates or frees memory.
+ *   - Every call is asynchronous on `stream` (a cudaStream_t passed as void*,
+ *     NULL = the legacy default stream) and never synchronizes, except
+ *     nvfp4_get_device_status.  Calls are safe to capture in a CUDA graph.
+ *   - bf16 tensors are row-major with a leading dimension in elements.
+ *   - Host-side argument errors return a status before anything is launched.
+ *     Faults only visible on the device (capacity overflow, a bad tensor
+ *     scale, a bounded wait that timed out) set a per-device status word that
+ *     nvfp4_get_device_status reads and clears; the kernel skips the affected
+ *     writes and returns instead of trapping.
+ *   - No C++ exceptions cross this boundary.
+ *
+ * Number formats
+ *   codes  : packed E2M1, two per byte, element 2j in bits 0-3 and element
+ *            2j+1 in bits 4-7 of byte j; a row of K elements is K/2 bytes.
+ *   scales : unsigned E4M3 (OCP E4M3FN bit layout, sign always 0), one byte per
+ *            16 consecutive elements of a row, in one of two storage orders
+ *            (nvfp4_scale_layout).
+ *   g      : FP32 tensor scale; an element dequantizes to e2m1 * e4m3 * g.
+ *
+ * Quantization recipe (the paper fixes the format, not the rounding; this is
+ * the library's reading, identical in every kernel): per block of 16,
+ *   s = amax / (6 g) in fp32; S = E4M3(s) round-to-nearest-even, saturating
+ *   at 448; if S == 0 the block's codes are signed zeros, else each element
+ *   becomes E2M1(x * (1 / (S g))) round-to-nearest-even, saturating at 6,
+ *   sign kept.
+ */
+#ifndef NVFP4_H
+#define NVFP4_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  NVFP4_OK = 0,
+  NVFP4_ERR_INVALID_ARG = 1, /* null pointer, bad enum, non-finite scale      */
+  NVFP4_ERR_SHAPE = 2,       /* unsupported or inconsistent sizes             */
+  NVFP4_ERR_ALIGN = 3,       /* pointer / leading dimension not 16-B aligned  */
+  NVFP4_ERR_UNSUPPORTED = 4, /* no sm_103a device, or device lacks a feature  */
+  NVFP4_ERR_CUDA = 5,        /* a CUDA runtime/driver call or launch failed   */
+  NVFP4_ERR_TIMEOUT = 6,     /* a bounded on-device wait gave up              */
+  NVFP4_ERR_CAPACITY = 7     /* KV append position beyond the cache capacity  */
+} nvfp4_status;
+
+typedef enum {
+  /* scales[r * (cols/16) + kb]: plain row-major [rows, cols/16].            */
+  NVFP4_SCALES_ROWMAJOR = 0,
+  /* The order the tensor core reads block scales in: rows grouped in tiles  *
+   * of 128, K-blocks in groups of 4; each (row tile, k group) owns 512      *
+   * contiguous bytes, k group fastest; inside, row r / k-block kb is at     *
+   * (r%32)*16 + ((r%128)/32)*4 + kb%4.  Needs cols % 64 == 0; the buffer    *
+   * holds ceil(rows/128)*128*(cols/16) bytes and padding rows are zeroed.   */
+  NVFP4_SCALES_MMA = 1
+} nvfp4_scale_layout;
+
+/* Bytes of a scale buffer for a [rows, cols] tensor in the given layout. */
+size_t nvfp4_scales_bytes(int64_t rows, int64_t cols, nvfp4_scale_layout layout);
+
+/*
+ * a1. FP32 tensor scale  g = amax(|x|) / (6 * 448)   (Appendix A: the FP32
+ * global scale; with it the tensor's largest element maps onto the largest
+ * NVFP4 value, E2M1 6 times E4M3 448).  An all-zero tensor gets g = 1.
+ *   x_bf16 : [rows, cols] bf16, leading dimension ld >= cols (elements).
+ *   g_dev  : one float, written on the device (never read first).
+ * Three stream operations (clear, reduce, finalize).  Errors: null pointers
+ * -> INVALID_ARG; rows or cols < 0, ld < cols -> SHAPE; x not 16-B aligned or
+ * ld % 8 != 0 -> ALIGN.  rows*cols == 0 gives g = 1.
+ */
+nvfp4_status nvfp4_tensor_scale(const void* x_bf16, int64_t rows, int64_t cols, int64_t ld,
+                                float* g_dev, void* stream);
+
+/*
+ * a2. NVFP4 quantization of a bf16 tensor along its rows (Appendix A format,
+ * recipe above).  Used for activations on the fly and, once, for weights.
+ *   x_bf16  : [rows, cols] bf16, leading dimension ld (elements, ld % 8 == 0).
+ *   g_dev   : device float, the tensor scale (from nvfp4_tensor_scale or a
+ *             static calibration value).  g <= 0 or non-finite: the kernel
+ *             writes zero codes and scales and sets INVALID_ARG on the device.
+ *   codes   : [rows, cols/2] bytes, row pitch cols/2.
+ *   scales  : nvfp4_scales_bytes(rows, cols, layout) bytes.
+ * cols % 16 == 0 (ROWMAJOR) or cols % 64 == 0 (MMA), else SHAPE.  x must be
+ * 16-B aligned, codes 8-B aligned (ALIGN).
+ */
+nvfp4_status nvfp4_quantize(const void* x_bf16, int64_t rows, int64_t cols, int64_t ld,
+                            const float* g_dev, uint8_t* codes, uint8_t* scales,
+                            nvfp4_scale_layout layout, void* stream);
+
+/*
+ * Reorder block scales between the two storage orders (both directions).
+ * src and dst must not overlap.  cols % 64 == 0.
+ */
+nvfp4_status nvfp4_scales_relayout(const uint8_t* src, uint8_t* dst, int64_t rows, int64_t cols,
+                                   nvfp4_scale_layout from, nvfp4_scale_layout to, void* stream);
+
+/*
+ * a3. Block-scaled FP4 x FP4 linear layer with bf16 output (every linear of
+ * the decoder is quantized, Appendix D.1; the 4-bit GEMM is where the
+ * paper's compute speedup comes from, Sec. 5.3):
+ *   out[m, n] = bf16_rne( (g_a * g_w) * sum_k a[m,k] * w[n,k] )
+ * with a[m,k] = e2m1 * e4m3 of A (no g) and likewise for W; the sum is
+ * accumulated in fp32 by the tensor core (tcgen05 block-scaled MMA).
+ *   a_codes  : [M, K/2] bytes (K-major), 16-B aligned.
+ *   a_scales : MMA layout for [M, K].
+ *   w_codes  : [N, K/2] bytes (K-major, i.e. the nn.Linear weight [N, K]).
+ *   w_scales : MMA layout for [N, K].
+ *   g_a,g_w  : device floats.
+ *   out_bf16 : [M, N] bf16 with leading dimension ldo >= N (elements).
+ * Requires K % 256 == 0, N % 16 == 0, ldo % 8 == 0, M,N,K > 0 (SHAPE),
+ * pointers 16-B aligned (ALIGN).
+ */
+nvfp4_status nvfp4_linear(const uint8_t* a_codes, const uint8_t* a_scales, const float* g_a,
+                          const uint8_t* w_codes, const uint8_t* w_scales, const float* g_w,
+                          int64_t M, int64_t N, int64_t K, void* out_bf16, int64_t ldo,
+                          void* stream);
+
+/*
+ * NVFP4 KV cache (W4A4KV4; the B200 deployment uses a native 4-bit KV cache,
+ * Appendix D.3).  One row per (sequence, KV head, position); the 16-element
+ * blocks run along head_dim, so an appended token never touches older rows.
+ *   k_codes, v_codes   : [batch, num_kv_heads, capacity, head_dim/2] bytes
+ *   k_scales, v_scales : [batch, num_kv_heads, capacity, head_dim/16] bytes
+ *   seq_lens           : device int32 [batch], valid tokens per sequence
+ *                        (maintained by the caller; read by attention).
+ *   k_gscale, v_gscale : static per-layer FP32 tensor scales (an append-only
+ *                        cache cannot re-scale rows it already holds).
+ * head_dim must be 128.  Buffers 16-B aligned.
+ */
+typedef struct {
+  uint8_t* k_codes;
+  uint8_t* k_scales;
+  uint8_t* v_codes;
+  uint8_t* v_scales;
+  const int32_t* seq_lens;
+  int32_t batch;
+  int32_t num_kv_heads;
+  int32_t head_dim;
+  int32_t capacity;
+  float k_gscale;
+  float v_gscale;
+} nvfp4_kv_cache;
+
+/*
+ * a4. Quantize n_new K/V rows and append them to the cache.  With k_shift the
+ * Q-FIT post-RoPE shift is applied first, K~ = R(K) - m (Eq. 2; the paper
+ * applies it after an unfused RoPE, Appendix D.3), in fp32.
+ *   k_bf16, v_bf16 : [n_new, num_kv_heads, head_dim] bf16 (K already rotated).
+ *   seq_idx, pos   : device int32 [n_new]: destination sequence and position.
+ *   k_shift        : device float [num_kv_heads, head_dim] or NULL.
+ * A row whose seq_idx is outside [0, batch) or pos outside [0, capacity) is
+ * skipped and sets CAPACITY on the device.
+ */
+nvfp4_status kv_append_nvfp4(const nvfp4_kv_cache* cache, const void* k_bf16, const void* v_bf16,
+                             const int32_t* seq_idx, const int32_t* pos, int64_t n_new,
+                             const float* k_shift, void* stream);
+
+/*
+ * a5. Decode attention straight from the NVFP4 cache (Sec. 2.1):
+ *   out[b, h] = softmax(softmax_scale * q[b,h] . K_hat[b,kv,t]) V_hat[b,kv,t],
+ *   t < seq_lens[b], kv = h / (num_q_heads / num_kv_heads) (contiguous
+ *   grouped-query replication, as in Algorithm 1's Replicate step).
+ * Softmax in fp32; K/V are dequantized in registers and multiplied on the
+ * tensor cores.  Split-KV partials go to `workspace`, then a combine kernel
+ * writes out.
+ *   q_bf16   : [batch, num_q_heads, head_dim] bf16.
+ *   out_bf16 : [batch, num_q_heads, head_dim] bf16.
+ *   workspace: at least decode_attention_nvfp4_workspace_size(...) bytes, 16-B
+ *              aligned; contents on entry are ignored.
+ * num_q_heads % num_kv_heads == 0 and num_q_heads/num_kv_heads <= 8 (SHAPE).
+ * A sequence with seq_lens[b] == 0 gets zeros; seq_lens[b] > capacity sets
+ * CAPACITY on the device and is clamped to capacity.
+ */
+size_t decode_attention_nvfp4_workspace_size(int32_t batch, int32_t num_q_heads, int32_t capacity);
+nvfp4_status decode_attention_nvfp4(const nvfp4_kv_cache* cache, const void* q_bf16,
+                                    int32_t num_q_heads, float softmax_scale, void* out_bf16,
+                                    void* workspace, size_t workspace_bytes, void* stream);
+
+/* Synchronize `stream`, copy the device status word of the current device to
+ * *status_host (an nvfp4_status value) and clear it. */
+nvfp4_status nvfp4_get_device_status(int32_t* status_host, void* stream);
+
+/* Static, human-readable name of a status. */
+const char* nvfp4_status_string(nvfp4_status s);
+
+/* Number of kernels this library has launched in this process (host counter). */
+uint64_t nvfp4_launch_count(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* NVFP4_H */

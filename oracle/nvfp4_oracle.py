@@ -236,31 +236,29 @@ def mma_scale_bytes(rows, cols):
     return ((rows + 127) // 128) * 128 * (cols // BLOCK)
 
 
+def _mma_offsets(rows, kblocks):
+    """Byte offset of every (row, k-block) scale in the MMA layout, [rows, kblocks]."""
+    kgroups = kblocks // 4
+    r = np.arange(rows, dtype=np.int64)[:, None]
+    kb = np.arange(kblocks, dtype=np.int64)[None, :]
+    return ((r // 128) * kgroups + kb // 4) * 512 + (r % 32) * 16 + ((r % 128) // 32) * 4 + kb % 4
+
+
 def scales_to_mma(scales):
-    """Row-major [rows, cols/16] scales -> flat MMA-layout byte array."""
+    """Row-major [rows, cols/16] scales -> flat MMA-layout byte array (padding rows zero)."""
     scales = np.asarray(scales, dtype=np.uint8)
     rows, kblocks = scales.shape
     if kblocks % 4:
         raise ValueError("cols must be a multiple of 64 for the MMA layout")
-    kgroups = kblocks // 4
     out = np.zeros(mma_scale_bytes(rows, kblocks * BLOCK), dtype=np.uint8)
-    for r in range(rows):
-        for kb in range(kblocks):
-            atom = (r // 128) * kgroups + kb // 4
-            off = atom * 512 + (r % 32) * 16 + ((r % 128) // 32) * 4 + kb % 4
-            out[off] = scales[r, kb]
+    out[_mma_offsets(rows, kblocks)] = scales
     return out
 
 
 def scales_from_mma(flat, rows, cols):
     """Inverse of ``scales_to_mma`` (drops padding rows)."""
     flat = np.asarray(flat, dtype=np.uint8).reshape(-1)
-    kblocks = cols // BLOCK
-    kgroups = kblocks // 4
-    r = np.arange(rows)[:, None]
-    kb = np.arange(kblocks)[None, :]
-    off = ((r // 128) * kgroups + kb // 4) * 512 + (r % 32) * 16 + ((r % 128) // 32) * 4 + kb % 4
-    return flat[off]
+    return flat[_mma_offsets(rows, cols // BLOCK)]
 
 
 # ---------------------------------------------------------------------------

@@ -1,0 +1,241 @@
+// a1 tensor scale and a2 NVFP4 quantization (Appendix A format).
+//
+// Both kernels stream bf16 with 128-bit loads, one 8-element chunk per lane
+// per step; a warp covers 256 contiguous elements, so every load and every
+// code store of a warp is one contiguous span.  They are HBM-bound: the
+// quantizer moves 2 B in and 0.5625 B out per element.
+#include <cfloat>
+
+#include "common.cuh"
+#include "nvfp4_quant.cuh"
+
+namespace nvfp4 {
+namespace {
+
+constexpr int kThreads = 256;
+constexpr int kUnroll = 4;
+
+// Chunk c (8 elements) of a [rows, cols] tensor with leading dimension ld.
+struct ChunkMap {
+  FastDiv cpr;   // chunks per row
+  uint32_t total;
+  int64_t ld;
+  bool dense;    // ld == cols: chunk c starts at element 8c
+  __device__ __forceinline__ int64_t elem(uint32_t c, uint32_t* row, uint32_t* chunk_in_row) const {
+    const uint32_t r = cpr.div(c);
+    *row = r;
+    *chunk_in_row = c - r * cpr.d;
+    return dense ? static_cast<int64_t>(c) * 8 : static_cast<int64_t>(r) * ld + static_cast<int64_t>(*chunk_in_row) * 8;
+  }
+};
+
+__global__ void __launch_bounds__(kThreads) amax_kernel(const uint16_t* __restrict__ x, ChunkMap map,
+                                                        uint32_t* __restrict__ amax_bits) {
+  const uint32_t stride = gridDim.x * blockDim.x;
+  uint32_t m = 0;
+  for (uint32_t c0 = blockIdx.x * blockDim.x; c0 < map.total; c0 += stride * kUnroll) {
+    uint4 v[kUnroll];
+#pragma unroll
+    for (int u = 0; u < kUnroll; ++u) {
+      const uint32_t c = c0 + u * stride + threadIdx.x;
+      uint32_t r, j;
+      v[u] = c < map.total ? __ldg(reinterpret_cast<const uint4*>(x + map.elem(c, &r, &j))) : make_uint4(0, 0, 0, 0);
+    }
+#pragma unroll
+    for (int u = 0; u < kUnroll; ++u) m = max(m, amax_bits_bf16x8(v[u]));
+  }
+  m = __reduce_max_sync(0xffffffffu, m);
+  __shared__ uint32_t warp_max[kThreads / 32];
+  if ((threadIdx.x & 31) == 0) warp_max[threadIdx.x >> 5] = m;
+  __syncthreads();
+  if (threadIdx.x < 32) {
+    m = threadIdx.x < kThreads / 32 ? warp_max[threadIdx.x] : 0u;
+    m = __reduce_max_sync(0xffffffffu, m);
+    if (threadIdx.x == 0 && m) atomicMax(amax_bits, m);
+  }
+}
+
+// g = amax / (6 * 448) in fp32, or 1 for an all-zero tensor.
+__global__ void tensor_scale_finalize(float* g) {
+  const uint32_t bits = *reinterpret_cast<uint32_t*>(g);
+  const float amax = __uint_as_float(bits << 16);
+  *g = amax > 0.0f ? __fdiv_rn(amax, 2688.0f) : 1.0f;
+}
+
+template <bool kMMA>
+__global__ void __launch_bounds__(kThreads) quantize_kernel(const uint16_t* __restrict__ x, ChunkMap map,
+                                                            uint32_t rows, uint32_t kblocks,
+                                                            const float* __restrict__ g_ptr,
+                                                            uint32_t* __restrict__ codes,
+                                                            uint8_t* __restrict__ scales, int* status) {
+  const float g_in = *g_ptr;
+  const bool g_ok = g_in > 0.0f && g_in <= FLT_MAX;
+  if (!g_ok && blockIdx.x == 0 && threadIdx.x == 0) set_status(status, NVFP4_ERR_INVALID_ARG);
+  const float g = g_ok ? g_in : 1.0f;
+  const float six_g = __fmul_rn(6.0f, g);
+  const uint32_t lane = threadIdx.x & 31;
+  const uint32_t stride = gridDim.x * blockDim.x;
+  const uint32_t kgroups = kblocks >> 2;
+
+  // c0 is warp-uniform, so every lane runs every iteration (the amax shuffle
+  // needs the whole warp); lanes past the end only skip their memory ops.
+  for (uint32_t c0 = blockIdx.x * blockDim.x + (threadIdx.x & ~31u); c0 < map.total; c0 += stride * kUnroll) {
+    uint4 v[kUnroll];
+    int64_t off[kUnroll];
+    uint32_t row[kUnroll], chk[kUnroll];
+#pragma unroll
+    for (int u = 0; u < kUnroll; ++u) {
+      const uint32_t c = c0 + u * stride + lane;
+      off[u] = c < map.total ? map.elem(c, &row[u], &chk[u]) : 0;
+      v[u] = c < map.total ? __ldg(reinterpret_cast<const uint4*>(x + off[u])) : make_uint4(0, 0, 0, 0);
+    }
+#pragma unroll
+    for (int u = 0; u < kUnroll; ++u) {
+      const uint32_t c = c0 + u * stride + lane;
+      float xf[8];
+      unpack_bf16x8(v[u], xf);
+      const float amax_own = __uint_as_float(amax_bits_bf16x8(v[u]) << 16);
+      uint32_t sc;
+      uint32_t packed = quantize8_pair(xf, amax_own, g, six_g, &sc);
+      if (!g_ok) { packed = 0; sc = 0; }
+      if (c < map.total) {
+        codes[c] = packed;  // codes are dense: row pitch cols/2 bytes = 4 bytes per chunk
+        if ((lane & 1) == 0) {
+          const uint32_t kb = chk[u] >> 1;
+          const uint64_t so = kMMA ? mma_scale_offset(row[u], kb, kgroups)
+                                   : static_cast<uint64_t>(row[u]) * kblocks + kb;
+          scales[so] = static_cast<uint8_t>(sc);
+        }
+      }
+    }
+  }
+  if (kMMA) {
+    // Zero the scales of the padding rows up to the next multiple of 128.
+    const uint32_t padded = (rows + 127u) & ~127u;
+    const uint32_t pad = (padded - rows) * kblocks;
+    for (uint32_t i = blockIdx.x * blockDim.x + threadIdx.x; i < pad; i += stride) {
+      const uint32_t r = rows + i / kblocks, kb = i % kblocks;
+      scales[mma_scale_offset(r, kb, kgroups)] = 0;
+    }
+  }
+}
+
+template <bool kToMMA>
+__global__ void relayout_kernel(const uint8_t* __restrict__ src, uint8_t* __restrict__ dst, uint32_t rows,
+                                uint32_t kblocks) {
+  const uint32_t kgroups = kblocks >> 2;
+  const uint32_t padded = (rows + 127u) & ~127u;
+  const uint32_t n = padded * kblocks;
+  for (uint32_t i = blockIdx.x * blockDim.x + threadIdx.x; i < n; i += gridDim.x * blockDim.x) {
+    const uint32_t r = i / kblocks, kb = i % kblocks;
+    const uint64_t m = mma_scale_offset(r, kb, kgroups);
+    if (kToMMA) {
+      dst[m] = r < rows ? src[i] : 0;
+    } else if (r < rows) {
+      dst[i] = src[m];
+    }
+  }
+}
+
+int grid_for(uint64_t work_items, int threads) {
+  const uint64_t want = (work_items + threads - 1) / threads;
+  const uint64_t cap = static_cast<uint64_t>(sm_count()) * 8;
+  return static_cast<int>(want < 1 ? 1 : (want > cap ? cap : want));
+}
+
+nvfp4_status check_bf16_matrix(const void* x, int64_t rows, int64_t cols, int64_t ld, int64_t col_mult) {
+  if (!x) return NVFP4_ERR_INVALID_ARG;
+  if (rows < 0 || cols < 0 || ld < cols || cols % col_mult) return NVFP4_ERR_SHAPE;
+  if (rows * (cols / 8) >= (1ll << 32) || rows >= (1ll << 31)) return NVFP4_ERR_SHAPE;
+  if (!aligned(x, 16) || ld % 8) return NVFP4_ERR_ALIGN;
+  return NVFP4_OK;
+}
+
+ChunkMap make_map(int64_t rows, int64_t cols, int64_t ld) {
+  ChunkMap m;
+  m.cpr = FastDiv(static_cast<uint32_t>(cols / 8 > 0 ? cols / 8 : 1));
+  m.total = static_cast<uint32_t>(rows * (cols / 8));
+  m.ld = ld;
+  m.dense = (ld == cols);
+  return m;
+}
+
+}  // namespace
+}  // namespace nvfp4
+
+using namespace nvfp4;
+
+NVFP4_API size_t nvfp4_scales_bytes(int64_t rows, int64_t cols, nvfp4_scale_layout layout) {
+  if (rows < 0 || cols < 0) return 0;
+  const int64_t r = layout == NVFP4_SCALES_MMA ? ((rows + 127) / 128) * 128 : rows;
+  return static_cast<size_t>(r * (cols / 16));
+}
+
+NVFP4_API nvfp4_status nvfp4_tensor_scale(const void* x_bf16, int64_t rows, int64_t cols, int64_t ld,
+                                          float* g_dev, void* stream) {
+  if (!g_dev) return NVFP4_ERR_INVALID_ARG;
+  nvfp4_status st = check_bf16_matrix(x_bf16, rows, cols, ld, 8);
+  if (st != NVFP4_OK) return st;
+  if (!aligned(g_dev, 4)) return NVFP4_ERR_ALIGN;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (cudaMemsetAsync(g_dev, 0, sizeof(float), s) != cudaSuccess) return NVFP4_ERR_CUDA;
+  const ChunkMap map = make_map(rows, cols, ld);
+  if (map.total) {
+    amax_kernel<<<grid_for(map.total, kThreads * kUnroll), kThreads, 0, s>>>(
+        static_cast<const uint16_t*>(x_bf16), map, reinterpret_cast<uint32_t*>(g_dev));
+    count_launches(1);
+  }
+  tensor_scale_finalize<<<1, 1, 0, s>>>(g_dev);
+  count_launches(1);
+  return launch_status();
+}
+
+NVFP4_API nvfp4_status nvfp4_quantize(const void* x_bf16, int64_t rows, int64_t cols, int64_t ld,
+                                      const float* g_dev, uint8_t* codes, uint8_t* scales,
+                                      nvfp4_scale_layout layout, void* stream) {
+  if (!g_dev || !codes || !scales) return NVFP4_ERR_INVALID_ARG;
+  if (layout != NVFP4_SCALES_ROWMAJOR && layout != NVFP4_SCALES_MMA) return NVFP4_ERR_INVALID_ARG;
+  nvfp4_status st = check_bf16_matrix(x_bf16, rows, cols, ld, layout == NVFP4_SCALES_MMA ? 64 : 16);
+  if (st != NVFP4_OK) return st;
+  if (!aligned(codes, 8) || !aligned(g_dev, 4)) return NVFP4_ERR_ALIGN;
+  if (rows == 0 || cols == 0) return NVFP4_OK;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const ChunkMap map = make_map(rows, cols, ld);
+  const uint32_t kblocks = static_cast<uint32_t>(cols / 16);
+  const int grid = grid_for(map.total, kThreads * kUnroll);
+  if (layout == NVFP4_SCALES_MMA) {
+    quantize_kernel<true><<<grid, kThreads, 0, s>>>(static_cast<const uint16_t*>(x_bf16), map,
+                                                    static_cast<uint32_t>(rows), kblocks, g_dev,
+                                                    reinterpret_cast<uint32_t*>(codes), scales, status_word_dev());
+  } else {
+    quantize_kernel<false><<<grid, kThreads, 0, s>>>(static_cast<const uint16_t*>(x_bf16), map,
+                                                     static_cast<uint32_t>(rows), kblocks, g_dev,
+                                                     reinterpret_cast<uint32_t*>(codes), scales, status_word_dev());
+  }
+  count_launches(1);
+  return launch_status();
+}
+
+NVFP4_API nvfp4_status nvfp4_scales_relayout(const uint8_t* src, uint8_t* dst, int64_t rows, int64_t cols,
+                                             nvfp4_scale_layout from, nvfp4_scale_layout to, void* stream) {
+  if (!src || !dst) return NVFP4_ERR_INVALID_ARG;
+  if ((from != NVFP4_SCALES_ROWMAJOR && from != NVFP4_SCALES_MMA) ||
+      (to != NVFP4_SCALES_ROWMAJOR && to != NVFP4_SCALES_MMA))
+    return NVFP4_ERR_INVALID_ARG;
+  if (rows < 0 || cols < 0 || cols % 64 || rows >= (1ll << 24)) return NVFP4_ERR_SHAPE;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const size_t bytes = nvfp4_scales_bytes(rows, cols, from);
+  if (from == to) {
+    if (bytes && cudaMemcpyAsync(dst, src, bytes, cudaMemcpyDeviceToDevice, s) != cudaSuccess) return NVFP4_ERR_CUDA;
+    return NVFP4_OK;
+  }
+  if (rows == 0 || cols == 0) return NVFP4_OK;
+  const uint32_t kblocks = static_cast<uint32_t>(cols / 16);
+  const uint64_t n = static_cast<uint64_t>((rows + 127) / 128 * 128) * kblocks;
+  if (to == NVFP4_SCALES_MMA)
+    relayout_kernel<true><<<grid_for(n, 256), 256, 0, s>>>(src, dst, static_cast<uint32_t>(rows), kblocks);
+  else
+    relayout_kernel<false><<<grid_for(n, 256), 256, 0, s>>>(src, dst, static_cast<uint32_t>(rows), kblocks);
+  count_launches(1);
+  return launch_status();
+}

@@ -1,0 +1,168 @@
+"""Thin ctypes binding of libnvfp4.so (include/nvfp4.h).
+
+Argument marshalling only: every function takes torch CUDA tensors (or plain
+integers for scalars), passes their device pointers and the current CUDA
+stream to the C entry point of the same name, and raises ``NVFP4Error`` on a
+non-OK status.  No computation happens here, and there is no CPU fallback:
+if the library is missing, importing this module fails.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import torch
+
+_PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_PKG, "_build", "libnvfp4.so")
+
+SCALES_ROWMAJOR = 0
+SCALES_MMA = 1
+
+STATUS = {0: "ok", 1: "invalid argument", 2: "shape", 3: "alignment", 4: "unsupported", 5: "cuda",
+          6: "timeout", 7: "capacity"}
+
+
+class NVFP4Error(RuntimeError):
+    def __init__(self, fn, code):
+        self.code = code
+        super().__init__(f"{fn} failed: {STATUS.get(code, code)} ({code})")
+
+
+if not os.path.exists(LIB_PATH):
+    raise ImportError(f"{LIB_PATH} is missing: run paper_2606_15682_gb300.build.build() first")
+_lib = ctypes.CDLL(LIB_PATH)
+
+_p, _i64, _i32, _f32, _sz = ctypes.c_void_p, ctypes.c_int64, ctypes.c_int32, ctypes.c_float, ctypes.c_size_t
+
+
+class KVCacheStruct(ctypes.Structure):
+    _fields_ = [("k_codes", _p), ("k_scales", _p), ("v_codes", _p), ("v_scales", _p), ("seq_lens", _p),
+                ("batch", _i32), ("num_kv_heads", _i32), ("head_dim", _i32), ("capacity", _i32),
+                ("k_gscale", _f32), ("v_gscale", _f32)]
+
+
+def _sig(name, args, res=ctypes.c_int):
+    f = getattr(_lib, name)
+    f.argtypes = args
+    f.restype = res
+    return f
+
+
+_tensor_scale = _sig("nvfp4_tensor_scale", [_p, _i64, _i64, _i64, _p, _p])
+_quantize = _sig("nvfp4_quantize", [_p, _i64, _i64, _i64, _p, _p, _p, ctypes.c_int, _p])
+_relayout = _sig("nvfp4_scales_relayout", [_p, _p, _i64, _i64, ctypes.c_int, ctypes.c_int, _p])
+_linear = _sig("nvfp4_linear", [_p, _p, _p, _p, _p, _p, _i64, _i64, _i64, _p, _i64, _p])
+_kv_append = _sig("kv_append_nvfp4", [ctypes.POINTER(KVCacheStruct), _p, _p, _p, _p, _i64, _p, _p])
+_attn_ws = _sig("decode_attention_nvfp4_workspace_size", [_i32, _i32, _i32], _sz)
+_attn = _sig("decode_attention_nvfp4", [ctypes.POINTER(KVCacheStruct), _p, _i32, _f32, _p, _p, _sz, _p])
+_get_status = _sig("nvfp4_get_device_status", [ctypes.POINTER(_i32), _p])
+_status_string = _sig("nvfp4_status_string", [ctypes.c_int], ctypes.c_char_p)
+_launch_count = _sig("nvfp4_launch_count", [], ctypes.c_uint64)
+_scales_bytes = _sig("nvfp4_scales_bytes", [_i64, _i64, ctypes.c_int], _sz)
+
+
+def _stream(stream):
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return ctypes.c_void_p(stream.cuda_stream if hasattr(stream, "cuda_stream") else int(stream))
+
+
+def _ptr(t):
+    if t is None:
+        return None
+    return ctypes.c_void_p(t.data_ptr())
+
+
+def _check(fn, code):
+    if code != 0:
+        raise NVFP4Error(fn, code)
+
+
+def _ld(x):
+    if x.dim() != 2 or x.stride(1) != 1:
+        raise ValueError("expected a 2-D row-major tensor")
+    return x.stride(0)
+
+
+# ----------------------------------------------------------------- calls ---
+
+def nvfp4_scales_bytes(rows, cols, layout):
+    return int(_scales_bytes(rows, cols, layout))
+
+
+def nvfp4_tensor_scale(x, g, stream=None):
+    """g[0] <- amax(|x|) / (6*448) (device)."""
+    _check("nvfp4_tensor_scale", _tensor_scale(_ptr(x), x.shape[0], x.shape[1], _ld(x), _ptr(g), _stream(stream)))
+
+
+def nvfp4_quantize(x, g, codes, scales, layout=SCALES_MMA, stream=None):
+    _check("nvfp4_quantize", _quantize(_ptr(x), x.shape[0], x.shape[1], _ld(x), _ptr(g), _ptr(codes), _ptr(scales),
+                                       layout, _stream(stream)))
+
+
+def nvfp4_scales_relayout(src, dst, rows, cols, from_layout, to_layout, stream=None):
+    _check("nvfp4_scales_relayout", _relayout(_ptr(src), _ptr(dst), rows, cols, from_layout, to_layout,
+                                              _stream(stream)))
+
+
+def nvfp4_linear(a_codes, a_scales, g_a, w_codes, w_scales, g_w, out, M, N, K, ldo=None, stream=None):
+    _check("nvfp4_linear", _linear(_ptr(a_codes), _ptr(a_scales), _ptr(g_a), _ptr(w_codes), _ptr(w_scales),
+                                   _ptr(g_w), M, N, K, _ptr(out), N if ldo is None else ldo, _stream(stream)))
+
+
+def kv_append_nvfp4(cache, k, v, seq_idx, pos, k_shift=None, stream=None):
+    s = cache.struct()
+    _check("kv_append_nvfp4", _kv_append(ctypes.byref(s), _ptr(k), _ptr(v), _ptr(seq_idx), _ptr(pos), k.shape[0],
+                                         _ptr(k_shift), _stream(stream)))
+
+
+def decode_attention_nvfp4_workspace_size(batch, num_q_heads, capacity):
+    return int(_attn_ws(batch, num_q_heads, capacity))
+
+
+def decode_attention_nvfp4(cache, q, softmax_scale, out, workspace, stream=None):
+    s = cache.struct()
+    _check("decode_attention_nvfp4", _attn(ctypes.byref(s), _ptr(q), q.shape[1], softmax_scale, _ptr(out),
+                                           _ptr(workspace), workspace.numel() * workspace.element_size(),
+                                           _stream(stream)))
+
+
+def nvfp4_get_device_status(stream=None):
+    v = _i32(0)
+    _check("nvfp4_get_device_status", _get_status(ctypes.byref(v), _stream(stream)))
+    return int(v.value)
+
+
+def nvfp4_status_string(code):
+    return _status_string(code).decode()
+
+
+def nvfp4_launch_count():
+    return int(_launch_count())
+
+
+# ------------------------------------------------------------- KV cache ---
+
+class KVCache:
+    """Caller-owned NVFP4 KV cache buffers (layout of include/nvfp4.h)."""
+
+    def __init__(self, batch, num_kv_heads, capacity, k_gscale, v_gscale, head_dim=128, device="cuda"):
+        self.batch, self.num_kv_heads, self.capacity, self.head_dim = batch, num_kv_heads, capacity, head_dim
+        self.k_gscale, self.v_gscale = float(k_gscale), float(v_gscale)
+        shape = (batch, num_kv_heads, capacity)
+        self.k_codes = torch.zeros(shape + (head_dim // 2,), dtype=torch.uint8, device=device)
+        self.v_codes = torch.zeros_like(self.k_codes)
+        self.k_scales = torch.zeros(shape + (head_dim // 16,), dtype=torch.uint8, device=device)
+        self.v_scales = torch.zeros_like(self.k_scales)
+        self.seq_lens = torch.zeros(batch, dtype=torch.int32, device=device)
+
+    def struct(self):
+        return KVCacheStruct(self.k_codes.data_ptr(), self.k_scales.data_ptr(), self.v_codes.data_ptr(),
+                             self.v_scales.data_ptr(), self.seq_lens.data_ptr(), self.batch, self.num_kv_heads,
+                             self.head_dim, self.capacity, self.k_gscale, self.v_gscale)
+
+
+EXPORTED = ["nvfp4_scales_bytes", "nvfp4_tensor_scale", "nvfp4_quantize", "nvfp4_scales_relayout", "nvfp4_linear",
+            "kv_append_nvfp4", "decode_attention_nvfp4_workspace_size", "decode_attention_nvfp4",
+            "nvfp4_get_device_status", "nvfp4_status_string", "nvfp4_launch_count"]

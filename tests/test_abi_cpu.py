@@ -1,0 +1,77 @@
+"""Host-only checks of the C ABI: the library builds, loads, exports every
+function include/nvfp4.h declares, and rejects bad arguments before any
+launch.  No call here reaches a GPU."""
+import ctypes
+
+import pytest
+
+from _util import header_functions, lib
+
+
+def test_header_declares_the_hot_path_calls():
+    names = header_functions()
+    for n in ["nvfp4_tensor_scale", "nvfp4_quantize", "nvfp4_linear", "kv_append_nvfp4",
+              "decode_attention_nvfp4", "decode_attention_nvfp4_workspace_size", "nvfp4_get_device_status"]:
+        assert n in names
+
+
+def test_library_exports_every_declared_symbol():
+    N = lib()
+    so = ctypes.CDLL(N.LIB_PATH)
+    for name in header_functions():
+        assert hasattr(so, name), name
+    assert sorted(N.EXPORTED) == header_functions()
+
+
+def test_status_strings_and_sizes():
+    N = lib()
+    assert N.nvfp4_status_string(0) == "ok"
+    assert "capacity" in N.nvfp4_status_string(7)
+    assert N.nvfp4_scales_bytes(130, 256, N.SCALES_ROWMAJOR) == 130 * 16
+    assert N.nvfp4_scales_bytes(130, 256, N.SCALES_MMA) == 256 * 16
+    assert N.decode_attention_nvfp4_workspace_size(64, 40, 16384) > 0
+    assert N.decode_attention_nvfp4_workspace_size(0, 40, 16384) == 0
+
+
+def test_argument_validation_before_launch():
+    N = lib()
+    L = N._lib
+    p = ctypes.c_void_p(0x10000)      # aligned, never dereferenced: validation fails first
+    odd = ctypes.c_void_p(0x10001)
+    s = ctypes.c_void_p(0)
+    # null pointers
+    assert L.nvfp4_linear(None, p, p, p, p, p, 128, 128, 256, p, 128, s) == 1
+    assert L.nvfp4_tensor_scale(p, 4, 16, 16, None, s) == 1
+    # shapes: K not a multiple of 256, N not a multiple of 16, ldo < N
+    assert L.nvfp4_linear(p, p, p, p, p, p, 128, 128, 192, p, 128, s) == 2
+    assert L.nvfp4_linear(p, p, p, p, p, p, 128, 120, 256, p, 128, s) == 2
+    assert L.nvfp4_linear(p, p, p, p, p, p, 128, 128, 256, p, 64, s) == 2
+    assert L.nvfp4_quantize(p, 4, 40, 40, p, p, p, 0, s) == 2            # cols % 16
+    assert L.nvfp4_quantize(p, 4, 32, 32, p, p, p, 1, s) == 2            # MMA layout needs cols % 64
+    assert L.nvfp4_quantize(p, 4, 64, 64, p, p, p, 7, s) == 1            # bad layout enum
+    # alignment
+    assert L.nvfp4_linear(odd, p, p, p, p, p, 128, 128, 256, p, 128, s) == 3
+    assert L.nvfp4_quantize(odd, 4, 64, 64, p, p, p, 1, s) == 3
+    assert L.nvfp4_quantize(p, 4, 64, 68, p, p, p, 1, s) == 3            # ld % 8
+
+
+def test_kv_and_attention_validation():
+    N = lib()
+    import torch  # noqa: F401  (struct only; no device memory)
+
+    def cache(**kw):
+        c = N.KVCacheStruct(0x10000, 0x10000, 0x10000, 0x10000, 0x10000, 2, 2, 128, 64, 1.0, 1.0)
+        for k, v in kw.items():
+            setattr(c, k, v)
+        return c
+    L = N._lib
+    p = ctypes.c_void_p(0x10000)
+    s = ctypes.c_void_p(0)
+    assert L.kv_append_nvfp4(ctypes.byref(cache(head_dim=64)), p, p, p, p, 1, None, s) == 2
+    assert L.kv_append_nvfp4(ctypes.byref(cache(k_gscale=0.0)), p, p, p, p, 1, None, s) == 1
+    assert L.kv_append_nvfp4(ctypes.byref(cache()), None, p, p, p, 1, None, s) == 1
+    ws = N.decode_attention_nvfp4_workspace_size(2, 4, 64)
+    assert L.decode_attention_nvfp4(ctypes.byref(cache()), p, 3, ctypes.c_float(0.1), p, p, ws, s) == 2   # 3 % 2
+    assert L.decode_attention_nvfp4(ctypes.byref(cache()), p, 18, ctypes.c_float(0.1), p, p, 1 << 30, s) == 2  # group 9
+    assert L.decode_attention_nvfp4(ctypes.byref(cache()), p, 4, ctypes.c_float(0.1), p, p, ws - 16, s) == 2
+    assert L.decode_attention_nvfp4(ctypes.byref(cache()), p, 4, ctypes.c_float(-1.0), p, p, ws, s) == 1

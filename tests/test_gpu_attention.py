@@ -1,0 +1,189 @@
+"""GPU parity of a4 (KV quantize + append, optional Q-FIT shift) and a5 (decode
+attention over the NVFP4 cache) against the oracle."""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+from _util import assert_close, f32, lib, u8
+from oracle import nvfp4_oracle as O
+from paper_2606_15682_gb300 import synth
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def N():
+    assert torch.cuda.is_available(), "GPU tests need a CUDA device"
+    return lib()
+
+
+def oracle_cache(B, hkv, cap):
+    kc = np.zeros((B, hkv, cap, 64), np.uint8); ks = np.zeros((B, hkv, cap, 8), np.uint8)
+    return kc, ks, kc.copy(), ks.copy()
+
+
+def gscale(N, x):
+    g = torch.empty(1, dtype=torch.float32, device="cuda")
+    N.nvfp4_tensor_scale(x.reshape(-1, x.shape[-1]), g)
+    return g.item()
+
+
+def fill(N, cache, k, v, seq, pos, shift=None):
+    N.kv_append_nvfp4(cache, k.cuda(), v.cuda(), torch.as_tensor(seq, dtype=torch.int32, device="cuda"),
+                      torch.as_tensor(pos, dtype=torch.int32, device="cuda"),
+                      None if shift is None else shift.cuda())
+
+
+@pytest.mark.parametrize("shifted", [False, True])
+def test_kv_append_bit_exact(N, shifted):
+    B, hkv, cap, n = 3, 2, 40, 50
+    rec = synth.KVRecipe(hkv, seed=77)
+    k, v = rec.kv(n, seed=5)
+    shift = (f32(k).reshape(n, hkv, 128).mean(axis=0) * 0.7).astype(np.float32) if shifted else None
+    kf = f32(k) - (shift if shifted else 0)
+    gk, gv = O.tensor_scale(kf.astype(np.float32)), O.tensor_scale(f32(v))
+    cache = N.KVCache(B, hkv, cap, gk, gv)
+    rng = np.random.default_rng(3)
+    seq = rng.integers(0, B, n); pos = rng.permutation(B * cap)[:n] % cap
+    # unique (seq, pos) pairs so the write order does not matter
+    pairs = {}
+    for i in range(n):
+        pairs[(seq[i], pos[i])] = i
+    keep = np.array(sorted(pairs.values()))
+    k, v, seq, pos = k[keep], v[keep], seq[keep], pos[keep]
+    fill(N, cache, k, v, seq, pos, None if shift is None else torch.from_numpy(shift))
+    torch.cuda.synchronize()
+    assert N.nvfp4_get_device_status() == 0
+    rkc, rks, rvc, rvs = oracle_cache(B, hkv, cap)
+    O.kv_append(rkc, rks, rvc, rvs, f32(k), f32(v), seq, pos, np.float32(gk), np.float32(gv), k_shift=shift)
+    assert np.array_equal(u8(cache.k_codes), rkc) and np.array_equal(u8(cache.k_scales), rks)
+    assert np.array_equal(u8(cache.v_codes), rvc) and np.array_equal(u8(cache.v_scales), rvs)
+
+
+def test_kv_append_out_of_range_sets_capacity_and_skips(N):
+    B, hkv, cap = 2, 1, 8
+    k = torch.randn(3, hkv, 128).to(torch.bfloat16)
+    cache = N.KVCache(B, hkv, cap, 0.01, 0.01)
+    N.nvfp4_get_device_status()
+    fill(N, cache, k, k, [0, 1, 2], [8, 3, -1])
+    assert N.nvfp4_get_device_status() == 7
+    assert u8(cache.k_codes)[1, 0, 3].any()
+    assert not u8(cache.k_codes)[0].any()
+
+
+def run_attention(N, cache, q, scale):
+    B, hq = q.shape[0], q.shape[1]
+    ws = torch.empty(N.decode_attention_nvfp4_workspace_size(B, hq, cache.capacity) // 4, dtype=torch.float32,
+                     device="cuda")
+    out = torch.full((B, hq, 128), float("nan"), dtype=torch.bfloat16, device="cuda")
+    N.decode_attention_nvfp4(cache, q.cuda(), scale, out, ws)
+    torch.cuda.synchronize()
+    return out
+
+
+@pytest.mark.parametrize("B,hq,hkv,lens", [
+    (2, 10, 2, [1, 17]), (3, 40, 8, [1000, 15, 2049]), (1, 8, 8, [300]), (2, 8, 1, [4096, 1023]),
+    (2, 6, 2, [0, 33])])
+def test_decode_attention(N, B, hq, hkv, lens):
+    cap = max(max(lens), 1) + 5
+    rec = synth.KVRecipe(hkv, seed=B * 100 + hq)
+    T = sum(lens)
+    k, v = rec.kv(max(T, 1), seed=11)
+    seq = np.concatenate([np.full(l, b) for b, l in enumerate(lens)]).astype(np.int64)
+    pos = np.concatenate([np.arange(l) for l in lens]).astype(np.int64)
+    k, v = k[:T], v[:T]
+    gk, gv = O.tensor_scale(f32(k)), O.tensor_scale(f32(v))
+    cache = N.KVCache(B, hkv, cap, gk, gv)
+    if T:
+        fill(N, cache, k, v, seq, pos)
+    cache.seq_lens.copy_(torch.tensor(lens, dtype=torch.int32))
+    q = rec.queries(B, hq, seed=12)
+    scale = 1.0 / math.sqrt(128)
+    out = run_attention(N, cache, q, scale)
+    assert N.nvfp4_get_device_status() == 0
+    rkc, rks, rvc, rvs = oracle_cache(B, hkv, cap)
+    if T:
+        O.kv_append(rkc, rks, rvc, rvs, f32(k), f32(v), seq, pos, np.float32(gk), np.float32(gv))
+    assert np.array_equal(u8(cache.k_codes), rkc) and np.array_equal(u8(cache.v_scales), rvs)
+    ref = O.decode_attention(f32(q), rkc, rks, rvc, rvs, lens, gk, gv, scale)
+    got = f32(out)
+    for b, l in enumerate(lens):
+        if l == 0:
+            assert not got[b].any(), "an empty sequence must give zeros"
+        else:
+            assert_close(got[b], ref[b], what=f"seq {b} len {l}")
+
+
+def test_seq_len_beyond_capacity_is_clamped_and_reported(N):
+    B, hq, hkv, cap = 1, 4, 1, 64
+    rec = synth.KVRecipe(hkv, seed=3)
+    k, v = rec.kv(cap, seed=1)
+    gk, gv = O.tensor_scale(f32(k)), O.tensor_scale(f32(v))
+    cache = N.KVCache(B, hkv, cap, gk, gv)
+    fill(N, cache, k, v, np.zeros(cap, np.int64), np.arange(cap))
+    cache.seq_lens.fill_(cap + 100)
+    q = rec.queries(B, hq, seed=2)
+    N.nvfp4_get_device_status()
+    out = run_attention(N, cache, q, 0.088)
+    assert N.nvfp4_get_device_status() == 7
+    rkc, rks, rvc, rvs = oracle_cache(B, hkv, cap)
+    O.kv_append(rkc, rks, rvc, rvs, f32(k), f32(v), np.zeros(cap, np.int64), np.arange(cap), np.float32(gk), np.float32(gv))
+    ref = O.decode_attention(f32(q), rkc, rks, rvc, rvs, [cap], gk, gv, 0.088)
+    assert_close(f32(out)[0], ref[0])
+
+
+def test_decode_batch_kv_append_workload(N):
+    """The decode-batch workload's K/V append: 256 new rows x 8 KV heads (one token per sequence)."""
+    w = synth.WORKLOADS["qwen14b_decode_linears_m256"]["kv_append"]
+    n, hkv = w["n_new"], w["num_kv_heads"]
+    rec = synth.KVRecipe(hkv, seed=synth.seed_for("qwen14b_decode_linears_m256", "kv") % (1 << 31), device="cuda")
+    k, v = rec.kv(n, seed=21)
+    cap = 512
+    pos = torch.randint(0, cap, (n,), generator=torch.Generator().manual_seed(2)).numpy()
+    gk, gv = O.tensor_scale(f32(k)), O.tensor_scale(f32(v))
+    cache = N.KVCache(n, hkv, cap, gk, gv)
+    fill(N, cache, k, v, np.arange(n), pos)
+    torch.cuda.synchronize()
+    rkc, rks, rvc, rvs = oracle_cache(n, hkv, cap)
+    O.kv_append(rkc, rks, rvc, rvs, f32(k), f32(v), np.arange(n), pos, np.float32(gk), np.float32(gv))
+    assert np.array_equal(u8(cache.k_codes), rkc) and np.array_equal(u8(cache.k_scales), rks)
+    assert np.array_equal(u8(cache.v_codes), rvc) and np.array_equal(u8(cache.v_scales), rvs)
+
+
+def test_full_size_decode_attention_workload(N):
+    """B=64, 40/8 heads, 16384 tokens per sequence, in the bench's launch
+    configuration; codes, scales and outputs checked on sampled sequences."""
+    wl = "qwen14b_decode_attention_b64_t16384"
+    w = synth.WORKLOADS[wl]
+    B, hq, hkv, T = w["batch"], w["num_q_heads"], w["num_kv_heads"], w["context"]
+    rec = synth.kv_recipe(wl, device="cuda")
+    # Static per-layer scales from the amax of all generated K (resp. V).
+    k_all = []
+    v_all = []
+    for b in range(B):
+        k, v = rec.kv(T, seed=synth.seed_for(wl, f"kv:{b}") % (1 << 62))
+        k_all.append(k); v_all.append(v)
+    K = torch.stack(k_all); V = torch.stack(v_all)  # [B, T, hkv, 128]
+    gk, gv = gscale(N, K.view(-1, 128)), gscale(N, V.view(-1, 128))
+    # The oracle's scales: its own formula on the amax from a library reduction.
+    gk_ref = O.tensor_scale(np.array([K.abs().max().float().item()], np.float32))
+    gv_ref = O.tensor_scale(np.array([V.abs().max().float().item()], np.float32))
+    assert np.float32(gk) == gk_ref and np.float32(gv) == gv_ref
+    cache = N.KVCache(B, hkv, T, gk, gv)
+    seq = torch.arange(B, dtype=torch.int32, device="cuda").repeat_interleave(T)
+    pos = torch.arange(T, dtype=torch.int32, device="cuda").repeat(B)
+    N.kv_append_nvfp4(cache, K.view(-1, hkv, 128), V.view(-1, hkv, 128), seq, pos)
+    cache.seq_lens.fill_(T)
+    q = rec.queries(B, hq, seed=synth.seed_for(wl, "q") % (1 << 62))
+    out = run_attention(N, cache, q, 1.0 / math.sqrt(128))
+    assert N.nvfp4_get_device_status() == 0
+    for b in (0, 37, B - 1):
+        kb, vb = f32(K[b]), f32(V[b])
+        rkc, rks, rvc, rvs = oracle_cache(1, hkv, T)
+        O.kv_append(rkc, rks, rvc, rvs, kb, vb, np.zeros(T, np.int64), np.arange(T), gk_ref, gv_ref)
+        assert np.array_equal(u8(cache.k_codes[b:b + 1]), rkc) and np.array_equal(u8(cache.k_scales[b:b + 1]), rks)
+        assert np.array_equal(u8(cache.v_codes[b:b + 1]), rvc) and np.array_equal(u8(cache.v_scales[b:b + 1]), rvs)
+        ref = O.decode_attention(f32(q[b:b + 1]), rkc, rks, rvc, rvs, [T], gk_ref, gv_ref, 1.0 / math.sqrt(128))
+        assert_close(f32(out[b]), ref[0], what=f"seq {b}")

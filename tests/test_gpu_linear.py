@@ -1,0 +1,136 @@
+"""GPU parity of a3 (block-scaled NVFP4 linear, tcgen05): outputs against the
+oracle's fp64 product of identical dequantized operands.
+
+Two kinds of inputs: (1) seeded random codes and scales handed to both sides
+(isolates the GEMM from the quantizer), (2) the workloads' bf16 activations
+and weights quantized by each side (codes are bit-exact, checked in
+test_gpu_quantize), so the dequantized operands are identical."""
+import numpy as np
+import pytest
+import torch
+
+from _util import TOL, assert_close, errors, f32, lib, u8
+from oracle import nvfp4_oracle as O
+from paper_2606_15682_gb300 import synth
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def N():
+    assert torch.cuda.is_available(), "GPU tests need a CUDA device"
+    return lib()
+
+
+def random_operand(rows, K, gen, scale_lo=0x30, scale_hi=0x48):
+    """Seeded random NVFP4 operand: packed codes, row-major scales (all codes, moderate scales)."""
+    codes = torch.randint(0, 256, (rows, K // 2), generator=gen, dtype=torch.int32).to(torch.uint8).numpy()
+    scales = torch.randint(scale_lo, scale_hi, (rows, K // 16), generator=gen, dtype=torch.int32).to(torch.uint8).numpy()
+    return codes, scales
+
+
+def run_linear(N, a_codes, a_scales_rm, g_a, w_codes, w_scales_rm, g_w, M, Nn, K, ldo=None):
+    dev = "cuda"
+    ac = torch.from_numpy(a_codes).to(dev)
+    wc = torch.from_numpy(w_codes).to(dev)
+    asf = torch.from_numpy(O.scales_to_mma(a_scales_rm)).to(dev)
+    wsf = torch.from_numpy(O.scales_to_mma(w_scales_rm)).to(dev)
+    ga = torch.tensor([g_a], dtype=torch.float32, device=dev)
+    gw = torch.tensor([g_w], dtype=torch.float32, device=dev)
+    ldo = Nn if ldo is None else ldo
+    out = torch.full((M, ldo), float("nan"), dtype=torch.bfloat16, device=dev)
+    N.nvfp4_linear(ac, asf, ga, wc, wsf, gw, out, M, Nn, K, ldo=ldo)
+    torch.cuda.synchronize()
+    assert N.nvfp4_get_device_status() == 0
+    return out
+
+
+@pytest.mark.parametrize("M,Nn,K", [(128, 128, 256), (1, 16, 256), (16, 128, 512), (130, 144, 512),
+                                    (257, 384, 1024), (300, 272, 2304), (128, 1024, 256)])
+def test_random_codes(N, M, Nn, K):
+    gen = torch.Generator().manual_seed(M * 1000 + Nn * 10 + K)
+    a_c, a_s = random_operand(M, K, gen)
+    w_c, w_s = random_operand(Nn, K, gen)
+    g_a, g_w = np.float32(0.0173), np.float32(0.00091)
+    out = run_linear(N, a_c, a_s, g_a, w_c, w_s, g_w, M, Nn, K)
+    ref = O.linear(a_c, a_s, g_a, w_c, w_s, g_w)
+    assert_close(f32(out), ref, what=f"{M}x{Nn}x{K}")
+
+
+def test_ldo_padding_untouched(N):
+    M, Nn, K, ldo = 200, 160, 512, 200
+    gen = torch.Generator().manual_seed(5)
+    a_c, a_s = random_operand(M, K, gen)
+    w_c, w_s = random_operand(Nn, K, gen)
+    out = run_linear(N, a_c, a_s, 1.0, w_c, w_s, 1.0, M, Nn, K, ldo=ldo)
+    ref = O.linear(a_c, a_s, 1.0, w_c, w_s, 1.0)
+    assert_close(f32(out[:, :Nn]), ref)
+    assert torch.isnan(out[:, Nn:].float()).all(), "columns beyond N must not be written"
+
+
+def test_single_block_structure(N):
+    # Only one nonzero 16-block per row: each output is one scaled block dot product,
+    # so a misplaced scale (row, k-block) shows up as a wrong value.
+    M, Nn, K = 128, 128, 512
+    rng = np.random.default_rng(9)
+    a_c = np.zeros((M, K // 2), np.uint8); w_c = np.zeros((Nn, K // 2), np.uint8)
+    kb_a = rng.integers(0, K // 16, M); kb_w = rng.integers(0, K // 16, Nn)
+    for r in range(M):
+        a_c[r, kb_a[r] * 8:(kb_a[r] + 1) * 8] = rng.integers(0, 256, 8)
+    for r in range(Nn):
+        w_c[r, kb_w[r] * 8:(kb_w[r] + 1) * 8] = rng.integers(0, 256, 8)
+    a_s = rng.integers(0x28, 0x50, (M, K // 16)).astype(np.uint8)
+    w_s = rng.integers(0x28, 0x50, (Nn, K // 16)).astype(np.uint8)
+    out = run_linear(N, a_c, a_s, 1.0, w_c, w_s, 1.0, M, Nn, K)
+    ref = O.linear(a_c, a_s, 1.0, w_c, w_s, 1.0)
+    assert_close(f32(out), ref)
+
+
+def test_deterministic(N):
+    M, Nn, K = 256, 256, 1024
+    gen = torch.Generator().manual_seed(11)
+    a_c, a_s = random_operand(M, K, gen)
+    w_c, w_s = random_operand(Nn, K, gen)
+    o1 = run_linear(N, a_c, a_s, 1.0, w_c, w_s, 1.0, M, Nn, K)
+    o2 = run_linear(N, a_c, a_s, 1.0, w_c, w_s, 1.0, M, Nn, K)
+    assert torch.equal(o1, o2)
+
+
+def quantize_gpu(N, x):
+    g = torch.empty(1, dtype=torch.float32, device="cuda")
+    N.nvfp4_tensor_scale(x, g)
+    codes = torch.empty(x.shape[0], x.shape[1] // 2, dtype=torch.uint8, device="cuda")
+    scales = torch.empty(N.nvfp4_scales_bytes(x.shape[0], x.shape[1], 1), dtype=torch.uint8, device="cuda")
+    N.nvfp4_quantize(x, g, codes, scales, 1)
+    return codes, scales, g
+
+
+WL = [w for w in synth.WORKLOADS if "linears" in synth.WORKLOADS[w]]
+
+
+@pytest.mark.parametrize("workload", WL)
+def test_workload_linears(N, workload):
+    """Every linear of every workload at full size, in the launch configuration the bench times.
+    Large outputs are compared on seeded samples of rows and columns."""
+    w = synth.WORKLOADS[workload]
+    report = []
+    for name, (Nn, K) in w["linears"].items():
+        a, W = synth.linear_inputs(workload, name, device="cuda")
+        M = a.shape[0]
+        ac, asf, ga = quantize_gpu(N, a)
+        wc, wsf, gw = quantize_gpu(N, W)
+        out = torch.empty(M, Nn, dtype=torch.bfloat16, device="cuda")
+        N.nvfp4_linear(ac, asf, ga, wc, wsf, gw, out, M, Nn, K)
+        torch.cuda.synchronize()
+        assert N.nvfp4_get_device_status() == 0
+        rng = np.random.default_rng(1)
+        rows = np.arange(M) if M * K <= 2048 * 8960 else np.sort(np.r_[rng.choice(M, 96, replace=False), M - 1])
+        cols = np.arange(Nn) if Nn * K <= 17920 * 1536 else np.sort(np.r_[rng.choice(Nn, 256, replace=False), Nn - 1])
+        g_a, g_w = O.tensor_scale(f32(a)), O.tensor_scale(f32(W))
+        assert np.float32(ga.item()) == g_a and np.float32(gw.item()) == g_w
+        ra_c, ra_s = O.quantize(f32(a[torch.as_tensor(rows, device="cuda")]), g_a)
+        rw_c, rw_s = O.quantize(f32(W[torch.as_tensor(cols, device="cuda")]), g_w)
+        ref = O.linear(ra_c, ra_s, g_a, rw_c, rw_s, g_w)
+        got = f32(out[torch.as_tensor(rows, device="cuda")][:, torch.as_tensor(cols, device="cuda")])
+        report.append((name,) + assert_close(got, ref, what=f"{workload}/{name}"))
+    print(workload, report)

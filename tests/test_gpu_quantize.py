@@ -1,0 +1,176 @@
+"""GPU parity of a1 (tensor scale) and a2 (NVFP4 quantize): bit-exact against
+the CPU oracle on the same seeded inputs."""
+import os
+
+import numpy as np
+import pytest
+import torch
+
+from _util import f32, lib, u8
+from oracle import nvfp4_oracle as O
+from paper_2606_15682_gb300 import synth
+
+pytestmark = pytest.mark.gpu
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+@pytest.fixture(scope="module")
+def N():
+    assert torch.cuda.is_available(), "GPU tests need a CUDA device"
+    return lib()
+
+
+def gpu_quantize(N, x, g, layout):
+    rows, cols = x.shape
+    codes = torch.empty(rows, cols // 2, dtype=torch.uint8, device="cuda")
+    scales = torch.full((N.nvfp4_scales_bytes(rows, cols, layout),), 0xEE, dtype=torch.uint8, device="cuda")
+    N.nvfp4_quantize(x, g, codes, scales, layout)
+    return codes, scales
+
+
+def check_quantize(N, x_bf16, g_np=None, layout=1, rows_sample=None):
+    """Quantize on the GPU with a GPU tensor scale (or a given g) and compare with the oracle."""
+    x = x_bf16.cuda()
+    g = torch.empty(1, dtype=torch.float32, device="cuda")
+    if g_np is None:
+        N.nvfp4_tensor_scale(x, g)
+        g_ref = O.tensor_scale(f32(x_bf16))
+        assert np.float32(g.item()) == g_ref
+    else:
+        g.fill_(float(g_np))
+        g_ref = np.float32(g_np)
+    codes, scales = gpu_quantize(N, x, g, layout)
+    torch.cuda.synchronize()
+    assert N.nvfp4_get_device_status() == 0
+    rows, cols = x.shape
+    sel = np.arange(rows) if rows_sample is None else np.asarray(rows_sample)
+    xc = f32(x_bf16[torch.as_tensor(sel)])
+    rc, rs = O.quantize(xc, g_ref)
+    gc = u8(codes)[sel]
+    gs = u8(scales)
+    gs = gs.reshape(rows, cols // 16)[sel] if layout == 0 else O.scales_from_mma(gs, rows, cols)[sel]
+    bad = np.argwhere(gc != rc)
+    assert bad.size == 0, f"{len(bad)} code bytes differ, first at {bad[:3].tolist()}: gpu {gc[tuple(bad[0])]:#x} oracle {rc[tuple(bad[0])]:#x}"
+    assert np.array_equal(gs, rs)
+    if layout == 1 and rows % 128:
+        pad = np.setdiff1d(np.arange(O.mma_scale_bytes(rows, cols)), O._mma_offsets(rows, cols // 16).ravel())
+        assert not u8(scales)[pad].any(), "padding rows of the MMA scale layout must be zero"
+    return codes, scales, g
+
+
+def _golden_blocks():
+    rows = []
+    for line in open(os.path.join(GOLDEN, "nvfp4_blocks.txt")):
+        line = line.split("#", 1)[0].strip()
+        if line:
+            g, vals, sc, packed = [p.strip() for p in line.split("|")]
+            rows.append((np.float32(float(g)), np.array([float(t) for t in vals.split()], np.float32),
+                         int(sc, 16), [int(t, 16) for t in packed.split()]))
+    return rows
+
+
+def test_golden_blocks_on_gpu(N):
+    # Hand-worked ties, saturation, signed zeros, scale underflow, subnormal scales.
+    for g, vals, sc, packed in _golden_blocks():
+        x = torch.from_numpy(np.tile(vals, 4)[None, :]).to(torch.bfloat16)
+        assert np.array_equal(f32(x)[0, :16], vals)
+        codes, scales = gpu_quantize(N, x.cuda(), torch.tensor([g], device="cuda"), 0)
+        assert u8(scales)[0] == sc
+        assert list(u8(codes)[0, :8]) == packed
+
+
+def test_signed_zero_and_tie_sweep(N):
+    # Every E2M1 midpoint, its float32 neighbours and tiny negatives, in blocks with S = 1, g = 1.
+    mids = [0.25, 0.75, 1.25, 1.75, 2.5, 3.5, 5.0]
+    vals = []
+    for m in mids:
+        for v in (m, float(np.nextafter(np.float32(m), 0)), float(np.nextafter(np.float32(m), 10))):
+            vals += [v, -v]
+    vals += [-0.1, -0.0, 0.0, -1e-3, 1e-3, 6.0, -6.0]
+    vals = np.array(vals, np.float32)
+    vals = vals[np.abs(vals) <= 6]
+    x = np.zeros((len(vals), 16), np.float32)
+    x[:, 0] = 6.0
+    x[:, 1] = vals
+    xb = torch.from_numpy(x).to(torch.bfloat16)  # neighbours round to bf16 values near the ties
+    check_quantize(N, xb, g_np=1.0, layout=0)
+
+
+@pytest.mark.parametrize("layout", [0, 1])
+@pytest.mark.parametrize("rows,cols,ld", [(1, 64, 64), (3, 16, 16), (130, 192, 192), (257, 512, 520), (64, 1536, 1536)])
+def test_random_blocks(N, rows, cols, ld, layout):
+    if layout == 1 and cols % 64:
+        pytest.skip("MMA layout needs cols % 64")
+    gen = torch.Generator().manual_seed(rows * 7919 + cols)
+    base = torch.randn(rows, ld, generator=gen)
+    # Per-block magnitudes over ~40 binades: exercises subnormal and saturated scales.
+    mag = torch.exp2(torch.randint(-30, 12, (rows, (ld + 15) // 16), generator=gen).float())
+    x = (base * mag.repeat_interleave(16, dim=1)[:, :ld]).to(torch.bfloat16)
+    x[0, :16] = 0
+    xv = x.cuda()[:, :cols] if ld != cols else x.cuda()
+    g = torch.empty(1, dtype=torch.float32, device="cuda")
+    N.nvfp4_tensor_scale(xv, g)
+    gref = O.tensor_scale(f32(x[:, :cols]))
+    assert np.float32(g.item()) == gref
+    codes, scales = gpu_quantize(N, xv, g, layout)
+    rc, rs = O.quantize(f32(x[:, :cols]), gref)
+    assert np.array_equal(u8(codes), rc)
+    gs = u8(scales).reshape(rows, cols // 16) if layout == 0 else O.scales_from_mma(u8(scales), rows, cols)
+    assert np.array_equal(gs, rs)
+
+
+def test_tensor_scale_all_zero_and_empty(N):
+    x = torch.zeros(5, 64, dtype=torch.bfloat16, device="cuda")
+    g = torch.full((1,), 7.0, device="cuda")
+    N.nvfp4_tensor_scale(x, g)
+    assert g.item() == 1.0
+    codes, scales = gpu_quantize(N, x, g, 1)
+    assert not u8(codes).any() and not u8(scales).any()
+    e = torch.zeros(0, 64, dtype=torch.bfloat16, device="cuda")
+    N.nvfp4_tensor_scale(e, g)
+    assert g.item() == 1.0
+
+
+def test_invalid_tensor_scale_sets_device_status(N):
+    x = torch.randn(4, 64, device="cuda").to(torch.bfloat16)
+    N.nvfp4_get_device_status()
+    codes, scales = gpu_quantize(N, x, torch.tensor([-1.0], device="cuda"), 0)
+    assert N.nvfp4_get_device_status() == 1
+    assert not u8(codes).any() and not u8(scales).any()
+    assert N.nvfp4_get_device_status() == 0
+
+
+def test_relayout_roundtrip(N):
+    rows, cols = 300, 320
+    s = torch.randint(0, 255, (rows, cols // 16), dtype=torch.uint8)
+    dst = torch.full((N.nvfp4_scales_bytes(rows, cols, 1),), 0xEE, dtype=torch.uint8, device="cuda")
+    N.nvfp4_scales_relayout(s.cuda(), dst, rows, cols, 0, 1)
+    assert np.array_equal(u8(dst), O.scales_to_mma(s.numpy()))
+    back = torch.zeros(rows * cols // 16, dtype=torch.uint8, device="cuda")
+    N.nvfp4_scales_relayout(dst, back, rows, cols, 1, 0)
+    assert np.array_equal(u8(back).reshape(rows, -1), s.numpy())
+
+
+WL = [w for w in synth.WORKLOADS if "linears" in synth.WORKLOADS[w]]
+
+
+@pytest.mark.parametrize("workload", WL)
+def test_workload_tensors_bit_exact(N, workload):
+    """Activations and weights of every linear of every workload, at full size."""
+    w = synth.WORKLOADS[workload]
+    big = w["M"] >= 8192
+    for name in w["linears"]:
+        a, W = synth.linear_inputs(workload, name, device="cuda")
+        rs = np.random.default_rng(0)
+        a_rows = np.sort(rs.choice(a.shape[0], 192, replace=False)) if big else None
+        w_rows = np.sort(rs.choice(W.shape[0], 384, replace=False)) if W.shape[0] * W.shape[1] > 5e7 else None
+        if big:
+            a_rows = np.concatenate([a_rows, [a.shape[0] - 1]])
+        for t, rows in ((a, a_rows), (W, w_rows)):
+            g_ref = O.tensor_scale(f32(t)) if rows is not None else None
+            if rows is not None:
+                # Same g as the GPU's own tensor-scale kernel, checked on the full tensor.
+                g = torch.empty(1, dtype=torch.float32, device="cuda")
+                N.nvfp4_tensor_scale(t, g)
+                assert np.float32(g.item()) == g_ref
+            check_quantize(N, t.cpu() if rows is None else t, g_np=g_ref, layout=1, rows_sample=rows)
