@@ -79,8 +79,9 @@ size_t nvfp4_scales_bytes(int64_t rows, int64_t cols, nvfp4_scale_layout layout)
  *   x_bf16 : [rows, cols] bf16, leading dimension ld >= cols (elements).
  *   g_dev  : one float, written on the device (never read first).
  * Three stream operations (clear, reduce, finalize).  Errors: null pointers
- * -> INVALID_ARG; rows or cols < 0, ld < cols -> SHAPE; x not 16-B aligned or
- * ld % 8 != 0 -> ALIGN.  rows*cols == 0 gives g = 1.
+ * -> INVALID_ARG (x may be NULL when rows*cols == 0); rows or cols < 0,
+ * ld < cols, cols % 8 != 0 -> SHAPE; x not 16-B aligned or ld % 8 != 0 ->
+ * ALIGN.  rows*cols == 0 gives g = 1.
  */
 nvfp4_status nvfp4_tensor_scale(const void* x_bf16, int64_t rows, int64_t cols, int64_t ld,
                                 float* g_dev, void* stream);
@@ -95,7 +96,8 @@ nvfp4_status nvfp4_tensor_scale(const void* x_bf16, int64_t rows, int64_t cols, 
  *   codes   : [rows, cols/2] bytes, row pitch cols/2.
  *   scales  : nvfp4_scales_bytes(rows, cols, layout) bytes.
  * cols % 16 == 0 (ROWMAJOR) or cols % 64 == 0 (MMA), else SHAPE.  x must be
- * 16-B aligned, codes 8-B aligned (ALIGN).
+ * 16-B aligned, codes 8-B aligned (ALIGN).  rows*cols == 0 is a no-op (any
+ * pointer may then be NULL); other null pointers -> INVALID_ARG.
  */
 nvfp4_status nvfp4_quantize(const void* x_bf16, int64_t rows, int64_t cols, int64_t ld,
                             const float* g_dev, uint8_t* codes, uint8_t* scales,

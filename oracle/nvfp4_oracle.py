@@ -322,6 +322,8 @@ def decode_attention(q_f32, k_codes, k_scales, v_codes, v_scales, seq_lens, g_k,
         s_t = softmax_scale * (q . K_hat_t),  t < seq_lens[b]
         o   = sum_t softmax(s)_t * V_hat_t
     q_f32: [batch, H_q, d].  Returns fp64 [len(batches), len(heads), d].
+    A sequence with no cached token has no softmax; its output is defined as
+    zeros (the library's reading; the paper does not consider that case).
     """
     q = np.asarray(q_f32, dtype=np.float64)
     B, Hq, d = q.shape
@@ -335,6 +337,8 @@ def decode_attention(q_f32, k_codes, k_scales, v_codes, v_scales, seq_lens, g_k,
     out = np.zeros((len(batches), len(heads), d))
     for i, b in enumerate(batches):
         T = int(seq_lens[b])
+        if T == 0:
+            continue
         cache = {}
         for j, h in enumerate(heads):
             kv = h // group

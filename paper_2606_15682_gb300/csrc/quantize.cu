@@ -144,7 +144,7 @@ int grid_for(uint64_t work_items, int threads) {
 }
 
 nvfp4_status check_bf16_matrix(const void* x, int64_t rows, int64_t cols, int64_t ld, int64_t col_mult) {
-  if (!x) return NVFP4_ERR_INVALID_ARG;
+  if (!x && rows * cols != 0) return NVFP4_ERR_INVALID_ARG;
   if (rows < 0 || cols < 0 || ld < cols || cols % col_mult) return NVFP4_ERR_SHAPE;
   if (rows * (cols / 8) >= (1ll << 32) || rows >= (1ll << 31)) return NVFP4_ERR_SHAPE;
   if (!aligned(x, 16) || ld % 8) return NVFP4_ERR_ALIGN;
@@ -193,12 +193,12 @@ NVFP4_API nvfp4_status nvfp4_tensor_scale(const void* x_bf16, int64_t rows, int6
 NVFP4_API nvfp4_status nvfp4_quantize(const void* x_bf16, int64_t rows, int64_t cols, int64_t ld,
                                       const float* g_dev, uint8_t* codes, uint8_t* scales,
                                       nvfp4_scale_layout layout, void* stream) {
-  if (!g_dev || !codes || !scales) return NVFP4_ERR_INVALID_ARG;
   if (layout != NVFP4_SCALES_ROWMAJOR && layout != NVFP4_SCALES_MMA) return NVFP4_ERR_INVALID_ARG;
   nvfp4_status st = check_bf16_matrix(x_bf16, rows, cols, ld, layout == NVFP4_SCALES_MMA ? 64 : 16);
   if (st != NVFP4_OK) return st;
-  if (!aligned(codes, 8) || !aligned(g_dev, 4)) return NVFP4_ERR_ALIGN;
   if (rows == 0 || cols == 0) return NVFP4_OK;
+  if (!g_dev || !codes || !scales) return NVFP4_ERR_INVALID_ARG;
+  if (!aligned(codes, 8) || !aligned(g_dev, 4)) return NVFP4_ERR_ALIGN;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   const ChunkMap map = make_map(rows, cols, ld);
   const uint32_t kblocks = static_cast<uint32_t>(cols / 16);

@@ -69,20 +69,28 @@ def _stream(stream):
 
 
 def _ptr(t):
+    """Device pointer of a dense tensor (None -> NULL)."""
     if t is None:
         return None
+    if not t.is_contiguous():
+        raise ValueError("tensor arguments must be contiguous (row-padded 2-D inputs go through the ld argument)")
     return ctypes.c_void_p(t.data_ptr())
+
+
+def _mat(x):
+    """(pointer, rows, cols, ld) of a 2-D row-major tensor whose rows may be padded."""
+    if x.dim() != 2 or (x.shape[1] > 1 and x.stride(1) != 1):
+        raise ValueError("expected a 2-D row-major tensor")
+    rows, cols = x.shape
+    ld = x.stride(0) if rows > 1 else cols
+    if rows > 1 and ld < cols:
+        raise ValueError("rows overlap")
+    return ctypes.c_void_p(x.data_ptr()), rows, cols, ld
 
 
 def _check(fn, code):
     if code != 0:
         raise NVFP4Error(fn, code)
-
-
-def _ld(x):
-    if x.dim() != 2 or x.stride(1) != 1:
-        raise ValueError("expected a 2-D row-major tensor")
-    return x.stride(0)
 
 
 # ----------------------------------------------------------------- calls ---
@@ -93,12 +101,11 @@ def nvfp4_scales_bytes(rows, cols, layout):
 
 def nvfp4_tensor_scale(x, g, stream=None):
     """g[0] <- amax(|x|) / (6*448) (device)."""
-    _check("nvfp4_tensor_scale", _tensor_scale(_ptr(x), x.shape[0], x.shape[1], _ld(x), _ptr(g), _stream(stream)))
+    _check("nvfp4_tensor_scale", _tensor_scale(*_mat(x), _ptr(g), _stream(stream)))
 
 
 def nvfp4_quantize(x, g, codes, scales, layout=SCALES_MMA, stream=None):
-    _check("nvfp4_quantize", _quantize(_ptr(x), x.shape[0], x.shape[1], _ld(x), _ptr(g), _ptr(codes), _ptr(scales),
-                                       layout, _stream(stream)))
+    _check("nvfp4_quantize", _quantize(*_mat(x), _ptr(g), _ptr(codes), _ptr(scales), layout, _stream(stream)))
 
 
 def nvfp4_scales_relayout(src, dst, rows, cols, from_layout, to_layout, stream=None):

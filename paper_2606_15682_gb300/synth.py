@@ -120,7 +120,7 @@ class KVRecipe:
         v = torch.randn(n_tokens, self.num_kv_heads, self.head_dim, generator=g, device=self.device) * self.v_spread
         k = torch.einsum("thc,hcd->thd", k, self.R32)
         v = torch.einsum("thc,hcd->thd", v, self.R32)
-        return k.to(torch.bfloat16), v.to(torch.bfloat16)
+        return k.to(torch.bfloat16).contiguous(), v.to(torch.bfloat16).contiguous()
 
     def queries(self, batch, num_q_heads, seed):
         """q bf16 [batch, H_q, d], rotated by the R of each head's KV head (contiguous groups)."""
@@ -128,7 +128,7 @@ class KVRecipe:
         q = torch.randn(batch, num_q_heads, self.head_dim, generator=g, device=self.device)
         group = num_q_heads // self.num_kv_heads
         R = self.R32.repeat_interleave(group, dim=0)  # [H_q, d, d]
-        return torch.einsum("bhc,hcd->bhd", q, R).to(torch.bfloat16)
+        return torch.einsum("bhc,hcd->bhd", q, R).to(torch.bfloat16).contiguous()
 
 
 def kv_recipe(workload="qwen14b_decode_attention_b64_t16384", device="cpu"):

@@ -263,6 +263,14 @@ def test_attention_single_token_returns_v():
             assert np.array_equal(out[b, h], O.dequantize(vc[b, h // 3, :1], vs[b, h // 3, :1], gv)[0])
 
 
+def test_attention_empty_sequence_is_zero():
+    rng = np.random.default_rng(10)
+    kc, ks, vc, vs, gk, gv = _cache(rng, 2, 1, 3)
+    q = rng.standard_normal((2, 2, 128)).astype(np.float32)
+    out = O.decode_attention(q, kc, ks, vc, vs, [0, 3], gk, gv, 0.1)
+    assert not out[0].any() and out[1].any()
+
+
 def test_attention_equal_keys_or_zero_query_is_mean_of_v():
     rng = np.random.default_rng(12)
     kc, ks, vc, vs, gk, gv = _cache(rng, 1, 1, 37)
