@@ -1,0 +1,102 @@
+"""Run one kernel of the hot path on one workload a few times (for profilers).
+
+    python -m paper_2606_15682_gb300.cases gemm --workload qwen1.5b_prefill_linears_m2048 --linear gate_up
+    python -m paper_2606_15682_gb300.cases quantize --workload qwen1.5b_prefill_linears_m2048 --linear down
+    python -m paper_2606_15682_gb300.cases attention --batch 64 --context 16384
+
+Inputs are seeded synthetic tensors (paper_2606_15682_gb300.synth); for the
+attention case the cache is filled with seeded random codes and scales
+directly, which is enough to time the kernel.  Prints the mean CUDA-event time
+of the measured call.
+"""
+from __future__ import annotations
+
+import argparse
+import math
+
+import torch
+
+from . import build as _build
+
+_build.build()
+from . import nvfp4 as N  # noqa: E402
+from . import synth  # noqa: E402
+
+
+def _quantized(x):
+    g = torch.empty(1, dtype=torch.float32, device=x.device)
+    N.nvfp4_tensor_scale(x, g)
+    c = torch.empty(x.shape[0], x.shape[1] // 2, dtype=torch.uint8, device=x.device)
+    s = torch.empty(N.nvfp4_scales_bytes(x.shape[0], x.shape[1], N.SCALES_MMA), dtype=torch.uint8, device=x.device)
+    N.nvfp4_quantize(x, g, c, s, N.SCALES_MMA)
+    return c, s, g
+
+
+def _time(fn, iters):
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
+    fn()
+    torch.cuda.synchronize()
+    ev[0].record()
+    for _ in range(iters):
+        fn()
+    ev[1].record()
+    torch.cuda.synchronize()
+    return ev[0].elapsed_time(ev[1]) / iters
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("kernel", choices=["gemm", "quantize", "tensor_scale", "attention"])
+    ap.add_argument("--workload", default="qwen1.5b_prefill_linears_m2048")
+    ap.add_argument("--linear", default="gate_up")
+    ap.add_argument("--batch", type=int, default=64)
+    ap.add_argument("--context", type=int, default=16384)
+    ap.add_argument("--iters", type=int, default=3)
+    a = ap.parse_args()
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    if a.kernel in ("gemm", "quantize", "tensor_scale"):
+        x, W = synth.linear_inputs(a.workload, a.linear, device=dev)
+        M, K = x.shape
+        Nn = W.shape[0]
+        if a.kernel == "gemm":
+            ac, asf, ga = _quantized(x)
+            wc, wsf, gw = _quantized(W)
+            del W
+            out = torch.empty(M, Nn, dtype=torch.bfloat16, device=dev)
+            ms = _time(lambda: N.nvfp4_linear(ac, asf, ga, wc, wsf, gw, out, M, Nn, K), a.iters)
+            print(f"gemm {a.workload}/{a.linear} {M}x{Nn}x{K}: {ms * 1e3:.1f} us, "
+                  f"{2 * M * Nn * K / ms / 1e9:.1f} TFLOP/s")
+        else:
+            g = torch.empty(1, dtype=torch.float32, device=dev)
+            N.nvfp4_tensor_scale(x, g)
+            c = torch.empty(M, K // 2, dtype=torch.uint8, device=dev)
+            s = torch.empty(N.nvfp4_scales_bytes(M, K, N.SCALES_MMA), dtype=torch.uint8, device=dev)
+            if a.kernel == "quantize":
+                ms = _time(lambda: N.nvfp4_quantize(x, g, c, s, N.SCALES_MMA), a.iters)
+                byt = M * K * (2 + 0.5 + 1 / 16)
+            else:
+                ms = _time(lambda: N.nvfp4_tensor_scale(x, g), a.iters)
+                byt = M * K * 2
+            print(f"{a.kernel} {a.workload}/{a.linear} {M}x{K}: {ms * 1e3:.1f} us, {byt / ms / 1e6:.0f} GB/s")
+    else:
+        B, hq, hkv, T = a.batch, 40, 8, a.context
+        gen = torch.Generator(device=dev)
+        gen.manual_seed(5)
+        cache = N.KVCache(B, hkv, T, 0.01, 0.01, device=dev)
+        for t in (cache.k_codes, cache.v_codes):
+            t.copy_(torch.randint(0, 256, t.shape, generator=gen, device=dev, dtype=torch.int32).to(torch.uint8))
+        for t in (cache.k_scales, cache.v_scales):
+            t.copy_(torch.randint(0x20, 0x58, t.shape, generator=gen, device=dev, dtype=torch.int32).to(torch.uint8))
+        cache.seq_lens.fill_(T)
+        q = torch.randn(B, hq, 128, generator=gen, device=dev).to(torch.bfloat16)
+        ws = torch.empty(N.decode_attention_nvfp4_workspace_size(B, hq, T) // 4, dtype=torch.float32, device=dev)
+        out = torch.empty(B, hq, 128, dtype=torch.bfloat16, device=dev)
+        ms = _time(lambda: N.decode_attention_nvfp4(cache, q, 1 / math.sqrt(128), out, ws), a.iters)
+        byt = B * hkv * T * 144
+        print(f"attention B={B} T={T}: {ms * 1e3:.1f} us, {byt / ms / 1e6:.0f} GB/s (K/V codes+scales)")
+    assert N.nvfp4_get_device_status() == 0
+
+
+if __name__ == "__main__":
+    main()
