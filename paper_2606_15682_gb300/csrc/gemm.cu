@@ -4,20 +4,29 @@
 //
 //   out[m, n] = bf16( g_a g_w sum_k a[m,k] w[n,k] )      (all linears, Appendix D.1)
 //
-// Persistent, warp-specialized CTA (one per SM), tile 128 x 128 x 256:
-//   warp 0      TMA producer: codes via 2-D tensor maps (128-byte swizzle),
-//               block-scale atoms via 1-D bulk copies, into a 5-stage ring.
-//   warp 1      allocates 512 TMEM columns; one lane copies the stage's scales
-//               smem -> TMEM (tcgen05.cp) and issues 4 MMAs of K = 64 per stage.
-//   warps 2..5  epilogue: tcgen05.ld the accumulator (double-buffered in TMEM so
-//               the next tile's MMAs overlap it), scale by g_a g_w, round to
-//               bf16, store.
+// Persistent, warp-specialized CTAs (one per SM), tile 128 x BN x 256, launched
+// in clusters of CM CTAs that work on CM consecutive 128-row tiles of the
+// same BN-column tile:
+//   warp 0      TMA producer: its own A tile (codes via a 2-D tensor map with
+//               the 128-byte swizzle) and A block scales (1-D bulk copy), plus
+//               1/CM of the shared W tile and W scales, multicast to every CTA
+//               of the cluster -- W bytes leave L2 once per cluster.
+//   warp 1      allocates 512 TMEM columns; one lane issues 4 MMAs of K = 64
+//               per stage; its commit releases the stage in every CTA of the
+//               cluster.
+//   warp 2      one lane copies each stage's block scales smem -> TMEM
+//               (tcgen05.cp) as soon as the stage lands, so the copies run
+//               ahead of, and in a different issue stream from, the MMAs.
+//   warps 3..   epilogue: drain 128 accumulator columns into registers, hand
+//               the accumulator back, scale by g_a g_w, round to bf16, stage in
+//               swizzled shared memory and write with TMA stores.
 // Every wait is bounded (NVFP4_ERR_TIMEOUT on expiry); the CTA then drains
 // its copies and MMAs and frees TMEM before returning.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
 #include <cfloat>
+#include <map>
 #include <mutex>
 
 #include "common.cuh"
@@ -26,24 +35,43 @@ namespace nvfp4 {
 namespace {
 
 constexpr int BM = 128;
-constexpr int BN = 128;
-constexpr int BK = 256;                  // elements per k-block = 128 bytes per row
-constexpr int kStages = 5;
-constexpr int kThreads = 192;
-constexpr uint32_t kTileBytesA = BM * BK / 2;  // 16 KiB
-constexpr uint32_t kTileBytesB = BN * BK / 2;  // 16 KiB
-constexpr uint32_t kSfBytes = 128 * (BK / 16); // 2 KiB: four 512-byte scale atoms
-constexpr uint32_t kStageBytes = kTileBytesA + kTileBytesB + 2 * kSfBytes;
+constexpr int BK = 256;  // elements per k-block = 128 bytes per row
 constexpr uint32_t kTmemCols = 512;
-constexpr uint32_t kSfTmemCol = 2 * BN;        // scale slots after the two accumulators
-constexpr size_t kSmemBytes = 1024 /*align slack*/ + kStages * kStageBytes + 256 /*barriers*/;
+constexpr int kEpiRows = 32, kEpiCols = 64;                 // one TMA store box (bf16)
+constexpr uint32_t kEpiBufBytes = kEpiRows * kEpiCols * 2;  // 4 KiB per epilogue warp
 
-static_assert(kSfTmemCol + kStages * 32 <= kTmemCols, "TMEM budget");
-
-// Instruction descriptor, kind::mxf4nvf4: A and B are packed E2M1 (format 1),
-// both K-major, scale type UE4M3 (bit 23 = 0), N >> 3 at bit 17, M >> 4 at bit 24.
-constexpr uint32_t kIdesc = (1u << 7) | (1u << 10) | (static_cast<uint32_t>(BN >> 3) << 17) |
-                            (static_cast<uint32_t>(BM >> 4) << 24);
+// BN = 128: double-buffered TMEM accumulator, 4 epilogue warps.  BN = 256:
+// one accumulator (TMEM also holds the scale slots) and 8 epilogue warps that
+// drain it into registers and release it before storing.
+template <int BN_, int STAGES_, int CM_>
+struct Cfg {
+  static constexpr int BN = BN_;
+  static constexpr int kStages = STAGES_;
+  static constexpr int CM = CM_;  // cluster size along M
+  static constexpr int kAccBufs = BN == 128 ? 2 : 1;
+  static constexpr int kEpiWarps = BN / 32;  // 128 accumulator columns each
+  static constexpr int kThreads = 96 + 32 * kEpiWarps;  // producer, MMA, scale copier, epilogue
+  static constexpr uint32_t kTileBytesA = BM * BK / 2;  // 16 KiB
+  static constexpr uint32_t kTileBytesB = BN * BK / 2;
+  static constexpr uint32_t kSfaBytes = 128 * (BK / 16);  // four 512-byte scale atoms
+  static constexpr uint32_t kSfbBytes = kSfaBytes * (BN / 128);
+  static constexpr uint32_t kStageBytes = kTileBytesA + kTileBytesB + kSfaBytes + kSfbBytes;
+  static constexpr int kBRowsPerCta = BN / CM;           // W rows each CTA loads and multicasts
+  static constexpr uint32_t kSfbSlice = kSfbBytes / CM;  // W scale bytes each CTA loads
+  static constexpr uint32_t kSfbColsPerMma = 4 * (BN / 128);
+  static constexpr uint32_t kSfCols = 16 + 4 * kSfbColsPerMma;  // TMEM columns of one stage's scales
+  static constexpr uint32_t kSfTmemCol = kAccBufs * BN;
+  static constexpr size_t kSmemBytes =
+      1024 /*align slack*/ + kStages * kStageBytes + kEpiWarps * kEpiBufBytes + 512 /*barriers*/;
+  // Instruction descriptor, kind::mxf4nvf4: A and B packed E2M1 (format 1),
+  // both K-major, UE4M3 scales (bit 23 = 0), N >> 3 at bit 17, M >> 4 at bit 24.
+  static constexpr uint32_t kIdesc = (1u << 7) | (1u << 10) | (static_cast<uint32_t>(BN >> 3) << 17) |
+                                     (static_cast<uint32_t>(BM >> 4) << 24);
+  static_assert(kSfTmemCol + kStages * kSfCols <= kTmemCols, "TMEM budget");
+  static_assert(kSmemBytes <= 227 * 1024, "shared memory budget");
+  static_assert(kBRowsPerCta % 8 == 0 && kSfbSlice % 16 == 0, "multicast slice granularity");
+  static_assert(kSfbSlice <= kSfaBytes || kSfbSlice % kSfaBytes == 0, "scale slices stay inside 128-row tiles");
+};
 
 // Shared-memory matrix descriptor of a K-major operand tile stored with the
 // 128-byte swizzle: rows of 128 B, 8-row groups 1024 B apart (SBO).
@@ -58,13 +86,13 @@ __device__ __forceinline__ uint64_t desc_sf(uint32_t saddr) {
          (static_cast<uint64_t>(128 >> 4) << 32) | (1ull << 46);
 }
 
-__device__ __forceinline__ void mma_fp4(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t sfa, uint32_t sfb,
-                                        uint32_t accumulate) {
+__device__ __forceinline__ void mma_fp4(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc, uint32_t sfa,
+                                        uint32_t sfb, uint32_t accumulate) {
   asm volatile(
       "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
       " tcgen05.mma.cta_group::1.kind::mxf4nvf4.block_scale.scale_vec::4X [%0], %1, %2, %3, [%5], [%6], p;\n}" ::"r"(
           d_tmem),
-      "l"(adesc), "l"(bdesc), "r"(kIdesc), "r"(accumulate), "r"(sfa), "r"(sfb)
+      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate), "r"(sfa), "r"(sfb)
       : "memory");
 }
 
@@ -72,7 +100,8 @@ __device__ __forceinline__ void copy_sf_to_tmem(uint32_t taddr, uint64_t desc) {
   asm volatile("tcgen05.cp.cta_group::1.32x128b.warpx4 [%0], %1;" ::"r"(taddr), "l"(desc) : "memory");
 }
 
-__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t r[32]) {
+// 32 lanes x 32 consecutive fp32 columns; completion via tmem_ld_wait().
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t* r) {
   asm volatile(
       "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,%17,%18,%19,"
       "%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
@@ -81,8 +110,8 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t r[32]) {
         "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]),
         "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
       : "r"(taddr));
-  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
+__device__ __forceinline__ void tmem_ld_wait() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
 
 __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   uint32_t d;
@@ -90,61 +119,79 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   return d;
 }
 
+__device__ __forceinline__ void st_shared_v4(uint32_t addr, uint32_t a, uint32_t b, uint32_t c, uint32_t d) {
+  asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(a), "r"(b), "r"(c), "r"(d) : "memory");
+}
+
 struct GemmArgs {
   const uint8_t* sfa;
   const uint8_t* sfb;
   const float* ga;
   const float* gb;
-  uint16_t* out;
-  int64_t ldo;
   int M, N, K;
   int tiles_m, tiles_n;
   int* status;
 };
 
-__global__ void __launch_bounds__(kThreads, 1)
+template <class C>
+__global__ void __launch_bounds__(C::kThreads, 1)
     nvfp4_gemm_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_constant__ CUtensorMap tmap_b,
-                      const GemmArgs args) {
+                      const __grid_constant__ CUtensorMap tmap_out, const GemmArgs args) {
+  constexpr int BN = C::BN;
+  constexpr int kStages = C::kStages;
+  constexpr int CM = C::CM;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* sA = smem;
-  uint8_t* sB = sA + kStages * kTileBytesA;
-  uint8_t* sSFA = sB + kStages * kTileBytesB;
-  uint8_t* sSFB = sSFA + kStages * kSfBytes;
-  uint64_t* full = reinterpret_cast<uint64_t*>(sSFB + kStages * kSfBytes);
+  uint8_t* sB = sA + kStages * C::kTileBytesA;
+  uint8_t* sEpi = sB + kStages * C::kTileBytesB;  // 1024-aligned: every tile above is a multiple of 1 KiB
+  uint8_t* sSFA = sEpi + C::kEpiWarps * kEpiBufBytes;
+  uint8_t* sSFB = sSFA + kStages * C::kSfaBytes;
+  uint64_t* full = reinterpret_cast<uint64_t*>(sSFB + kStages * C::kSfbBytes);
   uint64_t* empty = full + kStages;
-  uint64_t* tfull = empty + kStages;
+  uint64_t* sfready = empty + kStages;
+  uint64_t* tfull = sfready + kStages;
   uint64_t* tempty = tfull + 2;
   uint64_t* drain = tempty + 2;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+  uint64_t* drain_cp = drain + 1;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain_cp + 1);
   __shared__ volatile int abort_flag;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int kblocks = args.K / BK;
   const int kgroups = args.K / 64;
-  const int total_tiles = args.tiles_m * args.tiles_n;
+  const uint32_t rank = CM > 1 ? cluster_ctarank() : 0;
+  const uint16_t cluster_mask = static_cast<uint16_t>((1u << CM) - 1);
+  // Work unit: CM consecutive 128-row tiles x one BN-column tile, one per cluster.
+  const int msup = (args.tiles_m + CM - 1) / CM;
+  const int total_units = msup * args.tiles_n;
+  const int cluster_id = blockIdx.x / CM, n_clusters = gridDim.x / CM;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
       mbar_init(&full[s], 1);
-      mbar_init(&empty[s], 1);
+      mbar_init(&empty[s], CM);  // one MMA commit from every CTA reading the stage
+      mbar_init(&sfready[s], 1);
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(&tfull[a], 1);
-      mbar_init(&tempty[a], 4);
+      mbar_init(&tempty[a], C::kEpiWarps);
     }
     mbar_init(drain, 1);
+    mbar_init(drain_cp, 1);
     abort_flag = 0;
     fence_mbar_init();
     prefetch_tmap(&tmap_a);
     prefetch_tmap(&tmap_b);
+    prefetch_tmap(&tmap_out);
   }
   if (warp == 1) {
     tmem_alloc(tmem_slot, kTmemCols);
     tmem_relinquish();
   }
   tc_fence_before();
-  __syncthreads();
+  if (CM > 1) cluster_sync_all();  // peers' barriers exist before any multicast lands
+  else __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
 
@@ -160,24 +207,39 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint32_t issued_parity[kStages];
     bool issued[kStages];
     for (int s = 0; s < kStages; ++s) issued[s] = false;
-    for (int tile = blockIdx.x; tile < total_tiles && !abort_flag; tile += gridDim.x) {
-      const int mb = tile % args.tiles_m, nb = tile / args.tiles_m;
+    for (int u = cluster_id; u < total_units && !abort_flag; u += n_clusters) {
+      const int nb = u / msup;
+      const int mb = min((u % msup) * CM + static_cast<int>(rank), args.tiles_m - 1);  // spare CTAs redo the last tile
       const uint8_t* sfa_tile = args.sfa + (static_cast<size_t>(mb) * kgroups) * 512;
-      const uint8_t* sfb_tile = args.sfb + (static_cast<size_t>(nb) * kgroups) * 512;
+      const uint8_t* sfb_tiles = args.sfb + (static_cast<size_t>(nb) * (BN / 128) * kgroups) * 512;
       for (int kb = 0; kb < kblocks; ++kb) {
         if (!mbar_wait_bounded(&empty[stage], phase ^ 1u, &abort_flag)) { fail(); break; }
-        mbar_arrive_expect_tx(&full[stage], kStageBytes);
-        tma_load_2d(sA + stage * kTileBytesA, &tmap_a, &full[stage], kb * (BK / 2), mb * BM);
-        tma_load_2d(sB + stage * kTileBytesB, &tmap_b, &full[stage], kb * (BK / 2), nb * BN);
-        bulk_load(sSFA + stage * kSfBytes, sfa_tile + static_cast<size_t>(kb) * kSfBytes, kSfBytes, &full[stage]);
-        bulk_load(sSFB + stage * kSfBytes, sfb_tile + static_cast<size_t>(kb) * kSfBytes, kSfBytes, &full[stage]);
+        mbar_arrive_expect_tx(&full[stage], C::kStageBytes);
+        tma_load_2d(sA + stage * C::kTileBytesA, &tmap_a, &full[stage], kb * (BK / 2), mb * BM);
+        bulk_load(sSFA + stage * C::kSfaBytes, sfa_tile + static_cast<size_t>(kb) * C::kSfaBytes, C::kSfaBytes,
+                  &full[stage]);
+        // This CTA's share of the stage's W scales: bytes [rank*slice, +slice) of
+        // the stage buffer, which holds BN/128 row tiles of 2 KiB each.
+#pragma unroll
+        for (uint32_t off = rank * C::kSfbSlice; off < (rank + 1) * C::kSfbSlice; off += C::kSfaBytes) {
+          const uint32_t len = C::kSfbSlice < C::kSfaBytes ? C::kSfbSlice : C::kSfaBytes;
+          const uint32_t j = off / C::kSfaBytes, within = off % C::kSfaBytes;
+          const uint8_t* src =
+              sfb_tiles + (static_cast<size_t>(j) * kgroups) * 512 + static_cast<size_t>(kb) * C::kSfaBytes + within;
+          if (CM > 1) bulk_load_mc(sSFB + stage * C::kSfbBytes + off, src, len, &full[stage], cluster_mask);
+          else bulk_load(sSFB + stage * C::kSfbBytes + off, src, len, &full[stage]);
+        }
+        uint8_t* b_dst = sB + stage * C::kTileBytesB + rank * C::kBRowsPerCta * (BK / 2);
+        const int b_row = nb * BN + static_cast<int>(rank) * C::kBRowsPerCta;
+        if (CM > 1) tma_load_2d_mc(b_dst, &tmap_b, &full[stage], kb * (BK / 2), b_row, cluster_mask);
+        else tma_load_2d(b_dst, &tmap_b, &full[stage], kb * (BK / 2), b_row);
         issued[stage] = true;
         issued_parity[stage] = phase;
         if (++stage == kStages) { stage = 0; phase ^= 1u; }
       }
     }
     if (abort_flag) {
-      // Let every copy this thread started land before the CTA exits.
+      // Let every copy destined for this CTA land before it exits.
       for (int s = 0; s < kStages; ++s)
         if (issued[s]) mbar_wait_bounded(&full[s], issued_parity[s], nullptr);
     }
@@ -187,28 +249,26 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint32_t phase = 0;
     int local = 0;
     const uint32_t sA0 = smem_u32(sA), sB0 = smem_u32(sB), sSFA0 = smem_u32(sSFA), sSFB0 = smem_u32(sSFB);
-    for (int tile = blockIdx.x; tile < total_tiles && !abort_flag; tile += gridDim.x, ++local) {
-      const int acc = local & 1;
-      const uint32_t acc_phase = (local >> 1) & 1;
+    for (int u = cluster_id; u < total_units && !abort_flag; u += n_clusters, ++local) {
+      const int acc = local % C::kAccBufs;
+      const uint32_t acc_phase = (local / C::kAccBufs) & 1;
       if (!mbar_wait_bounded(&tempty[acc], acc_phase ^ 1u, &abort_flag)) { fail(); break; }
       tc_fence_after();
       const uint32_t d_tmem = tmem + acc * BN;
       bool ok = true;
       for (int kb = 0; kb < kblocks; ++kb) {
-        if (!mbar_wait_bounded(&full[stage], phase, &abort_flag)) { fail(); ok = false; break; }
+        if (!mbar_wait_bounded(&sfready[stage], phase, &abort_flag)) { fail(); ok = false; break; }
         tc_fence_after();
-        const uint32_t sf_col = tmem + kSfTmemCol + stage * 32;
+        const uint32_t sfa_col = tmem + C::kSfTmemCol + stage * C::kSfCols;
+        const uint32_t sfb_col = sfa_col + 16;
 #pragma unroll
         for (int kk = 0; kk < 4; ++kk) {
-          copy_sf_to_tmem(sf_col + kk * 4, desc_sf(sSFA0 + stage * kSfBytes + kk * 512));
-          copy_sf_to_tmem(sf_col + 16 + kk * 4, desc_sf(sSFB0 + stage * kSfBytes + kk * 512));
+          mma_fp4(d_tmem, desc_sw128(sA0 + stage * C::kTileBytesA + kk * 32),
+                  desc_sw128(sB0 + stage * C::kTileBytesB + kk * 32), C::kIdesc, sfa_col + kk * 4,
+                  sfb_col + kk * C::kSfbColsPerMma, (kb | kk) != 0);
         }
-#pragma unroll
-        for (int kk = 0; kk < 4; ++kk) {
-          mma_fp4(d_tmem, desc_sw128(sA0 + stage * kTileBytesA + kk * 32), desc_sw128(sB0 + stage * kTileBytesB + kk * 32),
-                  sf_col + kk * 4, sf_col + 16 + kk * 4, (kb | kk) != 0);
-        }
-        tc_commit(&empty[stage]);
+        if (CM > 1) tc_commit_mc(&empty[stage], cluster_mask);
+        else tc_commit(&empty[stage]);
         if (++stage == kStages) { stage = 0; phase ^= 1u; }
       }
       if (!ok) break;
@@ -217,15 +277,48 @@ __global__ void __launch_bounds__(kThreads, 1)
     // Wait until every MMA issued above has retired before TMEM is freed.
     tc_commit(drain);
     mbar_wait_bounded(drain, 0, nullptr);
-  } else if (warp >= 2) {
+  } else if (warp == 2 && lane == 0) {
+    // ---------------------------------------------- block scales -> TMEM ---
+    // Slot `stage` is rewritten only after the stage's next `full` phase, which
+    // the producer starts only after the MMAs that read the slot have retired.
+    int stage = 0;
+    uint32_t phase = 0;
+    const uint32_t sSFA0 = smem_u32(sSFA), sSFB0 = smem_u32(sSFB);
+    for (int u = cluster_id; u < total_units && !abort_flag; u += n_clusters) {
+      bool ok = true;
+      for (int kb = 0; kb < kblocks; ++kb) {
+        if (!mbar_wait_bounded(&full[stage], phase, &abort_flag)) { fail(); ok = false; break; }
+        tc_fence_after();
+        const uint32_t sfa_col = tmem + C::kSfTmemCol + stage * C::kSfCols;
+        const uint32_t sfb_col = sfa_col + 16;
+#pragma unroll
+        for (int kk = 0; kk < 4; ++kk) {
+          copy_sf_to_tmem(sfa_col + kk * 4, desc_sf(sSFA0 + stage * C::kSfaBytes + kk * 512));
+#pragma unroll
+          for (int j = 0; j < BN / 128; ++j)
+            copy_sf_to_tmem(sfb_col + kk * C::kSfbColsPerMma + j * 4,
+                            desc_sf(sSFB0 + stage * C::kSfbBytes + j * C::kSfaBytes + kk * 512));
+        }
+        tc_commit(&sfready[stage]);
+        if (++stage == kStages) { stage = 0; phase ^= 1u; }
+      }
+      if (!ok) break;
+    }
+    tc_commit(drain_cp);
+    mbar_wait_bounded(drain_cp, 0, nullptr);
+  } else if (warp >= 3) {
     // --------------------------------------------------------- epilogue ---
-    const int quarter = warp & 3;  // TMEM lanes this warp may access
+    const int quarter = warp & 3;                 // TMEM lanes this warp may access
+    const int colbase = ((warp - 3) >> 2) * 128;  // accumulator columns this warp drains
+    uint8_t* buf_ptr = sEpi + (warp - 3) * kEpiBufBytes;
+    const uint32_t buf = smem_u32(buf_ptr);
     const float scale = __fmul_rn(__ldg(args.ga), __ldg(args.gb));
     int local = 0;
-    for (int tile = blockIdx.x; tile < total_tiles; tile += gridDim.x, ++local) {
-      const int mb = tile % args.tiles_m, nb = tile / args.tiles_m;
-      const int acc = local & 1;
-      const uint32_t acc_phase = (local >> 1) & 1;
+    for (int u = cluster_id; u < total_units; u += n_clusters, ++local) {
+      const int nb = u / msup;
+      const int mb = (u % msup) * CM + static_cast<int>(rank);  // spare CTAs (mb >= tiles_m) store nothing
+      const int acc = local % C::kAccBufs;
+      const uint32_t acc_phase = (local / C::kAccBufs) & 1;
       // Lane 0 waits and broadcasts, so the warp stays converged for the
       // .sync.aligned TMEM loads below even on the timeout path.
       int ok = 1;
@@ -235,36 +328,46 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       if (!__shfl_sync(0xffffffffu, ok, 0)) break;
       tc_fence_after();
-      const int row = mb * BM + quarter * 32 + lane;
-      const uint32_t taddr = tmem + (static_cast<uint32_t>(quarter * 32) << 16) + acc * BN;
-#pragma unroll 1
-      for (int c = 0; c < BN / 32; ++c) {
-        uint32_t r[32];
-        tmem_ld32(taddr + c * 32, r);
-        const int col0 = nb * BN + c * 32;
-        if (row < args.M) {
-          uint16_t* dst = args.out + static_cast<int64_t>(row) * args.ldo + col0;
+      // Drain 128 columns into registers, then hand the accumulator back.
+      uint32_t r[128];
+      const uint32_t taddr = tmem + (static_cast<uint32_t>(quarter * 32) << 16) + acc * BN + colbase;
 #pragma unroll
-          for (int v = 0; v < 4; ++v) {
-            if (col0 + v * 8 < args.N) {
-              uint4 w;
-              w.x = pack_bf16x2(__uint_as_float(r[8 * v + 0]) * scale, __uint_as_float(r[8 * v + 1]) * scale);
-              w.y = pack_bf16x2(__uint_as_float(r[8 * v + 2]) * scale, __uint_as_float(r[8 * v + 3]) * scale);
-              w.z = pack_bf16x2(__uint_as_float(r[8 * v + 4]) * scale, __uint_as_float(r[8 * v + 5]) * scale);
-              w.w = pack_bf16x2(__uint_as_float(r[8 * v + 6]) * scale, __uint_as_float(r[8 * v + 7]) * scale);
-              reinterpret_cast<uint4*>(dst)[v] = w;
-            }
-          }
-        }
-      }
+      for (int c = 0; c < 4; ++c) tmem_ld32(taddr + c * 32, r + 32 * c);
+      tmem_ld_wait();
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&tempty[acc]);
+
+      // Two 32 x 64 bf16 boxes; row `lane` of a box is 8 chunks of 16 B stored
+      // at chunk position (c ^ lane%8): the 128-byte swizzle the store expects.
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {
+        if (lane == 0) bulk_wait_read_all();  // the previous box has left the buffer
+        __syncwarp();
+#pragma unroll
+        for (int c = 0; c < 8; ++c) {
+          const uint32_t* v = r + 64 * h + 8 * c;
+          st_shared_v4(buf + lane * 128 + ((c ^ (lane & 7)) << 4),
+                       pack_bf16x2(__uint_as_float(v[0]) * scale, __uint_as_float(v[1]) * scale),
+                       pack_bf16x2(__uint_as_float(v[2]) * scale, __uint_as_float(v[3]) * scale),
+                       pack_bf16x2(__uint_as_float(v[4]) * scale, __uint_as_float(v[5]) * scale),
+                       pack_bf16x2(__uint_as_float(v[6]) * scale, __uint_as_float(v[7]) * scale));
+        }
+        fence_proxy_async_smem();
+        __syncwarp();
+        const int x = nb * BN + colbase + h * kEpiCols, y = mb * BM + quarter * 32;
+        if (lane == 0 && x < args.N && y < args.M) {  // boxes reaching past M or N are clipped by the TMA unit
+          tma_store_2d(&tmap_out, buf_ptr, x, y);
+          bulk_commit_group();
+        }
+      }
     }
+    if (lane == 0) bulk_wait_all();
   }
 
   tc_fence_before();
-  __syncthreads();
+  if (CM > 1) cluster_sync_all();  // no peer may still multicast into, or arrive on, this CTA
+  else __syncthreads();
   tc_fence_after();
   if (warp == 1) tmem_dealloc(tmem, kTmemCols);
 }
@@ -298,18 +401,106 @@ bool make_code_map(CUtensorMap* map, const uint8_t* base, int64_t rows, int64_t 
   return r == CUDA_SUCCESS;
 }
 
-bool ensure_smem_attr() {
-  static bool done[64] = {};
-  int d = 0;
-  if (cudaGetDevice(&d) != cudaSuccess || d < 0 || d >= 64) return false;
-  if (!done[d]) {
-    if (cudaFuncSetAttribute(nvfp4_gemm_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             static_cast<int>(kSmemBytes)) != cudaSuccess)
-      return false;
-    done[d] = true;
-  }
-  return true;
+// bf16 [M, N] output with row pitch ldo, stored in 32 x 64 boxes, 128-B swizzle.
+bool make_out_map(CUtensorMap* map, void* base, int64_t M, int64_t N, int64_t ldo) {
+  auto enc = tensor_map_encoder();
+  if (!enc) return false;
+  cuuint64_t dims[2] = {static_cast<cuuint64_t>(N), static_cast<cuuint64_t>(M)};
+  cuuint64_t strides[1] = {static_cast<cuuint64_t>(ldo * 2)};
+  cuuint32_t box[2] = {kEpiCols, kEpiRows};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, base, dims, strides, box, estr,
+                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_NONE,
+                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
 }
+
+// Per-device, per-configuration launch set-up: the shared-memory opt-in and
+// the number of clusters resident on the GPU at once (persistent grid).
+template <class C>
+int resident_clusters() {
+  static std::mutex mu;
+  static std::map<int, int> cache;
+  int d = 0;
+  if (cudaGetDevice(&d) != cudaSuccess) return 0;
+  std::lock_guard<std::mutex> lock(mu);
+  auto it = cache.find(d);
+  if (it != cache.end()) return it->second;
+  if (cudaFuncSetAttribute(nvfp4_gemm_kernel<C>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           static_cast<int>(C::kSmemBytes)) != cudaSuccess)
+    return 0;
+  int n = sm_count() / C::CM;
+  if (C::CM > 1) {
+    cudaLaunchConfig_t cfg = {};
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = C::CM;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.gridDim = dim3(C::CM * n, 1, 1);
+    cfg.blockDim = dim3(C::kThreads, 1, 1);
+    cfg.dynamicSmemBytes = C::kSmemBytes;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    int clusters = 0;
+    if (cudaOccupancyMaxActiveClusters(&clusters, nvfp4_gemm_kernel<C>, &cfg) != cudaSuccess || clusters <= 0) {
+      cudaGetLastError();
+      return 0;
+    }
+    n = clusters;
+  }
+  cache[d] = n;
+  return n;
+}
+
+template <class C>
+nvfp4_status launch(const uint8_t* a_codes, const uint8_t* a_scales, const float* g_a, const uint8_t* w_codes,
+                    const uint8_t* w_scales, const float* g_w, int64_t M, int64_t N, int64_t K, void* out_bf16,
+                    int64_t ldo, cudaStream_t stream) {
+  const int64_t tiles_m = (M + BM - 1) / BM, tiles_n = (N + C::BN - 1) / C::BN;
+  const int64_t units = ((tiles_m + C::CM - 1) / C::CM) * tiles_n;
+  if (units >= (1ll << 31)) return NVFP4_ERR_SHAPE;
+  CUtensorMap ma, mb, mo;
+  if (!make_code_map(&ma, a_codes, M, K, BM) || !make_code_map(&mb, w_codes, N, K, C::kBRowsPerCta) ||
+      !make_out_map(&mo, out_bf16, M, N, ldo))
+    return NVFP4_ERR_CUDA;
+  const int clusters_max = resident_clusters<C>();
+  if (clusters_max <= 0) return NVFP4_ERR_CUDA;
+  GemmArgs args;
+  args.sfa = a_scales;
+  args.sfb = w_scales;
+  args.ga = g_a;
+  args.gb = g_w;
+  args.M = static_cast<int>(M);
+  args.N = static_cast<int>(N);
+  args.K = static_cast<int>(K);
+  args.tiles_m = static_cast<int>(tiles_m);
+  args.tiles_n = static_cast<int>(tiles_n);
+  args.status = status_word_dev();
+  const int clusters = static_cast<int>(units < clusters_max ? units : clusters_max);
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = C::CM;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.gridDim = dim3(clusters * C::CM, 1, 1);
+  cfg.blockDim = dim3(C::kThreads, 1, 1);
+  cfg.dynamicSmemBytes = C::kSmemBytes;
+  cfg.stream = stream;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  if (cudaLaunchKernelEx(&cfg, nvfp4_gemm_kernel<C>, ma, mb, mo, args) != cudaSuccess) return NVFP4_ERR_CUDA;
+  count_launches(1);
+  return launch_status();
+}
+
+#ifndef NVFP4_GEMM_BN
+#define NVFP4_GEMM_BN 0  // 0: choose per shape
+#endif
+#ifndef NVFP4_GEMM_CM
+#define NVFP4_GEMM_CM 0  // 0: choose per shape
+#endif
 
 }  // namespace
 }  // namespace nvfp4
@@ -325,27 +516,23 @@ NVFP4_API nvfp4_status nvfp4_linear(const uint8_t* a_codes, const uint8_t* a_sca
   if (!aligned(a_codes, 16) || !aligned(w_codes, 16) || !aligned(a_scales, 16) || !aligned(w_scales, 16) ||
       !aligned(out_bf16, 16) || !aligned(g_a, 4) || !aligned(g_w, 4))
     return NVFP4_ERR_ALIGN;
-  const int64_t tiles_m = (M + BM - 1) / BM, tiles_n = (N + BN - 1) / BN;
-  if (tiles_m * tiles_n >= (1ll << 31)) return NVFP4_ERR_SHAPE;
-  CUtensorMap ma, mb;
-  if (!make_code_map(&ma, a_codes, M, K, BM) || !make_code_map(&mb, w_codes, N, K, BN)) return NVFP4_ERR_CUDA;
-  if (!ensure_smem_attr()) return NVFP4_ERR_CUDA;
-  GemmArgs args;
-  args.sfa = a_scales;
-  args.sfb = w_scales;
-  args.ga = g_a;
-  args.gb = g_w;
-  args.out = static_cast<uint16_t*>(out_bf16);
-  args.ldo = ldo;
-  args.M = static_cast<int>(M);
-  args.N = static_cast<int>(N);
-  args.K = static_cast<int>(K);
-  args.tiles_m = static_cast<int>(tiles_m);
-  args.tiles_n = static_cast<int>(tiles_n);
-  args.status = status_word_dev();
-  const int64_t tiles = tiles_m * tiles_n;
-  const int grid = static_cast<int>(tiles < sm_count() ? tiles : sm_count());
-  nvfp4_gemm_kernel<<<grid, kThreads, kSmemBytes, static_cast<cudaStream_t>(stream)>>>(ma, mb, args);
-  count_launches(1);
-  return launch_status();
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const int64_t tiles_m = (M + BM - 1) / BM;
+  const int bn = NVFP4_GEMM_BN ? NVFP4_GEMM_BN : (N % 256 == 0 ? 256 : 128);
+  // Measured on GB300: sharing W tiles by cluster multicast did not beat
+  // independent CTAs on these shapes (the cluster waits for its slowest CTA),
+  // so clusters are off by default; the multicast path stays selectable.
+  const int cm = NVFP4_GEMM_CM ? NVFP4_GEMM_CM : 1;
+  (void)tiles_m;
+#define NVFP4_LAUNCH(BN_, ST_, CM_) \
+  return launch<Cfg<BN_, ST_, CM_>>(a_codes, a_scales, g_a, w_codes, w_scales, g_w, M, N, K, out_bf16, ldo, s)
+  if (bn == 256) {
+    if (cm >= 4) NVFP4_LAUNCH(256, 3, 4);
+    if (cm == 2) NVFP4_LAUNCH(256, 3, 2);
+    NVFP4_LAUNCH(256, 3, 1);
+  }
+  if (cm >= 4) NVFP4_LAUNCH(128, 5, 4);
+  if (cm == 2) NVFP4_LAUNCH(128, 5, 2);
+  NVFP4_LAUNCH(128, 5, 1);
+#undef NVFP4_LAUNCH
 }
