@@ -34,6 +34,10 @@
 namespace nvfp4 {
 namespace {
 
+#ifndef NVFP4_GEMM_COPY_WARPS
+#define NVFP4_GEMM_COPY_WARPS 2
+#endif
+
 constexpr int BM = 128;
 constexpr int BK = 256;  // elements per k-block = 128 bytes per row
 constexpr uint32_t kTmemCols = 512;
@@ -372,6 +376,316 @@ __global__ void __launch_bounds__(C::kThreads, 1)
   if (warp == 1) tmem_dealloc(tmem, kTmemCols);
 }
 
+// ------------------------------------------------------ CTA-pair kernel ---
+// A pair of CTAs (a cluster of 2 on neighbouring SMs) computes a 256 x 256
+// tile with tcgen05.mma.cta_group::2: each CTA holds its own 128 rows of A and
+// its own 128-row half of the W tile in shared memory, and its 128 x 256 slice
+// of the accumulator in its own TMEM.  Per SM this halves the W bytes loaded
+// and the scale copies issued for the same FLOPs.  W scales (all 256 rows) are
+// loaded by both CTAs so that each TMEM receives the full set.  The leader
+// (rank 0) issues the copies and the MMAs; the peer issues its own loads with
+// the pair form of TMA, whose completion is counted on the leader's barrier.
+
+__device__ __forceinline__ void mma_fp4_pair(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
+                                             uint32_t sfa, uint32_t sfb, uint32_t accumulate) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+      " tcgen05.mma.cta_group::2.kind::mxf4nvf4.block_scale.scale_vec::4X [%0], %1, %2, %3, [%5], [%6], p;\n}" ::"r"(
+          d_tmem),
+      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate), "r"(sfa), "r"(sfb)
+      : "memory");
+}
+__device__ __forceinline__ void copy_sf_to_tmem_pair(uint32_t taddr, uint64_t desc) {
+  asm volatile("tcgen05.cp.cta_group::2.32x128b.warpx4 [%0], %1;" ::"r"(taddr), "l"(desc) : "memory");
+}
+// Arrive on the barrier at this offset in every CTA of `mask` once all
+// tcgen05 operations this thread issued for the pair have completed.
+__device__ __forceinline__ void tc_commit_pair(uint64_t* bar, uint16_t mask) {
+  asm volatile("tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::"r"(
+                   smem_u32(bar)),
+               "h"(mask)
+               : "memory");
+}
+__device__ __forceinline__ void tmem_alloc_pair(uint32_t* smem_slot, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(smem_slot)),
+               "r"(ncols)
+               : "memory");
+}
+__device__ __forceinline__ void tmem_relinquish_pair() {
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc_pair(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
+}
+// 2-D TMA load into this CTA's shared memory whose completion is counted on
+// the barrier at offset `bar` in the leader CTA of the pair.
+__device__ __forceinline__ void tma_load_2d_to_leader(void* smem_dst, const void* tmap, uint64_t* bar, int x, int y) {
+  uint32_t remote;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(smem_u32(bar)), "r"(0));
+  asm volatile(
+      "cp.async.bulk.tensor.2d.cta_group::2.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%3, %4}], [%2];" ::"r"(smem_u32(smem_dst)),
+      "l"(reinterpret_cast<uint64_t>(tmap)), "r"(remote), "r"(x), "r"(y)
+      : "memory");
+}
+// Arrive on the barrier at this shared-memory offset in CTA `rank` of the cluster.
+__device__ __forceinline__ void mbar_arrive_cluster(uint64_t* bar, uint32_t rank) {
+  uint32_t remote;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(smem_u32(bar)), "r"(rank));
+  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(remote) : "memory");
+}
+
+template <int STAGES_>
+struct PairCfg {
+  static constexpr int BN = 256;                 // MMA N (both halves of the pair)
+  static constexpr int kStages = STAGES_;
+  static constexpr int kEpiWarps = 8;            // 128 rows x 256 accumulator columns per CTA
+  static constexpr int kCopyWarps = NVFP4_GEMM_COPY_WARPS;  // warps issuing the scale copies (1, 2 or 4)
+  static constexpr int kThreads = 64 + 32 * kCopyWarps + 32 * kEpiWarps;
+  static constexpr uint32_t kTileBytesA = BM * BK / 2;   // own 128 rows
+  static constexpr uint32_t kTileBytesB = 128 * BK / 2;  // own half of the 256-row W tile
+  static constexpr uint32_t kSfaBytes = 128 * (BK / 16);
+  static constexpr uint32_t kSfbBytes = 2 * kSfaBytes;   // all 256 W rows
+  static constexpr uint32_t kStageBytes = kTileBytesA + kTileBytesB + kSfaBytes + kSfbBytes;
+  static constexpr uint32_t kSfCols = 16 + 32;
+  static constexpr uint32_t kSfTmemCol = BN;
+  static constexpr size_t kSmemBytes =
+      1024 + kStages * kStageBytes + kEpiWarps * kEpiBufBytes + 512 /*barriers*/;
+  static constexpr uint32_t kIdesc = (1u << 7) | (1u << 10) | (static_cast<uint32_t>(BN >> 3) << 17) |
+                                     (static_cast<uint32_t>(256 >> 4) << 24);
+  static_assert(kSfTmemCol + kStages * kSfCols <= kTmemCols, "TMEM budget");
+  static_assert(kSmemBytes <= 227 * 1024, "shared memory budget");
+};
+
+template <class C>
+__global__ void __launch_bounds__(C::kThreads, 1)
+    nvfp4_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_constant__ CUtensorMap tmap_b,
+                           const __grid_constant__ CUtensorMap tmap_sfa, const __grid_constant__ CUtensorMap tmap_sfb,
+                           const __grid_constant__ CUtensorMap tmap_out, const GemmArgs args) {
+  constexpr int BN = C::BN;
+  constexpr int kStages = C::kStages;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* sA = smem;
+  uint8_t* sB = sA + kStages * C::kTileBytesA;
+  uint8_t* sEpi = sB + kStages * C::kTileBytesB;
+  uint8_t* sSFA = sEpi + C::kEpiWarps * kEpiBufBytes;
+  uint8_t* sSFB = sSFA + kStages * C::kSfaBytes;
+  uint64_t* full = reinterpret_cast<uint64_t*>(sSFB + kStages * C::kSfbBytes);
+  uint64_t* empty = full + kStages;
+  uint64_t* sfready = empty + kStages;
+  uint64_t* tfull = sfready + kStages;
+  uint64_t* tempty = tfull + 1;
+  uint64_t* drain = tempty + 1;
+  uint64_t* drain_cp = drain + 1;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain_cp + 1);
+  __shared__ volatile int abort_flag;
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int kblocks = args.K / BK;
+  const int kgroups = args.K / 64;
+  const uint32_t rank = cluster_ctarank();
+  const bool leader = rank == 0;
+  const int msup = (args.tiles_m + 1) / 2;
+  const int total_units = msup * args.tiles_n;
+  const int pair_id = blockIdx.x / 2, n_pairs = gridDim.x / 2;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(&full[s], 1);  // leader: its expect_tx covers both CTAs' bytes; unused in the peer
+      mbar_init(&empty[s], 1);
+      mbar_init(&sfready[s], C::kCopyWarps);  // one commit per copy warp
+    }
+    mbar_init(tfull, 1);
+    mbar_init(tempty, 2 * C::kEpiWarps);
+    mbar_init(drain, 1);
+    mbar_init(drain_cp, C::kCopyWarps);
+    abort_flag = 0;
+    fence_mbar_init();
+    prefetch_tmap(&tmap_a);
+    prefetch_tmap(&tmap_b);
+    prefetch_tmap(&tmap_sfa);
+    prefetch_tmap(&tmap_sfb);
+    prefetch_tmap(&tmap_out);
+  }
+  if (warp == 1) {
+    tmem_alloc_pair(tmem_slot, kTmemCols);
+    tmem_relinquish_pair();
+  }
+  tc_fence_before();
+  cluster_sync_all();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  auto fail = [&]() {
+    set_status(args.status, NVFP4_ERR_TIMEOUT);
+    abort_flag = 1;
+  };
+
+  if (warp == 0 && lane == 0) {
+    // ------------------------------------------------------ TMA producer ---
+    int stage = 0;
+    uint32_t phase = 0;
+    uint32_t issued_parity[kStages];
+    bool issued[kStages];
+    for (int s = 0; s < kStages; ++s) issued[s] = false;
+    for (int u = pair_id; u < total_units && !abort_flag; u += n_pairs) {
+      const int nb = u / msup;
+      const int mb = min((u % msup) * 2 + static_cast<int>(rank), args.tiles_m - 1);  // a spare CTA redoes the last tile
+      // Scale atoms through a [bytes / 256, 256] view: one (128-row tile,
+      // k-block) group of four 512-byte atoms is 8 rows of that view.
+      const int sfa_row = mb * kgroups * 2;
+      const int sfb_row = nb * 2 * kgroups * 2;
+      for (int kb = 0; kb < kblocks; ++kb) {
+        if (!mbar_wait_bounded(&empty[stage], phase ^ 1u, &abort_flag)) { fail(); break; }
+        uint8_t* a_dst = sA + stage * C::kTileBytesA;
+        uint8_t* b_dst = sB + stage * C::kTileBytesB;
+        uint8_t* sfa_dst = sSFA + stage * C::kSfaBytes;
+        uint8_t* sfb_dst = sSFB + stage * C::kSfbBytes;
+        const int kx = kb * (BK / 2), b_row = nb * BN + static_cast<int>(rank) * 128;
+        if (leader) {
+          mbar_arrive_expect_tx(&full[stage], 2 * C::kStageBytes);  // both CTAs' loads land on this barrier
+          tma_load_2d(a_dst, &tmap_a, &full[stage], kx, mb * BM);
+          tma_load_2d(b_dst, &tmap_b, &full[stage], kx, b_row);
+          tma_load_2d(sfa_dst, &tmap_sfa, &full[stage], 0, sfa_row + kb * 8);
+          tma_load_2d(sfb_dst, &tmap_sfb, &full[stage], 0, sfb_row + kb * 8);
+          tma_load_2d(sfb_dst + C::kSfaBytes, &tmap_sfb, &full[stage], 0, sfb_row + kgroups * 2 + kb * 8);
+        } else {
+          tma_load_2d_to_leader(a_dst, &tmap_a, &full[stage], kx, mb * BM);
+          tma_load_2d_to_leader(b_dst, &tmap_b, &full[stage], kx, b_row);
+          tma_load_2d_to_leader(sfa_dst, &tmap_sfa, &full[stage], 0, sfa_row + kb * 8);
+          tma_load_2d_to_leader(sfb_dst, &tmap_sfb, &full[stage], 0, sfb_row + kb * 8);
+          tma_load_2d_to_leader(sfb_dst + C::kSfaBytes, &tmap_sfb, &full[stage], 0, sfb_row + kgroups * 2 + kb * 8);
+        }
+        issued[stage] = true;
+        issued_parity[stage] = phase;
+        if (++stage == kStages) { stage = 0; phase ^= 1u; }
+      }
+    }
+    if (abort_flag && leader) {
+      // Both CTAs' copies complete on the leader's barriers: wait for them here.
+      for (int s = 0; s < kStages; ++s)
+        if (issued[s]) mbar_wait_bounded(&full[s], issued_parity[s], nullptr);
+    }
+  } else if (warp == 1 && lane == 0 && leader) {
+    // ------------------------------------------------ MMA issuer (leader) ---
+    int stage = 0;
+    uint32_t phase = 0;
+    int local = 0;
+    const uint32_t sA0 = smem_u32(sA), sB0 = smem_u32(sB);
+    for (int u = pair_id; u < total_units && !abort_flag; u += n_pairs, ++local) {
+      if (!mbar_wait_bounded(tempty, (local & 1) ^ 1u, &abort_flag)) { fail(); break; }
+      tc_fence_after();
+      bool ok = true;
+      for (int kb = 0; kb < kblocks; ++kb) {
+        if (!mbar_wait_bounded(&sfready[stage], phase, &abort_flag)) { fail(); ok = false; break; }
+        tc_fence_after();
+        const uint32_t sfa_col = tmem + C::kSfTmemCol + stage * C::kSfCols;
+        const uint32_t sfb_col = sfa_col + 16;
+#pragma unroll
+        for (int kk = 0; kk < 4; ++kk)
+          mma_fp4_pair(tmem, desc_sw128(sA0 + stage * C::kTileBytesA + kk * 32),
+                       desc_sw128(sB0 + stage * C::kTileBytesB + kk * 32), C::kIdesc, sfa_col + kk * 4,
+                       sfb_col + kk * 8, (kb | kk) != 0);
+        tc_commit_pair(&empty[stage], 0x3);
+        if (++stage == kStages) { stage = 0; phase ^= 1u; }
+      }
+      if (!ok) break;
+      tc_commit_pair(tfull, 0x3);
+    }
+    tc_commit_pair(drain, 0x1);
+    mbar_wait_bounded(drain, 0, nullptr);
+  } else if (warp >= 2 && warp < 2 + C::kCopyWarps && lane == 0 && leader) {
+    // ------------------------------------- leader: block scales -> TMEM ---
+    // The K=64 steps of a stage are spread over the copy warps: copies issued
+    // from different warps proceed concurrently, copies from one thread do not.
+    constexpr int kPerWarp = 4 / C::kCopyWarps;
+    const int kk0 = (warp - 2) * kPerWarp;
+    int stage = 0;
+    uint32_t phase = 0;
+    const uint32_t sSFA0 = smem_u32(sSFA), sSFB0 = smem_u32(sSFB);
+    for (int u = pair_id; u < total_units && !abort_flag; u += n_pairs) {
+      bool ok = true;
+      for (int kb = 0; kb < kblocks; ++kb) {
+        if (!mbar_wait_bounded(&full[stage], phase, &abort_flag)) { fail(); ok = false; break; }
+        {
+          tc_fence_after();
+          const uint32_t sfa_col = tmem + C::kSfTmemCol + stage * C::kSfCols;
+          const uint32_t sfb_col = sfa_col + 16;
+#pragma unroll
+          for (int kk = kk0; kk < kk0 + kPerWarp; ++kk) {
+            copy_sf_to_tmem_pair(sfa_col + kk * 4, desc_sf(sSFA0 + stage * C::kSfaBytes + kk * 512));
+#pragma unroll
+            for (int j = 0; j < 2; ++j)
+              copy_sf_to_tmem_pair(sfb_col + kk * 8 + j * 4,
+                                   desc_sf(sSFB0 + stage * C::kSfbBytes + j * C::kSfaBytes + kk * 512));
+          }
+          tc_commit_pair(&sfready[stage], 0x1);
+        }
+        if (++stage == kStages) { stage = 0; phase ^= 1u; }
+      }
+      if (!ok) break;
+    }
+    tc_commit_pair(drain_cp, 0x1);
+    mbar_wait_bounded(drain_cp, 0, nullptr);
+  } else if (warp >= 2 + C::kCopyWarps) {
+    // --------------------------------------------------------- epilogue ---
+    constexpr int kEpi0 = 2 + C::kCopyWarps;
+    const int quarter = warp & 3;
+    const int colbase = ((warp - kEpi0) >> 2) * 128;
+    uint8_t* buf_ptr = sEpi + (warp - kEpi0) * kEpiBufBytes;
+    const uint32_t buf = smem_u32(buf_ptr);
+    const float scale = __fmul_rn(__ldg(args.ga), __ldg(args.gb));
+    int local = 0;
+    for (int u = pair_id; u < total_units; u += n_pairs, ++local) {
+      const int nb = u / msup;
+      const int mb = (u % msup) * 2 + static_cast<int>(rank);  // mb >= tiles_m: nothing is stored
+      int ok = 1;
+      if (lane == 0) {
+        ok = !abort_flag && mbar_wait_bounded(tfull, local & 1, &abort_flag);
+        if (!ok && !abort_flag) fail();
+      }
+      if (!__shfl_sync(0xffffffffu, ok, 0)) break;
+      tc_fence_after();
+      uint32_t r[128];
+      const uint32_t taddr = tmem + (static_cast<uint32_t>(quarter * 32) << 16) + colbase;
+#pragma unroll
+      for (int c = 0; c < 4; ++c) tmem_ld32(taddr + c * 32, r + 32 * c);
+      tmem_ld_wait();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive_cluster(tempty, 0);
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {
+        if (lane == 0) bulk_wait_read_all();
+        __syncwarp();
+#pragma unroll
+        for (int c = 0; c < 8; ++c) {
+          const uint32_t* v = r + 64 * h + 8 * c;
+          st_shared_v4(buf + lane * 128 + ((c ^ (lane & 7)) << 4),
+                       pack_bf16x2(__uint_as_float(v[0]) * scale, __uint_as_float(v[1]) * scale),
+                       pack_bf16x2(__uint_as_float(v[2]) * scale, __uint_as_float(v[3]) * scale),
+                       pack_bf16x2(__uint_as_float(v[4]) * scale, __uint_as_float(v[5]) * scale),
+                       pack_bf16x2(__uint_as_float(v[6]) * scale, __uint_as_float(v[7]) * scale));
+        }
+        fence_proxy_async_smem();
+        __syncwarp();
+        const int x = nb * BN + colbase + h * kEpiCols, y = mb * BM + quarter * 32;
+        if (lane == 0 && x < args.N && y < args.M) {
+          tma_store_2d(&tmap_out, buf_ptr, x, y);
+          bulk_commit_group();
+        }
+      }
+    }
+    if (lane == 0) bulk_wait_all();
+  }
+
+  tc_fence_before();
+  cluster_sync_all();
+  tc_fence_after();
+  if (warp == 1) tmem_dealloc_pair(tmem, kTmemCols);
+}
+
 // ------------------------------------------------------------------- host ---
 
 PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
@@ -397,6 +711,22 @@ bool make_code_map(CUtensorMap* map, const uint8_t* base, int64_t rows, int64_t 
   cuuint32_t estr[2] = {1, 1};
   CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<uint8_t*>(base), dims, strides, box, estr,
                    CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
+// MMA-layout block scales of a [rows, K] operand viewed as [bytes / 256, 256]
+// bytes; a box of 8 rows is one (128-row tile, k-block) group of four atoms.
+bool make_scale_map(CUtensorMap* map, const uint8_t* base, int64_t rows, int64_t K) {
+  auto enc = tensor_map_encoder();
+  if (!enc) return false;
+  const int64_t bytes = ((rows + 127) / 128) * 128 * (K / 16);
+  cuuint64_t dims[2] = {256, static_cast<cuuint64_t>(bytes / 256)};
+  cuuint64_t strides[1] = {256};
+  cuuint32_t box[2] = {256, 8};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<uint8_t*>(base), dims, strides, box, estr,
+                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                    CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return r == CUDA_SUCCESS;
 }
@@ -495,11 +825,90 @@ nvfp4_status launch(const uint8_t* a_codes, const uint8_t* a_scales, const float
   return launch_status();
 }
 
+template <class C>
+int resident_pairs() {
+  static std::mutex mu;
+  static std::map<int, int> cache;
+  int d = 0;
+  if (cudaGetDevice(&d) != cudaSuccess) return 0;
+  std::lock_guard<std::mutex> lock(mu);
+  auto it = cache.find(d);
+  if (it != cache.end()) return it->second;
+  if (cudaFuncSetAttribute(nvfp4_gemm_pair_kernel<C>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           static_cast<int>(C::kSmemBytes)) != cudaSuccess)
+    return 0;
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.gridDim = dim3(2 * (sm_count() / 2), 1, 1);
+  cfg.blockDim = dim3(C::kThreads, 1, 1);
+  cfg.dynamicSmemBytes = C::kSmemBytes;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  int clusters = 0;
+  if (cudaOccupancyMaxActiveClusters(&clusters, nvfp4_gemm_pair_kernel<C>, &cfg) != cudaSuccess || clusters <= 0) {
+    cudaGetLastError();
+    return 0;
+  }
+  cache[d] = clusters;
+  return clusters;
+}
+
+template <class C>
+nvfp4_status launch_pair(const uint8_t* a_codes, const uint8_t* a_scales, const float* g_a, const uint8_t* w_codes,
+                         const uint8_t* w_scales, const float* g_w, int64_t M, int64_t N, int64_t K, void* out_bf16,
+                         int64_t ldo, cudaStream_t stream) {
+  const int64_t tiles_m = (M + BM - 1) / BM, tiles_n = N / C::BN;
+  const int64_t units = ((tiles_m + 1) / 2) * tiles_n;
+  if (units >= (1ll << 31)) return NVFP4_ERR_SHAPE;
+  CUtensorMap ma, mb, msa, msb, mo;
+  if (!make_code_map(&ma, a_codes, M, K, BM) || !make_code_map(&mb, w_codes, N, K, 128) ||
+      !make_scale_map(&msa, a_scales, M, K) || !make_scale_map(&msb, w_scales, N, K) ||
+      !make_out_map(&mo, out_bf16, M, N, ldo))
+    return NVFP4_ERR_CUDA;
+  const int pairs_max = resident_pairs<C>();
+  if (pairs_max <= 0) return NVFP4_ERR_CUDA;
+  GemmArgs args;
+  args.sfa = a_scales;
+  args.sfb = w_scales;
+  args.ga = g_a;
+  args.gb = g_w;
+  args.M = static_cast<int>(M);
+  args.N = static_cast<int>(N);
+  args.K = static_cast<int>(K);
+  args.tiles_m = static_cast<int>(tiles_m);
+  args.tiles_n = static_cast<int>(tiles_n);
+  args.status = status_word_dev();
+  const int pairs = static_cast<int>(units < pairs_max ? units : pairs_max);
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.gridDim = dim3(2 * pairs, 1, 1);
+  cfg.blockDim = dim3(C::kThreads, 1, 1);
+  cfg.dynamicSmemBytes = C::kSmemBytes;
+  cfg.stream = stream;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  if (cudaLaunchKernelEx(&cfg, nvfp4_gemm_pair_kernel<C>, ma, mb, msa, msb, mo, args) != cudaSuccess)
+    return NVFP4_ERR_CUDA;
+  count_launches(1);
+  return launch_status();
+}
+
 #ifndef NVFP4_GEMM_BN
 #define NVFP4_GEMM_BN 0  // 0: choose per shape
 #endif
 #ifndef NVFP4_GEMM_CM
 #define NVFP4_GEMM_CM 0  // 0: choose per shape
+#endif
+#ifndef NVFP4_GEMM_PAIR
+#define NVFP4_GEMM_PAIR 1  // 0: never use the CTA-pair kernel
 #endif
 
 }  // namespace
@@ -523,7 +932,8 @@ NVFP4_API nvfp4_status nvfp4_linear(const uint8_t* a_codes, const uint8_t* a_sca
   // independent CTAs on these shapes (the cluster waits for its slowest CTA),
   // so clusters are off by default; the multicast path stays selectable.
   const int cm = NVFP4_GEMM_CM ? NVFP4_GEMM_CM : 1;
-  (void)tiles_m;
+  if (NVFP4_GEMM_PAIR && N % 256 == 0 && tiles_m >= 2)
+    return launch_pair<PairCfg<5>>(a_codes, a_scales, g_a, w_codes, w_scales, g_w, M, N, K, out_bf16, ldo, s);
 #define NVFP4_LAUNCH(BN_, ST_, CM_) \
   return launch<Cfg<BN_, ST_, CM_>>(a_codes, a_scales, g_a, w_codes, w_scales, g_w, M, N, K, out_bf16, ldo, s)
   if (bn == 256) {
