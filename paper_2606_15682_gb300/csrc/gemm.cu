@@ -37,6 +37,9 @@ namespace {
 #ifndef NVFP4_GEMM_COPY_WARPS
 #define NVFP4_GEMM_COPY_WARPS 2
 #endif
+#ifndef NVFP4_GEMM_PAIR_STAGES
+#define NVFP4_GEMM_PAIR_STAGES 5
+#endif
 
 constexpr int BM = 128;
 constexpr int BK = 256;  // elements per k-block = 128 bytes per row
@@ -471,10 +474,11 @@ __global__ void __launch_bounds__(C::kThreads, 1)
   uint8_t* sEpi = sB + kStages * C::kTileBytesB;
   uint8_t* sSFA = sEpi + C::kEpiWarps * kEpiBufBytes;
   uint8_t* sSFB = sSFA + kStages * C::kSfaBytes;
-  uint64_t* full = reinterpret_cast<uint64_t*>(sSFB + kStages * C::kSfbBytes);
+  uint64_t* full = reinterpret_cast<uint64_t*>(sSFB + kStages * C::kSfbBytes);  // codes landed
   uint64_t* empty = full + kStages;
   uint64_t* sfready = empty + kStages;
-  uint64_t* tfull = sfready + kStages;
+  uint64_t* sffull = sfready + kStages;  // block scales landed (loaded first, so copies overlap the codes)
+  uint64_t* tfull = sffull + kStages;
   uint64_t* tempty = tfull + 1;
   uint64_t* drain = tempty + 1;
   uint64_t* drain_cp = drain + 1;
@@ -495,6 +499,7 @@ __global__ void __launch_bounds__(C::kThreads, 1)
       mbar_init(&full[s], 1);  // leader: its expect_tx covers both CTAs' bytes; unused in the peer
       mbar_init(&empty[s], 1);
       mbar_init(&sfready[s], C::kCopyWarps);  // one commit per copy warp
+      mbar_init(&sffull[s], 1);
     }
     mbar_init(tfull, 1);
     mbar_init(tempty, 2 * C::kEpiWarps);
@@ -543,19 +548,22 @@ __global__ void __launch_bounds__(C::kThreads, 1)
         uint8_t* sfa_dst = sSFA + stage * C::kSfaBytes;
         uint8_t* sfb_dst = sSFB + stage * C::kSfbBytes;
         const int kx = kb * (BK / 2), b_row = nb * BN + static_cast<int>(rank) * 128;
+        constexpr uint32_t kSfStage = C::kSfaBytes + C::kSfbBytes;
         if (leader) {
-          mbar_arrive_expect_tx(&full[stage], 2 * C::kStageBytes);  // both CTAs' loads land on this barrier
+          // Both CTAs' loads land on the leader's barriers.
+          mbar_arrive_expect_tx(&sffull[stage], 2 * kSfStage);
+          mbar_arrive_expect_tx(&full[stage], 2 * (C::kStageBytes - kSfStage));
+          tma_load_2d(sfa_dst, &tmap_sfa, &sffull[stage], 0, sfa_row + kb * 8);
+          tma_load_2d(sfb_dst, &tmap_sfb, &sffull[stage], 0, sfb_row + kb * 8);
+          tma_load_2d(sfb_dst + C::kSfaBytes, &tmap_sfb, &sffull[stage], 0, sfb_row + kgroups * 2 + kb * 8);
           tma_load_2d(a_dst, &tmap_a, &full[stage], kx, mb * BM);
           tma_load_2d(b_dst, &tmap_b, &full[stage], kx, b_row);
-          tma_load_2d(sfa_dst, &tmap_sfa, &full[stage], 0, sfa_row + kb * 8);
-          tma_load_2d(sfb_dst, &tmap_sfb, &full[stage], 0, sfb_row + kb * 8);
-          tma_load_2d(sfb_dst + C::kSfaBytes, &tmap_sfb, &full[stage], 0, sfb_row + kgroups * 2 + kb * 8);
         } else {
+          tma_load_2d_to_leader(sfa_dst, &tmap_sfa, &sffull[stage], 0, sfa_row + kb * 8);
+          tma_load_2d_to_leader(sfb_dst, &tmap_sfb, &sffull[stage], 0, sfb_row + kb * 8);
+          tma_load_2d_to_leader(sfb_dst + C::kSfaBytes, &tmap_sfb, &sffull[stage], 0, sfb_row + kgroups * 2 + kb * 8);
           tma_load_2d_to_leader(a_dst, &tmap_a, &full[stage], kx, mb * BM);
           tma_load_2d_to_leader(b_dst, &tmap_b, &full[stage], kx, b_row);
-          tma_load_2d_to_leader(sfa_dst, &tmap_sfa, &full[stage], 0, sfa_row + kb * 8);
-          tma_load_2d_to_leader(sfb_dst, &tmap_sfb, &full[stage], 0, sfb_row + kb * 8);
-          tma_load_2d_to_leader(sfb_dst + C::kSfaBytes, &tmap_sfb, &full[stage], 0, sfb_row + kgroups * 2 + kb * 8);
         }
         issued[stage] = true;
         issued_parity[stage] = phase;
@@ -565,7 +573,10 @@ __global__ void __launch_bounds__(C::kThreads, 1)
     if (abort_flag && leader) {
       // Both CTAs' copies complete on the leader's barriers: wait for them here.
       for (int s = 0; s < kStages; ++s)
-        if (issued[s]) mbar_wait_bounded(&full[s], issued_parity[s], nullptr);
+        if (issued[s]) {
+          mbar_wait_bounded(&sffull[s], issued_parity[s], nullptr);
+          mbar_wait_bounded(&full[s], issued_parity[s], nullptr);
+        }
     }
   } else if (warp == 1 && lane == 0 && leader) {
     // ------------------------------------------------ MMA issuer (leader) ---
@@ -578,7 +589,8 @@ __global__ void __launch_bounds__(C::kThreads, 1)
       tc_fence_after();
       bool ok = true;
       for (int kb = 0; kb < kblocks; ++kb) {
-        if (!mbar_wait_bounded(&sfready[stage], phase, &abort_flag)) { fail(); ok = false; break; }
+        if (!mbar_wait_bounded(&full[stage], phase, &abort_flag) ||
+            !mbar_wait_bounded(&sfready[stage], phase, &abort_flag)) { fail(); ok = false; break; }
         tc_fence_after();
         const uint32_t sfa_col = tmem + C::kSfTmemCol + stage * C::kSfCols;
         const uint32_t sfb_col = sfa_col + 16;
@@ -607,7 +619,7 @@ __global__ void __launch_bounds__(C::kThreads, 1)
     for (int u = pair_id; u < total_units && !abort_flag; u += n_pairs) {
       bool ok = true;
       for (int kb = 0; kb < kblocks; ++kb) {
-        if (!mbar_wait_bounded(&full[stage], phase, &abort_flag)) { fail(); ok = false; break; }
+        if (!mbar_wait_bounded(&sffull[stage], phase, &abort_flag)) { fail(); ok = false; break; }
         {
           tc_fence_after();
           const uint32_t sfa_col = tmem + C::kSfTmemCol + stage * C::kSfCols;
@@ -933,7 +945,7 @@ NVFP4_API nvfp4_status nvfp4_linear(const uint8_t* a_codes, const uint8_t* a_sca
   // so clusters are off by default; the multicast path stays selectable.
   const int cm = NVFP4_GEMM_CM ? NVFP4_GEMM_CM : 1;
   if (NVFP4_GEMM_PAIR && N % 256 == 0 && tiles_m >= 2)
-    return launch_pair<PairCfg<5>>(a_codes, a_scales, g_a, w_codes, w_scales, g_w, M, N, K, out_bf16, ldo, s);
+    return launch_pair<PairCfg<NVFP4_GEMM_PAIR_STAGES>>(a_codes, a_scales, g_a, w_codes, w_scales, g_w, M, N, K, out_bf16, ldo, s);
 #define NVFP4_LAUNCH(BN_, ST_, CM_) \
   return launch<Cfg<BN_, ST_, CM_>>(a_codes, a_scales, g_a, w_codes, w_scales, g_w, M, N, K, out_bf16, ldo, s)
   if (bn == 256) {
