@@ -183,7 +183,9 @@ nvfp4_status kv_append_nvfp4(const nvfp4_kv_cache* cache, const void* k_bf16, co
  *   out_bf16 : [batch, num_q_heads, head_dim] bf16.
  *   workspace: at least decode_attention_nvfp4_workspace_size(...) bytes, 16-B
  *              aligned; contents on entry are ignored.
- * num_q_heads % num_kv_heads == 0 and num_q_heads/num_kv_heads <= 8 (SHAPE).
+ * num_q_heads % num_kv_heads == 0, num_q_heads/num_kv_heads <= 8 and an even
+ * capacity (scale rows are streamed in 16-byte units) are required (SHAPE);
+ * the four cache arrays must be 16-B aligned (ALIGN).
  * A sequence with seq_lens[b] == 0 gets zeros; seq_lens[b] > capacity sets
  * CAPACITY on the device and is clamped to capacity.
  */

@@ -75,3 +75,5 @@ def test_kv_and_attention_validation():
     assert L.decode_attention_nvfp4(ctypes.byref(cache()), p, 18, ctypes.c_float(0.1), p, p, 1 << 30, s) == 2  # group 9
     assert L.decode_attention_nvfp4(ctypes.byref(cache()), p, 4, ctypes.c_float(0.1), p, p, ws - 16, s) == 2
     assert L.decode_attention_nvfp4(ctypes.byref(cache()), p, 4, ctypes.c_float(-1.0), p, p, ws, s) == 1
+    ws_odd = N.decode_attention_nvfp4_workspace_size(2, 4, 63)
+    assert L.decode_attention_nvfp4(ctypes.byref(cache(capacity=63)), p, 4, ctypes.c_float(0.1), p, p, ws_odd, s) == 2
