@@ -194,6 +194,38 @@ nvfp4_status decode_attention_nvfp4(const nvfp4_kv_cache* cache, const void* q_b
                                     int32_t num_q_heads, float softmax_scale, void* out_bf16,
                                     void* workspace, size_t workspace_bytes, void* stream);
 
+/*
+ * Decode attention without a caller workspace (no counterpart in the paper).
+ *
+ * Same computation and arguments as decode_attention_nvfp4, but the split-KV
+ * partials go to a scratch array that the library itself holds in device
+ * memory, so the call allocates nothing and needs no workspace pointer.  It is
+ * for callers that cannot obtain device memory at the point of the call: a
+ * runtime that reserves all GPU memory at start-up and forbids later
+ * allocations, a plug-in that is handed device pointers by a host framework
+ * that owns the allocator, or a code path where an allocation would
+ * synchronize the device or break a latency budget.
+ *
+ * Limits and sharing:
+ *   - The scratch holds NVFP4_ATTN_STATIC_SCRATCH_BYTES (24 MiB); a problem
+ *     whose decode_attention_nvfp4_workspace_size exceeds it returns SHAPE
+ *     without launching anything.  Every GPU that loads the library keeps
+ *     this array until the process exits.
+ *   - All calls share the one array and it keeps the last call's contents;
+ *     every value a call reads is written earlier in the same call, so no
+ *     clearing is needed.  Calls that can overlap on the GPU (different
+ *     streams, or concurrent host threads) race on the scratch and must be
+ *     serialized by the caller.
+ *   - The first call on a device looks up the device address of the array
+ *     (a one-time host-side query); make that first call before capturing
+ *     stream work into a CUDA graph.
+ * Errors: as decode_attention_nvfp4.
+ */
+#define NVFP4_ATTN_STATIC_SCRATCH_BYTES (24u << 20)
+nvfp4_status decode_attention_nvfp4_static_scratch(const nvfp4_kv_cache* cache, const void* q_bf16,
+                                                   int32_t num_q_heads, float softmax_scale, void* out_bf16,
+                                                   void* stream);
+
 /* Synchronize `stream`, copy the device status word of the current device to
  * *status_host (an nvfp4_status value) and clear it. */
 nvfp4_status nvfp4_get_device_status(int32_t* status_host, void* stream);

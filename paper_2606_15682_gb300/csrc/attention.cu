@@ -519,3 +519,88 @@ NVFP4_API nvfp4_status decode_attention_nvfp4(const nvfp4_kv_cache* cache, const
   count_launches(2);
   return launch_status();
 }
+
+// ---------------------------------------------------------------------------
+// Decode attention for callers that cannot allocate device memory.  The
+// split-KV partials live in one file-scope device array instead of a caller
+// workspace; every GPU that loads the library holds it until the process
+// exits, and all calls share it.
+namespace nvfp4 {
+namespace {
+
+static __device__ __align__(256) float g_attn_static_scratch[NVFP4_ATTN_STATIC_SCRATCH_BYTES / sizeof(float)];
+
+// Device address of the static scratch for the current device, looked up once
+// per device with that device current.  Host code must not hand the symbol
+// itself to a kernel: on the host it is only a stand-in for the device array.
+float* attn_static_scratch_dev() {
+  static std::mutex mu;
+  static std::map<int, float*> addr;
+  int d = 0;
+  if (cudaGetDevice(&d) != cudaSuccess) return nullptr;
+  std::lock_guard<std::mutex> lock(mu);
+  auto it = addr.find(d);
+  if (it != addr.end()) return it->second;
+  float* p = nullptr;
+  if (cudaGetSymbolAddress(reinterpret_cast<void**>(&p), g_attn_static_scratch) != cudaSuccess || !p) return nullptr;
+  addr[d] = p;
+  return p;
+}
+
+}  // namespace
+}  // namespace nvfp4
+
+NVFP4_API nvfp4_status decode_attention_nvfp4_static_scratch(const nvfp4_kv_cache* cache, const void* q_bf16,
+                                                             int32_t num_q_heads, float softmax_scale,
+                                                             void* out_bf16, void* stream) {
+  if (!cache || !q_bf16 || !out_bf16 || !cache->seq_lens) return NVFP4_ERR_INVALID_ARG;
+  if (!cache->k_codes || !cache->k_scales || !cache->v_codes || !cache->v_scales) return NVFP4_ERR_INVALID_ARG;
+  if (!(cache->k_gscale > 0.0f && cache->k_gscale <= FLT_MAX) || !(cache->v_gscale > 0.0f && cache->v_gscale <= FLT_MAX) ||
+      !(softmax_scale > 0.0f && softmax_scale <= FLT_MAX))
+    return NVFP4_ERR_INVALID_ARG;
+  if (cache->head_dim != kD || cache->batch <= 0 || cache->num_kv_heads <= 0 || cache->capacity <= 0 ||
+      cache->capacity % 2 || num_q_heads <= 0 || num_q_heads % cache->num_kv_heads ||
+      num_q_heads / cache->num_kv_heads > 8)
+    return NVFP4_ERR_SHAPE;
+  if (static_cast<int64_t>(cache->batch) > 65535 || num_q_heads > 65535) return NVFP4_ERR_SHAPE;
+  const int64_t n_items = static_cast<int64_t>(cache->batch) * cache->num_kv_heads * splits_for(cache->capacity);
+  if (n_items >= (1ll << 31)) return NVFP4_ERR_SHAPE;
+  // The partials must fit in the static scratch; larger problems are refused.
+  if (decode_attention_nvfp4_workspace_size(cache->batch, num_q_heads, cache->capacity) >
+      NVFP4_ATTN_STATIC_SCRATCH_BYTES)
+    return NVFP4_ERR_SHAPE;
+  if (!aligned(q_bf16, 16) || !aligned(out_bf16, 16) || !aligned(cache->k_codes, 16) ||
+      !aligned(cache->v_codes, 16) || !aligned(cache->k_scales, 16) || !aligned(cache->v_scales, 16))
+    return NVFP4_ERR_ALIGN;
+  float* scratch = attn_static_scratch_dev();
+  if (!scratch) return NVFP4_ERR_CUDA;
+  const int ctas_max = resident_ctas();
+  if (ctas_max <= 0) return NVFP4_ERR_CUDA;
+  Params prm;
+  prm.k_codes = cache->k_codes;
+  prm.k_scales = cache->k_scales;
+  prm.v_codes = cache->v_codes;
+  prm.v_scales = cache->v_scales;
+  prm.seq_lens = cache->seq_lens;
+  prm.q = static_cast<const uint16_t*>(q_bf16);
+  prm.status = status_word_dev();
+  prm.hkv = cache->num_kv_heads;
+  prm.capacity = cache->capacity;
+  prm.hq = num_q_heads;
+  prm.group = num_q_heads / cache->num_kv_heads;
+  prm.n_splits = splits_for(cache->capacity);
+  prm.n_items = static_cast<int>(n_items);
+  prm.logit_mult = softmax_scale * cache->k_gscale * kLog2e;
+  // Every record the combine kernel reads is written by the partial kernel of
+  // the same call, so nothing left from an earlier call needs clearing.
+  prm.o_ws = scratch;
+  prm.ml_ws = prm.o_ws + static_cast<size_t>(cache->batch) * num_q_heads * prm.n_splits * kD;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const int grid = static_cast<int>(n_items < ctas_max ? n_items : ctas_max);
+  attn_partial_kernel<<<grid, kThreads, kSmemBytes, s>>>(prm);
+  attn_combine_kernel<<<dim3(num_q_heads, cache->batch), kD, 0, s>>>(prm.o_ws, prm.ml_ws, prm.n_splits,
+                                                                     cache->v_gscale,
+                                                                     static_cast<uint16_t*>(out_bf16));
+  count_launches(2);
+  return launch_status();
+}

@@ -56,6 +56,7 @@ _linear = _sig("nvfp4_linear", [_p, _p, _p, _p, _p, _p, _i64, _i64, _i64, _p, _i
 _kv_append = _sig("kv_append_nvfp4", [ctypes.POINTER(KVCacheStruct), _p, _p, _p, _p, _i64, _p, _p])
 _attn_ws = _sig("decode_attention_nvfp4_workspace_size", [_i32, _i32, _i32], _sz)
 _attn = _sig("decode_attention_nvfp4", [ctypes.POINTER(KVCacheStruct), _p, _i32, _f32, _p, _p, _sz, _p])
+_attn_static = _sig("decode_attention_nvfp4_static_scratch", [ctypes.POINTER(KVCacheStruct), _p, _i32, _f32, _p, _p])
 _get_status = _sig("nvfp4_get_device_status", [ctypes.POINTER(_i32), _p])
 _status_string = _sig("nvfp4_status_string", [ctypes.c_int], ctypes.c_char_p)
 _launch_count = _sig("nvfp4_launch_count", [], ctypes.c_uint64)
@@ -135,6 +136,16 @@ def decode_attention_nvfp4(cache, q, softmax_scale, out, workspace, stream=None)
                                            _stream(stream)))
 
 
+ATTN_STATIC_SCRATCH_BYTES = 24 << 20
+
+
+def decode_attention_nvfp4_static_scratch(cache, q, softmax_scale, out, stream=None):
+    """Decode attention whose partials live in the library's own device scratch (no workspace)."""
+    s = cache.struct()
+    _check("decode_attention_nvfp4_static_scratch", _attn_static(ctypes.byref(s), _ptr(q), q.shape[1], softmax_scale,
+                                                                 _ptr(out), _stream(stream)))
+
+
 def nvfp4_get_device_status(stream=None):
     v = _i32(0)
     _check("nvfp4_get_device_status", _get_status(ctypes.byref(v), _stream(stream)))
@@ -172,4 +183,5 @@ class KVCache:
 
 EXPORTED = ["nvfp4_scales_bytes", "nvfp4_tensor_scale", "nvfp4_quantize", "nvfp4_scales_relayout", "nvfp4_linear",
             "kv_append_nvfp4", "decode_attention_nvfp4_workspace_size", "decode_attention_nvfp4",
+            "decode_attention_nvfp4_static_scratch",
             "nvfp4_get_device_status", "nvfp4_status_string", "nvfp4_launch_count"]
