@@ -130,6 +130,18 @@ __device__ __forceinline__ void st_shared_v4(uint32_t addr, uint32_t a, uint32_t
   asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(a), "r"(b), "r"(c), "r"(d) : "memory");
 }
 
+// Work-unit order: units walk the N tiles within groups of kGroupM row
+// super-tiles, so the CTAs running at the same time share a few A and W
+// tiles that stay in L2 instead of streaming all of A for every column.
+constexpr int kGroupM = 8;
+__device__ __forceinline__ void unit_coords(int u, int msup, int tiles_n, int* ms, int* nb) {
+  const int per_group = kGroupM * tiles_n;
+  const int group = u / per_group, r = u - group * per_group;
+  const int rows = min(kGroupM, msup - group * kGroupM);
+  *ms = group * kGroupM + r % rows;
+  *nb = r / rows;
+}
+
 struct GemmArgs {
   const uint8_t* sfa;
   const uint8_t* sfb;
@@ -215,8 +227,9 @@ __global__ void __launch_bounds__(C::kThreads, 1)
     bool issued[kStages];
     for (int s = 0; s < kStages; ++s) issued[s] = false;
     for (int u = cluster_id; u < total_units && !abort_flag; u += n_clusters) {
-      const int nb = u / msup;
-      const int mb = min((u % msup) * CM + static_cast<int>(rank), args.tiles_m - 1);  // spare CTAs redo the last tile
+      int ms, nb;
+      unit_coords(u, msup, args.tiles_n, &ms, &nb);
+      const int mb = min(ms * CM + static_cast<int>(rank), args.tiles_m - 1);  // spare CTAs redo the last tile
       const uint8_t* sfa_tile = args.sfa + (static_cast<size_t>(mb) * kgroups) * 512;
       const uint8_t* sfb_tiles = args.sfb + (static_cast<size_t>(nb) * (BN / 128) * kgroups) * 512;
       for (int kb = 0; kb < kblocks; ++kb) {
@@ -322,8 +335,9 @@ __global__ void __launch_bounds__(C::kThreads, 1)
     const float scale = __fmul_rn(__ldg(args.ga), __ldg(args.gb));
     int local = 0;
     for (int u = cluster_id; u < total_units; u += n_clusters, ++local) {
-      const int nb = u / msup;
-      const int mb = (u % msup) * CM + static_cast<int>(rank);  // spare CTAs (mb >= tiles_m) store nothing
+      int ms, nb;
+      unit_coords(u, msup, args.tiles_n, &ms, &nb);
+      const int mb = ms * CM + static_cast<int>(rank);  // spare CTAs (mb >= tiles_m) store nothing
       const int acc = local % C::kAccBufs;
       const uint32_t acc_phase = (local / C::kAccBufs) & 1;
       // Lane 0 waits and broadcasts, so the warp stays converged for the
@@ -535,8 +549,9 @@ __global__ void __launch_bounds__(C::kThreads, 1)
     bool issued[kStages];
     for (int s = 0; s < kStages; ++s) issued[s] = false;
     for (int u = pair_id; u < total_units && !abort_flag; u += n_pairs) {
-      const int nb = u / msup;
-      const int mb = min((u % msup) * 2 + static_cast<int>(rank), args.tiles_m - 1);  // a spare CTA redoes the last tile
+      int ms, nb;
+      unit_coords(u, msup, args.tiles_n, &ms, &nb);
+      const int mb = min(ms * 2 + static_cast<int>(rank), args.tiles_m - 1);  // a spare CTA redoes the last tile
       // Scale atoms through a [bytes / 256, 256] view: one (128-row tile,
       // k-block) group of four 512-byte atoms is 8 rows of that view.
       const int sfa_row = mb * kgroups * 2;
@@ -650,8 +665,9 @@ __global__ void __launch_bounds__(C::kThreads, 1)
     const float scale = __fmul_rn(__ldg(args.ga), __ldg(args.gb));
     int local = 0;
     for (int u = pair_id; u < total_units; u += n_pairs, ++local) {
-      const int nb = u / msup;
-      const int mb = (u % msup) * 2 + static_cast<int>(rank);  // mb >= tiles_m: nothing is stored
+      int ms, nb;
+      unit_coords(u, msup, args.tiles_n, &ms, &nb);
+      const int mb = ms * 2 + static_cast<int>(rank);  // mb >= tiles_m: nothing is stored
       int ok = 1;
       if (lane == 0) {
         ok = !abort_flag && mbar_wait_bounded(tfull, local & 1, &abort_flag);

@@ -1,9 +1,9 @@
 // a1 tensor scale and a2 NVFP4 quantization (Appendix A format).
 //
-// Both kernels stream bf16 with 128-bit loads, one 8-element chunk per lane
-// per step; a warp covers 256 contiguous elements, so every load and every
-// code store of a warp is one contiguous span.  They are HBM-bound: the
-// quantizer moves 2 B in and 0.5625 B out per element.
+// Both kernels stream bf16 with 128-bit loads.  The tensor-scale reduction
+// takes one 8-element chunk per lane per step; the quantizer one 16-element
+// block per lane.  They are HBM-bound: the quantizer moves 2 B in and
+// 0.5625 B out per element.
 #include <cfloat>
 
 #include "common.cuh"
@@ -62,50 +62,66 @@ __global__ void tensor_scale_finalize(float* g) {
   *g = amax > 0.0f ? __fdiv_rn(amax, 2688.0f) : 1.0f;
 }
 
+// One thread quantizes one 16-element block: two 128-bit loads (the second
+// half of the 32 bytes is in L1 after the first load of the warp), one scale
+// computation, one 64-bit code store.  A warp covers 32 consecutive blocks.
 template <bool kMMA>
-__global__ void __launch_bounds__(kThreads) quantize_kernel(const uint16_t* __restrict__ x, ChunkMap map,
-                                                            uint32_t rows, uint32_t kblocks,
-                                                            const float* __restrict__ g_ptr,
-                                                            uint32_t* __restrict__ codes,
-                                                            uint8_t* __restrict__ scales, int* status) {
+__global__ void __launch_bounds__(kThreads) quantize_kernel(const uint16_t* __restrict__ x, FastDiv kblocks_div,
+                                                            uint32_t total_blocks, int64_t ld, bool dense,
+                                                            uint32_t rows, const float* __restrict__ g_ptr,
+                                                            uint2* __restrict__ codes, uint8_t* __restrict__ scales,
+                                                            int* status) {
   const float g_in = *g_ptr;
   const bool g_ok = g_in > 0.0f && g_in <= FLT_MAX;
   if (!g_ok && blockIdx.x == 0 && threadIdx.x == 0) set_status(status, NVFP4_ERR_INVALID_ARG);
   const float g = g_ok ? g_in : 1.0f;
   const float six_g = __fmul_rn(6.0f, g);
+  const uint32_t kblocks = kblocks_div.d;
+  const uint32_t kgroups = kblocks >> 2;
   const uint32_t lane = threadIdx.x & 31;
   const uint32_t stride = gridDim.x * blockDim.x;
-  const uint32_t kgroups = kblocks >> 2;
 
-  // c0 is warp-uniform, so every lane runs every iteration (the amax shuffle
-  // needs the whole warp); lanes past the end only skip their memory ops.
-  for (uint32_t c0 = blockIdx.x * blockDim.x + (threadIdx.x & ~31u); c0 < map.total; c0 += stride * kUnroll) {
-    uint4 v[kUnroll];
-    int64_t off[kUnroll];
-    uint32_t row[kUnroll], chk[kUnroll];
+  // bidx0 is warp-uniform so every lane takes part in the scale gather.
+  for (uint32_t bidx0 = blockIdx.x * blockDim.x + (threadIdx.x & ~31u); bidx0 < total_blocks; bidx0 += stride * kUnroll) {
+    uint4 v0[kUnroll], v1[kUnroll];
+    uint32_t row[kUnroll], kb[kUnroll];
 #pragma unroll
     for (int u = 0; u < kUnroll; ++u) {
-      const uint32_t c = c0 + u * stride + lane;
-      off[u] = c < map.total ? map.elem(c, &row[u], &chk[u]) : 0;
-      v[u] = c < map.total ? __ldg(reinterpret_cast<const uint4*>(x + off[u])) : make_uint4(0, 0, 0, 0);
+      const uint32_t b = bidx0 + u * stride + lane;
+      row[u] = kblocks_div.div(b);
+      kb[u] = b - row[u] * kblocks;
+      const int64_t off = dense ? static_cast<int64_t>(b) * 16 : static_cast<int64_t>(row[u]) * ld + kb[u] * 16;
+      const uint4* src = reinterpret_cast<const uint4*>(x + off);
+      const bool live = b < total_blocks;
+      v0[u] = live ? __ldg(src) : make_uint4(0, 0, 0, 0);
+      v1[u] = live ? __ldg(src + 1) : make_uint4(0, 0, 0, 0);
     }
 #pragma unroll
     for (int u = 0; u < kUnroll; ++u) {
-      const uint32_t c = c0 + u * stride + lane;
-      float xf[8];
-      unpack_bf16x8(v[u], xf);
-      const float amax_own = __uint_as_float(amax_bits_bf16x8(v[u]) << 16);
-      uint32_t sc;
-      uint32_t packed = quantize8_pair(xf, amax_own, g, six_g, &sc);
-      if (!g_ok) { packed = 0; sc = 0; }
-      if (c < map.total) {
-        codes[c] = packed;  // codes are dense: row pitch cols/2 bytes = 4 bytes per chunk
-        if ((lane & 1) == 0) {
-          const uint32_t kb = chk[u] >> 1;
-          const uint64_t so = kMMA ? mma_scale_offset(row[u], kb, kgroups)
-                                   : static_cast<uint64_t>(row[u]) * kblocks + kb;
-          scales[so] = static_cast<uint8_t>(sc);
-        }
+      const uint32_t b = bidx0 + u * stride + lane;
+      const bool live = b < total_blocks;
+      float xf[16];
+      unpack_bf16x8(v0[u], xf);
+      unpack_bf16x8(v1[u], xf + 8);
+      const float amax = __uint_as_float(max(amax_bits_bf16x8(v0[u]), amax_bits_bf16x8(v1[u])) << 16);
+      const BlockScale bs = block_scale(amax, g, six_g);
+      float q[16];
+#pragma unroll
+      for (int i = 0; i < 16; ++i) q[i] = __fmul_rn(xf[i], bs.mult);
+      uint2 packed = make_uint2(e2m1x8(q), e2m1x8(q + 8));
+      uint32_t sc = bs.code;
+      if (!g_ok) { packed = make_uint2(0, 0); sc = 0; }
+      if (live) codes[b] = packed;
+      if (kMMA) {
+        // Lanes 4j..4j+3 hold the four k-blocks of one MMA scale group (kblocks % 4 == 0,
+        // so a group never straddles rows): assemble them into one 32-bit store.
+        uint32_t w = sc << (8 * (lane & 3));
+        w |= __shfl_xor_sync(0xffffffffu, w, 1);
+        w |= __shfl_xor_sync(0xffffffffu, w, 2);
+        if (live && (lane & 3) == 0)
+          *reinterpret_cast<uint32_t*>(scales + mma_scale_offset(row[u], kb[u], kgroups)) = w;
+      } else if (live) {
+        scales[static_cast<uint64_t>(row[u]) * kblocks + kb[u]] = static_cast<uint8_t>(sc);
       }
     }
   }
@@ -114,8 +130,8 @@ __global__ void __launch_bounds__(kThreads) quantize_kernel(const uint16_t* __re
     const uint32_t padded = (rows + 127u) & ~127u;
     const uint32_t pad = (padded - rows) * kblocks;
     for (uint32_t i = blockIdx.x * blockDim.x + threadIdx.x; i < pad; i += stride) {
-      const uint32_t r = rows + i / kblocks, kb = i % kblocks;
-      scales[mma_scale_offset(r, kb, kgroups)] = 0;
+      const uint32_t r = rows + i / kblocks, k = i % kblocks;
+      scales[mma_scale_offset(r, k, kgroups)] = 0;
     }
   }
 }
@@ -200,17 +216,18 @@ NVFP4_API nvfp4_status nvfp4_quantize(const void* x_bf16, int64_t rows, int64_t 
   if (!g_dev || !codes || !scales) return NVFP4_ERR_INVALID_ARG;
   if (!aligned(codes, 8) || !aligned(g_dev, 4)) return NVFP4_ERR_ALIGN;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  const ChunkMap map = make_map(rows, cols, ld);
   const uint32_t kblocks = static_cast<uint32_t>(cols / 16);
-  const int grid = grid_for(map.total, kThreads * kUnroll);
+  const uint32_t total_blocks = static_cast<uint32_t>(rows * kblocks);
+  const int grid = grid_for(total_blocks, kThreads * kUnroll);
+  const bool dense = (ld == cols);
   if (layout == NVFP4_SCALES_MMA) {
-    quantize_kernel<true><<<grid, kThreads, 0, s>>>(static_cast<const uint16_t*>(x_bf16), map,
-                                                    static_cast<uint32_t>(rows), kblocks, g_dev,
-                                                    reinterpret_cast<uint32_t*>(codes), scales, status_word_dev());
+    quantize_kernel<true><<<grid, kThreads, 0, s>>>(static_cast<const uint16_t*>(x_bf16), FastDiv(kblocks),
+                                                    total_blocks, ld, dense, static_cast<uint32_t>(rows), g_dev,
+                                                    reinterpret_cast<uint2*>(codes), scales, status_word_dev());
   } else {
-    quantize_kernel<false><<<grid, kThreads, 0, s>>>(static_cast<const uint16_t*>(x_bf16), map,
-                                                     static_cast<uint32_t>(rows), kblocks, g_dev,
-                                                     reinterpret_cast<uint32_t*>(codes), scales, status_word_dev());
+    quantize_kernel<false><<<grid, kThreads, 0, s>>>(static_cast<const uint16_t*>(x_bf16), FastDiv(kblocks),
+                                                     total_blocks, ld, dense, static_cast<uint32_t>(rows), g_dev,
+                                                     reinterpret_cast<uint2*>(codes), scales, status_word_dev());
   }
   count_launches(1);
   return launch_status();
