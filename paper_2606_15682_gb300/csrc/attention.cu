@@ -162,6 +162,7 @@ __global__ void __launch_bounds__(kThreads, NVFP4_ATTN_MIN_CTAS) attn_partial_ke
     fence_mbar_init();
   }
   __syncthreads();
+  griddep_wait_and_release();
   if (p.capacity > 0 && blockIdx.x == 0 && threadIdx.x == 0) {
     for (int b = 0; b < p.n_items / (p.n_splits * p.hkv); ++b)
       if (__ldg(p.seq_lens + b) > p.capacity) { set_status(p.status, NVFP4_ERR_CAPACITY); break; }
@@ -418,6 +419,7 @@ __global__ void __launch_bounds__(kThreads, NVFP4_ATTN_MIN_CTAS) attn_partial_ke
 __global__ void __launch_bounds__(kD) attn_combine_kernel(const float* __restrict__ o_ws,
                                                          const float* __restrict__ ml_ws, int n_splits, float gv,
                                                          uint16_t* __restrict__ out) {
+  griddep_wait_and_release();
   const size_t bh = static_cast<size_t>(blockIdx.y) * gridDim.x + blockIdx.x;
   const float* ml = ml_ws + bh * n_splits * 2;
   float M = -INFINITY;
@@ -512,10 +514,11 @@ NVFP4_API nvfp4_status decode_attention_nvfp4(const nvfp4_kv_cache* cache, const
   prm.ml_ws = prm.o_ws + static_cast<size_t>(cache->batch) * num_q_heads * prm.n_splits * kD;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   const int grid = static_cast<int>(n_items < ctas_max ? n_items : ctas_max);
-  attn_partial_kernel<<<grid, kThreads, kSmemBytes, s>>>(prm);
-  attn_combine_kernel<<<dim3(num_q_heads, cache->batch), kD, 0, s>>>(prm.o_ws, prm.ml_ws, prm.n_splits,
-                                                                     cache->v_gscale,
-                                                                     static_cast<uint16_t*>(out_bf16));
+  if (launch_pdl(attn_partial_kernel, dim3(grid), dim3(kThreads), kSmemBytes, s, prm) != cudaSuccess ||
+      launch_pdl(attn_combine_kernel, dim3(num_q_heads, cache->batch), dim3(kD), 0, s,
+                 static_cast<const float*>(prm.o_ws), static_cast<const float*>(prm.ml_ws), prm.n_splits,
+                 cache->v_gscale, static_cast<uint16_t*>(out_bf16)) != cudaSuccess)
+    return NVFP4_ERR_CUDA;
   count_launches(2);
   return launch_status();
 }
@@ -597,10 +600,11 @@ NVFP4_API nvfp4_status decode_attention_nvfp4_static_scratch(const nvfp4_kv_cach
   prm.ml_ws = prm.o_ws + static_cast<size_t>(cache->batch) * num_q_heads * prm.n_splits * kD;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   const int grid = static_cast<int>(n_items < ctas_max ? n_items : ctas_max);
-  attn_partial_kernel<<<grid, kThreads, kSmemBytes, s>>>(prm);
-  attn_combine_kernel<<<dim3(num_q_heads, cache->batch), kD, 0, s>>>(prm.o_ws, prm.ml_ws, prm.n_splits,
-                                                                     cache->v_gscale,
-                                                                     static_cast<uint16_t*>(out_bf16));
+  if (launch_pdl(attn_partial_kernel, dim3(grid), dim3(kThreads), kSmemBytes, s, prm) != cudaSuccess ||
+      launch_pdl(attn_combine_kernel, dim3(num_q_heads, cache->batch), dim3(kD), 0, s,
+                 static_cast<const float*>(prm.o_ws), static_cast<const float*>(prm.ml_ws), prm.n_splits,
+                 cache->v_gscale, static_cast<uint16_t*>(out_bf16)) != cudaSuccess)
+    return NVFP4_ERR_CUDA;
   count_launches(2);
   return launch_status();
 }

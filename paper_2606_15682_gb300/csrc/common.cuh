@@ -8,6 +8,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <utility>
+
 #include "../../include/nvfp4.h"
 
 #define NVFP4_API extern "C" __attribute__((visibility("default")))
@@ -31,7 +33,36 @@ inline nvfp4_status launch_status() {
   return e == cudaSuccess ? NVFP4_OK : NVFP4_ERR_CUDA;
 }
 
+// Launch with programmatic stream serialization: the kernel may be scheduled
+// while the previous kernel in the stream is still finishing; it must call
+// griddep_wait() before touching global memory.
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t stream,
+                       Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
+
 // --------------------------------------------------------------- device ---
+
+// Programmatic dependent launch: wait until the previous kernel in the stream
+// has completed and its memory is visible (a no-op without a programmatic
+// dependency), then let the next kernel begin launching.  Called by every
+// kernel of the library before its first global-memory access, so only
+// prologues (barrier set-up, TMEM allocation) overlap the previous kernel.
+__device__ __forceinline__ void griddep_wait_and_release() {
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
 
 // First error wins; later errors do not overwrite it.
 __device__ __forceinline__ void set_status(int* status, int code) {
@@ -86,6 +117,31 @@ __device__ __forceinline__ bool mbar_wait_bounded(uint64_t* bar, uint32_t parity
   uint64_t t0 = globaltimer_ns();
   for (uint32_t it = 1;; ++it) {
     if (mbar_try_wait(bar, parity)) return true;
+    if ((it & 255u) == 0) {
+      if (abort && *abort) return false;
+      if (globaltimer_ns() - t0 > kWaitLimitNs) return false;
+    }
+  }
+}
+
+// The same for a barrier that threads of another CTA of the cluster arrive on
+// (acquire at cluster scope, pairing with their release.cluster arrivals).
+__device__ __forceinline__ bool mbar_try_wait_cluster(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred p;\n"
+      " mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n"
+      " selp.u32 %0, 1, 0, p;\n}"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+__device__ __forceinline__ bool mbar_wait_bounded_cluster(uint64_t* bar, uint32_t parity, volatile int* abort) {
+  if (mbar_try_wait_cluster(bar, parity)) return true;
+  uint64_t t0 = globaltimer_ns();
+  for (uint32_t it = 1;; ++it) {
+    if (mbar_try_wait_cluster(bar, parity)) return true;
     if ((it & 255u) == 0) {
       if (abort && *abort) return false;
       if (globaltimer_ns() - t0 > kWaitLimitNs) return false;

@@ -212,6 +212,7 @@ __global__ void __launch_bounds__(C::kThreads, 1)
   if (CM > 1) cluster_sync_all();  // peers' barriers exist before any multicast lands
   else __syncthreads();
   tc_fence_after();
+  griddep_wait_and_release();
   const uint32_t tmem = *tmem_slot;
 
   auto fail = [&]() {
@@ -534,6 +535,7 @@ __global__ void __launch_bounds__(C::kThreads, 1)
   tc_fence_before();
   cluster_sync_all();
   tc_fence_after();
+  griddep_wait_and_release();
   const uint32_t tmem = *tmem_slot;
 
   auto fail = [&]() {
@@ -600,7 +602,8 @@ __global__ void __launch_bounds__(C::kThreads, 1)
     int local = 0;
     const uint32_t sA0 = smem_u32(sA), sB0 = smem_u32(sB);
     for (int u = pair_id; u < total_units && !abort_flag; u += n_pairs, ++local) {
-      if (!mbar_wait_bounded(tempty, (local & 1) ^ 1u, &abort_flag)) { fail(); break; }
+      // The peer's epilogue warps arrive on tempty with release at cluster scope.
+      if (!mbar_wait_bounded_cluster(tempty, (local & 1) ^ 1u, &abort_flag)) { fail(); break; }
       tc_fence_after();
       bool ok = true;
       for (int kb = 0; kb < kblocks; ++kb) {
@@ -837,7 +840,9 @@ nvfp4_status launch(const uint8_t* a_codes, const uint8_t* a_scales, const float
   args.status = status_word_dev();
   const int clusters = static_cast<int>(units < clusters_max ? units : clusters_max);
   cudaLaunchConfig_t cfg = {};
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = C::CM;
   attr[0].val.clusterDim.y = 1;
@@ -847,7 +852,7 @@ nvfp4_status launch(const uint8_t* a_codes, const uint8_t* a_scales, const float
   cfg.dynamicSmemBytes = C::kSmemBytes;
   cfg.stream = stream;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = 2;
   if (cudaLaunchKernelEx(&cfg, nvfp4_gemm_kernel<C>, ma, mb, mo, args) != cudaSuccess) return NVFP4_ERR_CUDA;
   count_launches(1);
   return launch_status();
@@ -866,7 +871,9 @@ int resident_pairs() {
                            static_cast<int>(C::kSmemBytes)) != cudaSuccess)
     return 0;
   cudaLaunchConfig_t cfg = {};
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = 2;
   attr[0].val.clusterDim.y = 1;
@@ -912,7 +919,9 @@ nvfp4_status launch_pair(const uint8_t* a_codes, const uint8_t* a_scales, const 
   args.status = status_word_dev();
   const int pairs = static_cast<int>(units < pairs_max ? units : pairs_max);
   cudaLaunchConfig_t cfg = {};
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = 2;
   attr[0].val.clusterDim.y = 1;
@@ -922,7 +931,7 @@ nvfp4_status launch_pair(const uint8_t* a_codes, const uint8_t* a_scales, const 
   cfg.dynamicSmemBytes = C::kSmemBytes;
   cfg.stream = stream;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = 2;
   if (cudaLaunchKernelEx(&cfg, nvfp4_gemm_pair_kernel<C>, ma, mb, msa, msb, mo, args) != cudaSuccess)
     return NVFP4_ERR_CUDA;
   count_launches(1);

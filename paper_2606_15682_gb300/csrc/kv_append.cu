@@ -85,11 +85,12 @@ NVFP4_API nvfp4_status kv_append_nvfp4(const nvfp4_kv_cache* cache, const void* 
   uint64_t grid = (items + kThreads - 1) / kThreads;
   const uint64_t cap = static_cast<uint64_t>(sm_count()) * 8;
   if (grid > cap) grid = cap;
-  kv_append_kernel<<<static_cast<int>(grid), kThreads, 0, static_cast<cudaStream_t>(stream)>>>(
-      static_cast<const uint16_t*>(k_bf16), static_cast<const uint16_t*>(v_bf16), seq_idx, pos, k_shift, n_rows,
-      FastDiv(static_cast<uint32_t>(cache->num_kv_heads)), static_cast<uint32_t>(cache->batch),
-      static_cast<uint32_t>(cache->capacity), cache->k_codes, cache->k_scales, cache->v_codes, cache->v_scales,
-      cache->k_gscale, cache->v_gscale, status_word_dev());
+  if (launch_pdl(kv_append_kernel, dim3(static_cast<int>(grid)), dim3(kThreads), 0, static_cast<cudaStream_t>(stream),
+                 static_cast<const uint16_t*>(k_bf16), static_cast<const uint16_t*>(v_bf16), seq_idx, pos, k_shift,
+                 n_rows, FastDiv(static_cast<uint32_t>(cache->num_kv_heads)), static_cast<uint32_t>(cache->batch),
+                 static_cast<uint32_t>(cache->capacity), cache->k_codes, cache->k_scales, cache->v_codes,
+                 cache->v_scales, cache->k_gscale, cache->v_gscale, status_word_dev()) != cudaSuccess)
+    return NVFP4_ERR_CUDA;
   count_launches(1);
   return launch_status();
 }

@@ -1,4 +1,5 @@
 // a1 tensor scale and a2 NVFP4 quantization (Appendix A format).
+// All kernels are launched with programmatic dependent launch.
 //
 // Both kernels stream bf16 with 128-bit loads.  The tensor-scale reduction
 // takes one 8-element chunk per lane per step; the quantizer one 16-element
@@ -31,6 +32,7 @@ struct ChunkMap {
 
 __global__ void __launch_bounds__(kThreads) amax_kernel(const uint16_t* __restrict__ x, ChunkMap map,
                                                         uint32_t* __restrict__ amax_bits) {
+  griddep_wait_and_release();
   const uint32_t stride = gridDim.x * blockDim.x;
   uint32_t m = 0;
   for (uint32_t c0 = blockIdx.x * blockDim.x; c0 < map.total; c0 += stride * kUnroll) {
@@ -55,8 +57,15 @@ __global__ void __launch_bounds__(kThreads) amax_kernel(const uint16_t* __restri
   }
 }
 
+// The amax accumulator (the bits of *g) starts at zero.
+__global__ void tensor_scale_init(float* g) {
+  griddep_wait_and_release();
+  *reinterpret_cast<uint32_t*>(g) = 0u;
+}
+
 // g = amax / (6 * 448) in fp32, or 1 for an all-zero tensor.
 __global__ void tensor_scale_finalize(float* g) {
+  griddep_wait_and_release();
   const uint32_t bits = *reinterpret_cast<uint32_t*>(g);
   const float amax = __uint_as_float(bits << 16);
   *g = amax > 0.0f ? __fdiv_rn(amax, 2688.0f) : 1.0f;
@@ -71,6 +80,7 @@ __global__ void __launch_bounds__(kThreads) quantize_kernel(const uint16_t* __re
                                                             uint32_t rows, const float* __restrict__ g_ptr,
                                                             uint2* __restrict__ codes, uint8_t* __restrict__ scales,
                                                             int* status) {
+  griddep_wait_and_release();
   const float g_in = *g_ptr;
   const bool g_ok = g_in > 0.0f && g_in <= FLT_MAX;
   if (!g_ok && blockIdx.x == 0 && threadIdx.x == 0) set_status(status, NVFP4_ERR_INVALID_ARG);
@@ -139,6 +149,7 @@ __global__ void __launch_bounds__(kThreads) quantize_kernel(const uint16_t* __re
 template <bool kToMMA>
 __global__ void relayout_kernel(const uint8_t* __restrict__ src, uint8_t* __restrict__ dst, uint32_t rows,
                                 uint32_t kblocks) {
+  griddep_wait_and_release();
   const uint32_t kgroups = kblocks >> 2;
   const uint32_t padded = (rows + 127u) & ~127u;
   const uint32_t n = padded * kblocks;
@@ -194,14 +205,16 @@ NVFP4_API nvfp4_status nvfp4_tensor_scale(const void* x_bf16, int64_t rows, int6
   if (st != NVFP4_OK) return st;
   if (!aligned(g_dev, 4)) return NVFP4_ERR_ALIGN;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  if (cudaMemsetAsync(g_dev, 0, sizeof(float), s) != cudaSuccess) return NVFP4_ERR_CUDA;
+  if (launch_pdl(tensor_scale_init, dim3(1), dim3(1), 0, s, g_dev) != cudaSuccess) return NVFP4_ERR_CUDA;
+  count_launches(1);
   const ChunkMap map = make_map(rows, cols, ld);
   if (map.total) {
-    amax_kernel<<<grid_for(map.total, kThreads * kUnroll), kThreads, 0, s>>>(
-        static_cast<const uint16_t*>(x_bf16), map, reinterpret_cast<uint32_t*>(g_dev));
+    if (launch_pdl(amax_kernel, dim3(grid_for(map.total, kThreads * kUnroll)), dim3(kThreads), 0, s,
+                   static_cast<const uint16_t*>(x_bf16), map, reinterpret_cast<uint32_t*>(g_dev)) != cudaSuccess)
+      return NVFP4_ERR_CUDA;
     count_launches(1);
   }
-  tensor_scale_finalize<<<1, 1, 0, s>>>(g_dev);
+  if (launch_pdl(tensor_scale_finalize, dim3(1), dim3(1), 0, s, g_dev) != cudaSuccess) return NVFP4_ERR_CUDA;
   count_launches(1);
   return launch_status();
 }
@@ -220,15 +233,11 @@ NVFP4_API nvfp4_status nvfp4_quantize(const void* x_bf16, int64_t rows, int64_t 
   const uint32_t total_blocks = static_cast<uint32_t>(rows * kblocks);
   const int grid = grid_for(total_blocks, kThreads * kUnroll);
   const bool dense = (ld == cols);
-  if (layout == NVFP4_SCALES_MMA) {
-    quantize_kernel<true><<<grid, kThreads, 0, s>>>(static_cast<const uint16_t*>(x_bf16), FastDiv(kblocks),
-                                                    total_blocks, ld, dense, static_cast<uint32_t>(rows), g_dev,
-                                                    reinterpret_cast<uint2*>(codes), scales, status_word_dev());
-  } else {
-    quantize_kernel<false><<<grid, kThreads, 0, s>>>(static_cast<const uint16_t*>(x_bf16), FastDiv(kblocks),
-                                                     total_blocks, ld, dense, static_cast<uint32_t>(rows), g_dev,
-                                                     reinterpret_cast<uint2*>(codes), scales, status_word_dev());
-  }
+  cudaError_t e = launch_pdl(layout == NVFP4_SCALES_MMA ? quantize_kernel<true> : quantize_kernel<false>, dim3(grid),
+                             dim3(kThreads), 0, s, static_cast<const uint16_t*>(x_bf16), FastDiv(kblocks),
+                             total_blocks, ld, dense, static_cast<uint32_t>(rows), g_dev,
+                             reinterpret_cast<uint2*>(codes), scales, status_word_dev());
+  if (e != cudaSuccess) return NVFP4_ERR_CUDA;
   count_launches(1);
   return launch_status();
 }
@@ -249,10 +258,9 @@ NVFP4_API nvfp4_status nvfp4_scales_relayout(const uint8_t* src, uint8_t* dst, i
   if (rows == 0 || cols == 0) return NVFP4_OK;
   const uint32_t kblocks = static_cast<uint32_t>(cols / 16);
   const uint64_t n = static_cast<uint64_t>((rows + 127) / 128 * 128) * kblocks;
-  if (to == NVFP4_SCALES_MMA)
-    relayout_kernel<true><<<grid_for(n, 256), 256, 0, s>>>(src, dst, static_cast<uint32_t>(rows), kblocks);
-  else
-    relayout_kernel<false><<<grid_for(n, 256), 256, 0, s>>>(src, dst, static_cast<uint32_t>(rows), kblocks);
+  if (launch_pdl(to == NVFP4_SCALES_MMA ? relayout_kernel<true> : relayout_kernel<false>, dim3(grid_for(n, 256)),
+                 dim3(256), 0, s, src, dst, static_cast<uint32_t>(rows), kblocks) != cudaSuccess)
+    return NVFP4_ERR_CUDA;
   count_launches(1);
   return launch_status();
 }
