@@ -103,6 +103,32 @@ nvfp4_status nvfp4_quantize(const void* x_bf16, int64_t rows, int64_t cols, int6
                             const float* g_dev, uint8_t* codes, uint8_t* scales,
                             nvfp4_scale_layout layout, void* stream);
 
+/* Bytes of caller-owned state used by nvfp4_quantize_dynamic. */
+#define NVFP4_DYNAMIC_STATE_BYTES 16
+
+/*
+ * a1 + a2 in one kernel launch: the tensor scale g of x (exactly as
+ * nvfp4_tensor_scale computes it) is stored in *g_dev and x is quantized
+ * with it (exactly as nvfp4_quantize does); codes, scales and g are
+ * bit-identical to the two calls in sequence.
+ *   state_dev : NVFP4_DYNAMIC_STATE_BYTES of device memory, 16-B aligned,
+ *               zero-filled once before its first use and left alone by the
+ *               caller afterwards.  Calls that may run concurrently (other
+ *               streams) need separate states; calls in one stream may share.
+ *   g_dev     : device float, written (never read first).
+ *   x, codes, scales, layout : as nvfp4_quantize.
+ * A cooperative launch: a grid-wide barrier separates the amax reduction
+ * from the quantization, and the second pass over x hits L2 when x fits in
+ * it.  A barrier that does not complete within 2 s sets NVFP4_ERR_TIMEOUT
+ * on the device and leaves the outputs unwritten; zero-fill the state again
+ * before reusing it.  rows*cols == 0 writes g = 1 and nothing else.
+ * Errors as nvfp4_quantize, plus: state_dev or g_dev NULL -> INVALID_ARG,
+ * state_dev not 16-B aligned -> ALIGN.
+ */
+nvfp4_status nvfp4_quantize_dynamic(const void* x_bf16, int64_t rows, int64_t cols, int64_t ld,
+                                    void* state_dev, float* g_dev, uint8_t* codes, uint8_t* scales,
+                                    nvfp4_scale_layout layout, void* stream);
+
 /*
  * Reorder block scales between the two storage orders (both directions).
  * src and dst must not overlap.  cols % 64 == 0.

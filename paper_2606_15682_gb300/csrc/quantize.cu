@@ -6,6 +6,8 @@
 // block per lane.  They are HBM-bound: the quantizer moves 2 B in and
 // 0.5625 B out per element.
 #include <cfloat>
+#include <map>
+#include <mutex>
 
 #include "common.cuh"
 #include "nvfp4_quant.cuh"
@@ -63,6 +65,12 @@ __global__ void tensor_scale_init(float* g) {
   *reinterpret_cast<uint32_t*>(g) = 0u;
 }
 
+// g of an empty tensor.
+__global__ void tensor_scale_finalize_empty(float* g) {
+  griddep_wait_and_release();
+  *g = 1.0f;
+}
+
 // g = amax / (6 * 448) in fp32, or 1 for an all-zero tensor.
 __global__ void tensor_scale_finalize(float* g) {
   griddep_wait_and_release();
@@ -75,16 +83,10 @@ __global__ void tensor_scale_finalize(float* g) {
 // half of the 32 bytes is in L1 after the first load of the warp), one scale
 // computation, one 64-bit code store.  A warp covers 32 consecutive blocks.
 template <bool kMMA>
-__global__ void __launch_bounds__(kThreads) quantize_kernel(const uint16_t* __restrict__ x, FastDiv kblocks_div,
-                                                            uint32_t total_blocks, int64_t ld, bool dense,
-                                                            uint32_t rows, const float* __restrict__ g_ptr,
-                                                            uint2* __restrict__ codes, uint8_t* __restrict__ scales,
-                                                            int* status) {
-  griddep_wait_and_release();
-  const float g_in = *g_ptr;
-  const bool g_ok = g_in > 0.0f && g_in <= FLT_MAX;
-  if (!g_ok && blockIdx.x == 0 && threadIdx.x == 0) set_status(status, NVFP4_ERR_INVALID_ARG);
-  const float g = g_ok ? g_in : 1.0f;
+__device__ __forceinline__ void quantize_blocks(const uint16_t* __restrict__ x, FastDiv kblocks_div,
+                                                uint32_t total_blocks, int64_t ld, bool dense, uint32_t rows,
+                                                float g, bool g_ok, uint2* __restrict__ codes,
+                                                uint8_t* __restrict__ scales) {
   const float six_g = __fmul_rn(6.0f, g);
   const uint32_t kblocks = kblocks_div.d;
   const uint32_t kgroups = kblocks >> 2;
@@ -144,6 +146,116 @@ __global__ void __launch_bounds__(kThreads) quantize_kernel(const uint16_t* __re
       scales[mma_scale_offset(r, k, kgroups)] = 0;
     }
   }
+}
+
+template <bool kMMA>
+__global__ void __launch_bounds__(kThreads) quantize_kernel(const uint16_t* __restrict__ x, FastDiv kblocks_div,
+                                                            uint32_t total_blocks, int64_t ld, bool dense,
+                                                            uint32_t rows, const float* __restrict__ g_ptr,
+                                                            uint2* __restrict__ codes, uint8_t* __restrict__ scales,
+                                                            int* status) {
+  griddep_wait_and_release();
+  const float g_in = *g_ptr;
+  const bool g_ok = g_in > 0.0f && g_in <= FLT_MAX;
+  if (!g_ok && blockIdx.x == 0 && threadIdx.x == 0) set_status(status, NVFP4_ERR_INVALID_ARG);
+  quantize_blocks<kMMA>(x, kblocks_div, total_blocks, ld, dense, rows, g_ok ? g_in : 1.0f, g_ok, codes, scales);
+}
+
+__device__ __forceinline__ unsigned long long ld_acquire_u64(const unsigned long long* p) {
+  unsigned long long v;
+  asm volatile("ld.acquire.gpu.global.u64 %0, [%1];" : "=l"(v) : "l"(p) : "memory");
+  return v;
+}
+
+// a1 + a2 in one cooperative launch.  Phase 1 reduces amax(|x|) over the
+// same 16-element blocks phase 2 quantizes; a grid-wide barrier separates
+// them.  Caller-owned state (two 64-bit words, zero before the first call):
+//   state[0] = (call epoch << 32) | blocks arrived in this epoch
+//   state[1] = (epoch << 32) | amax bits, combined with atomicMax
+// A newer epoch's tag dominates any older value, so nothing is cleared
+// between calls; the last block to arrive opens the next epoch.
+template <bool kMMA>
+__global__ void __launch_bounds__(kThreads) quantize_dynamic_kernel(
+    const uint16_t* __restrict__ x, FastDiv kblocks_div, uint32_t total_blocks, int64_t ld, bool dense, uint32_t rows,
+    unsigned long long* state, float* __restrict__ g_out, uint2* __restrict__ codes, uint8_t* __restrict__ scales,
+    int* status) {
+  griddep_wait_and_release();
+  const uint32_t kblocks = kblocks_div.d;
+  const uint32_t stride = gridDim.x * blockDim.x;
+  uint32_t m = 0;
+  for (uint32_t b0 = blockIdx.x * blockDim.x + threadIdx.x; b0 < total_blocks; b0 += stride * kUnroll) {
+    uint4 v[2 * kUnroll];
+#pragma unroll
+    for (int u = 0; u < kUnroll; ++u) {
+      const uint32_t b = b0 + u * stride;
+      const uint32_t row = kblocks_div.div(b), kb = b - row * kblocks;
+      const int64_t off = dense ? static_cast<int64_t>(b) * 16 : static_cast<int64_t>(row) * ld + kb * 16;
+      const uint4* src = reinterpret_cast<const uint4*>(x + off);
+      const bool live = b < total_blocks;
+      v[2 * u] = live ? __ldg(src) : make_uint4(0, 0, 0, 0);
+      v[2 * u + 1] = live ? __ldg(src + 1) : make_uint4(0, 0, 0, 0);
+    }
+#pragma unroll
+    for (int u = 0; u < 2 * kUnroll; ++u) m = max(m, amax_bits_bf16x8(v[u]));
+  }
+  m = __reduce_max_sync(0xffffffffu, m);
+  __shared__ uint32_t warp_max[kThreads / 32];
+  __shared__ uint32_t s_amax;
+  __shared__ int s_ok;
+  if ((threadIdx.x & 31) == 0) warp_max[threadIdx.x >> 5] = m;
+  __syncthreads();
+  if (threadIdx.x < 32) {
+    m = threadIdx.x < kThreads / 32 ? warp_max[threadIdx.x] : 0u;
+    m = __reduce_max_sync(0xffffffffu, m);
+    if (threadIdx.x == 0) {
+      const unsigned long long epoch = ld_acquire_u64(&state[0]) >> 32;
+      atomicMax(&state[1], (epoch << 32) | m);
+      __threadfence();
+      const unsigned long long old = atomicAdd(&state[0], 1ull);
+      int ok = (old >> 32) == epoch;
+      if (ok && static_cast<uint32_t>(old) == gridDim.x - 1) {
+        __threadfence();
+        atomicExch(&state[0], (epoch + 1) << 32);
+      } else if (ok) {
+        const uint64_t t0 = globaltimer_ns();
+        for (uint32_t it = 0; (ld_acquire_u64(&state[0]) >> 32) == epoch; ++it)
+          if ((it & 63u) == 63u && globaltimer_ns() - t0 > kWaitLimitNs) { ok = 0; break; }
+      }
+      const unsigned long long a = ld_acquire_u64(&state[1]);
+      if (ok && (a >> 32) != epoch) ok = 0;
+      if (!ok) set_status(status, NVFP4_ERR_TIMEOUT);
+      s_amax = static_cast<uint32_t>(a) & 0xFFFFu;
+      s_ok = ok;
+    }
+  }
+  __syncthreads();
+  if (!s_ok) return;
+  const float amax = __uint_as_float(s_amax << 16);
+  const float g = amax > 0.0f ? __fdiv_rn(amax, 2688.0f) : 1.0f;
+  if (blockIdx.x == 0 && threadIdx.x == 0) *g_out = g;
+  quantize_blocks<kMMA>(x, kblocks_div, total_blocks, ld, dense, rows, g, true, codes, scales);
+}
+
+// Blocks of quantize_dynamic_kernel that fit on the device at once (a
+// cooperative launch must not exceed it).
+template <bool kMMA>
+int dynamic_capacity() {
+  static std::mutex mu;
+  static std::map<int, int> cache;
+  int d = 0;
+  if (cudaGetDevice(&d) != cudaSuccess) return 0;
+  std::lock_guard<std::mutex> lock(mu);
+  auto it = cache.find(d);
+  if (it != cache.end()) return it->second;
+  int per_sm = 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, quantize_dynamic_kernel<kMMA>, kThreads, 0) !=
+          cudaSuccess ||
+      per_sm <= 0) {
+    cudaGetLastError();
+    return 0;
+  }
+  cache[d] = per_sm * sm_count();
+  return cache[d];
 }
 
 template <bool kToMMA>
@@ -237,6 +349,53 @@ NVFP4_API nvfp4_status nvfp4_quantize(const void* x_bf16, int64_t rows, int64_t 
                              dim3(kThreads), 0, s, static_cast<const uint16_t*>(x_bf16), FastDiv(kblocks),
                              total_blocks, ld, dense, static_cast<uint32_t>(rows), g_dev,
                              reinterpret_cast<uint2*>(codes), scales, status_word_dev());
+  if (e != cudaSuccess) return NVFP4_ERR_CUDA;
+  count_launches(1);
+  return launch_status();
+}
+
+NVFP4_API nvfp4_status nvfp4_quantize_dynamic(const void* x_bf16, int64_t rows, int64_t cols, int64_t ld,
+                                              void* state_dev, float* g_dev, uint8_t* codes, uint8_t* scales,
+                                              nvfp4_scale_layout layout, void* stream) {
+  if (layout != NVFP4_SCALES_ROWMAJOR && layout != NVFP4_SCALES_MMA) return NVFP4_ERR_INVALID_ARG;
+  nvfp4_status st = check_bf16_matrix(x_bf16, rows, cols, ld, layout == NVFP4_SCALES_MMA ? 64 : 16);
+  if (st != NVFP4_OK) return st;
+  if (!state_dev || !g_dev) return NVFP4_ERR_INVALID_ARG;
+  if (!aligned(state_dev, 16) || !aligned(g_dev, 4)) return NVFP4_ERR_ALIGN;
+  if (rows == 0 || cols == 0) {
+    // Nothing to quantize; the tensor scale of an empty tensor is 1.
+    if (launch_pdl(tensor_scale_finalize_empty, dim3(1), dim3(1), 0, static_cast<cudaStream_t>(stream), g_dev) !=
+        cudaSuccess)
+      return NVFP4_ERR_CUDA;
+    count_launches(1);
+    return launch_status();
+  }
+  if (!codes || !scales) return NVFP4_ERR_INVALID_ARG;
+  if (!aligned(codes, 8)) return NVFP4_ERR_ALIGN;
+  const bool mma = layout == NVFP4_SCALES_MMA;
+  const int cap = mma ? dynamic_capacity<true>() : dynamic_capacity<false>();
+  if (cap <= 0) return NVFP4_ERR_CUDA;
+  const uint32_t kblocks = static_cast<uint32_t>(cols / 16);
+  const uint32_t total_blocks = static_cast<uint32_t>(rows * kblocks);
+  int grid = grid_for(total_blocks, kThreads * kUnroll);
+  if (grid > cap) grid = cap;
+  // Cooperative: every block is resident at once, so the grid barrier can
+  // complete.  (Without programmatic serialization: measured no faster.)
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeCooperative;
+  attr[0].val.cooperative = 1;
+  cfg.gridDim = dim3(grid);
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = 0;
+  cfg.stream = static_cast<cudaStream_t>(stream);
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  const cudaError_t e =
+      cudaLaunchKernelEx(&cfg, mma ? quantize_dynamic_kernel<true> : quantize_dynamic_kernel<false>,
+                         static_cast<const uint16_t*>(x_bf16), FastDiv(kblocks), total_blocks, ld, ld == cols,
+                         static_cast<uint32_t>(rows), static_cast<unsigned long long*>(state_dev), g_dev,
+                         reinterpret_cast<uint2*>(codes), scales, status_word_dev());
   if (e != cudaSuccess) return NVFP4_ERR_CUDA;
   count_launches(1);
   return launch_status();

@@ -51,6 +51,7 @@ def _sig(name, args, res=ctypes.c_int):
 
 _tensor_scale = _sig("nvfp4_tensor_scale", [_p, _i64, _i64, _i64, _p, _p])
 _quantize = _sig("nvfp4_quantize", [_p, _i64, _i64, _i64, _p, _p, _p, ctypes.c_int, _p])
+_quantize_dynamic = _sig("nvfp4_quantize_dynamic", [_p, _i64, _i64, _i64, _p, _p, _p, _p, ctypes.c_int, _p])
 _relayout = _sig("nvfp4_scales_relayout", [_p, _p, _i64, _i64, ctypes.c_int, ctypes.c_int, _p])
 _linear = _sig("nvfp4_linear", [_p, _p, _p, _p, _p, _p, _i64, _i64, _i64, _p, _i64, _p])
 _kv_append = _sig("kv_append_nvfp4", [ctypes.POINTER(KVCacheStruct), _p, _p, _p, _p, _i64, _p, _p])
@@ -107,6 +108,16 @@ def nvfp4_tensor_scale(x, g, stream=None):
 
 def nvfp4_quantize(x, g, codes, scales, layout=SCALES_MMA, stream=None):
     _check("nvfp4_quantize", _quantize(*_mat(x), _ptr(g), _ptr(codes), _ptr(scales), layout, _stream(stream)))
+
+
+DYNAMIC_STATE_BYTES = 16
+
+
+def nvfp4_quantize_dynamic(x, state, g, codes, scales, layout=SCALES_MMA, stream=None):
+    """Tensor scale + quantization in one launch; `state` is a zero-filled
+    device buffer of DYNAMIC_STATE_BYTES bytes owned by the caller."""
+    _check("nvfp4_quantize_dynamic",
+           _quantize_dynamic(*_mat(x), _ptr(state), _ptr(g), _ptr(codes), _ptr(scales), layout, _stream(stream)))
 
 
 def nvfp4_scales_relayout(src, dst, rows, cols, from_layout, to_layout, stream=None):
@@ -181,7 +192,7 @@ class KVCache:
                              self.head_dim, self.capacity, self.k_gscale, self.v_gscale)
 
 
-EXPORTED = ["nvfp4_scales_bytes", "nvfp4_tensor_scale", "nvfp4_quantize", "nvfp4_scales_relayout", "nvfp4_linear",
+EXPORTED = ["nvfp4_scales_bytes", "nvfp4_tensor_scale", "nvfp4_quantize", "nvfp4_quantize_dynamic", "nvfp4_scales_relayout", "nvfp4_linear",
             "kv_append_nvfp4", "decode_attention_nvfp4_workspace_size", "decode_attention_nvfp4",
             "decode_attention_nvfp4_static_scratch",
             "nvfp4_get_device_status", "nvfp4_status_string", "nvfp4_launch_count"]

@@ -53,6 +53,13 @@ def test_argument_validation_before_launch():
     assert L.nvfp4_linear(odd, p, p, p, p, p, 128, 128, 256, p, 128, s) == 3
     assert L.nvfp4_quantize(odd, 4, 64, 64, p, p, p, 1, s) == 3
     assert L.nvfp4_quantize(p, 4, 64, 68, p, p, p, 1, s) == 3            # ld % 8
+    st = ctypes.c_void_p(0x20000)
+    assert L.nvfp4_quantize_dynamic(p, 4, 64, 64, None, p, p, p, 1, s) == 1   # no state
+    assert L.nvfp4_quantize_dynamic(p, 4, 64, 64, st, None, p, p, 1, s) == 1  # no g
+    assert L.nvfp4_quantize_dynamic(p, 4, 64, 64, odd, p, p, p, 1, s) == 3    # state not 16-B aligned
+    assert L.nvfp4_quantize_dynamic(p, 4, 32, 32, st, p, p, p, 1, s) == 2     # MMA layout needs cols % 64
+    assert L.nvfp4_quantize_dynamic(p, 4, 64, 64, st, p, p, p, 9, s) == 1     # bad layout enum
+    assert L.nvfp4_quantize_dynamic(p, 4, 64, 64, st, p, None, p, 1, s) == 1  # no codes
 
 
 def test_kv_and_attention_validation():

@@ -174,3 +174,86 @@ def test_workload_tensors_bit_exact(N, workload):
                 N.nvfp4_tensor_scale(t, g)
                 assert np.float32(g.item()) == g_ref
             check_quantize(N, t.cpu() if rows is None else t, g_np=g_ref, layout=1, rows_sample=rows)
+
+
+# ------------------------------------------------ one-launch a1 + a2 ---
+
+def dynamic(N, x, state, layout=1):
+    rows, cols = x.shape
+    g = torch.full((1,), float("nan"), dtype=torch.float32, device="cuda")
+    codes = torch.empty(rows, cols // 2, dtype=torch.uint8, device="cuda")
+    scales = torch.full((N.nvfp4_scales_bytes(rows, cols, layout),), 0xEE, dtype=torch.uint8, device="cuda")
+    N.nvfp4_quantize_dynamic(x, state, g, codes, scales, layout)
+    return codes, scales, g
+
+
+def test_dynamic_matches_oracle_and_two_call_path(N):
+    """Different shapes (so different grid sizes) and both layouts on one state:
+    each call starts a new epoch of the state without clearing it."""
+    state = torch.zeros(N.DYNAMIC_STATE_BYTES, dtype=torch.uint8, device="cuda")
+    gen = torch.Generator().manual_seed(77)
+    for i, (rows, cols, ld, layout) in enumerate([(130, 192, 192, 1), (3, 64, 64, 0), (2048, 1536, 1536, 1),
+                                                  (257, 512, 520, 0), (1, 64, 64, 1), (700, 8960, 8960, 1)]):
+        base = torch.randn(rows, ld, generator=gen)
+        mag = torch.exp2(torch.randint(-20, 8, (rows, (ld + 15) // 16), generator=gen).float())
+        x = (base * mag.repeat_interleave(16, dim=1)[:, :ld]).to(torch.bfloat16)
+        xv = x.cuda()[:, :cols] if ld != cols else x.cuda()
+        codes, scales, g = dynamic(N, xv, state, layout)
+        g2 = torch.empty(1, dtype=torch.float32, device="cuda")
+        N.nvfp4_tensor_scale(xv, g2)
+        c2, s2 = gpu_quantize(N, xv, g2, layout)
+        torch.cuda.synchronize()
+        assert N.nvfp4_get_device_status() == 0
+        gref = O.tensor_scale(f32(x[:, :cols]))
+        assert np.float32(g.item()) == gref == np.float32(g2.item()), f"call {i}"
+        assert torch.equal(codes, c2) and torch.equal(scales, s2), f"call {i}: differs from the two-call path"
+        sel = np.arange(rows) if rows <= 300 else np.r_[0:64, rows - 64:rows]
+        rc, rs = O.quantize(f32(x[:, :cols][torch.as_tensor(sel)]), gref)
+        assert np.array_equal(u8(codes)[sel], rc), f"call {i}"
+        gs = u8(scales).reshape(rows, cols // 16) if layout == 0 else O.scales_from_mma(u8(scales), rows, cols)
+        assert np.array_equal(gs[sel], rs), f"call {i}"
+    # Ten calls in a row (ten epochs), the last one checked.
+    x = torch.randn(512, 1024, generator=gen).to(torch.bfloat16).cuda()
+    for _ in range(10):
+        codes, scales, g = dynamic(N, x, state)
+    torch.cuda.synchronize()
+    assert N.nvfp4_get_device_status() == 0
+    assert np.float32(g.item()) == O.tensor_scale(f32(x))
+
+
+def test_dynamic_all_zero_and_empty(N):
+    state = torch.zeros(N.DYNAMIC_STATE_BYTES, dtype=torch.uint8, device="cuda")
+    codes, scales, g = dynamic(N, torch.zeros(5, 64, dtype=torch.bfloat16, device="cuda"), state)
+    assert g.item() == 1.0 and not u8(codes).any() and not u8(scales).any()
+    # An empty tensor: g = 1, the state is untouched, and the next call still works.
+    e = torch.zeros(0, 64, dtype=torch.bfloat16, device="cuda")
+    g = torch.full((1,), 3.0, device="cuda")
+    N.nvfp4_quantize_dynamic(e, state, g, None, None, 1)
+    assert g.item() == 1.0
+    x = torch.randn(64, 128, device="cuda").to(torch.bfloat16)
+    codes, scales, g = dynamic(N, x, state)
+    torch.cuda.synchronize()
+    assert N.nvfp4_get_device_status() == 0
+    assert np.float32(g.item()) == O.tensor_scale(f32(x))
+
+
+@pytest.mark.parametrize("workload", WL)
+def test_dynamic_workload_activations(N, workload):
+    """Every activation of every workload at full size, as the bench step quantizes it."""
+    state = torch.zeros(N.DYNAMIC_STATE_BYTES, dtype=torch.uint8, device="cuda")
+    for name in synth.WORKLOADS[workload]["linears"]:
+        a, _ = synth.linear_inputs(workload, name, device="cuda")
+        codes, scales, g = dynamic(N, a, state)
+        g2 = torch.empty(1, dtype=torch.float32, device="cuda")
+        N.nvfp4_tensor_scale(a, g2)
+        c2, s2 = gpu_quantize(N, a, g2, 1)
+        torch.cuda.synchronize()
+        assert N.nvfp4_get_device_status() == 0
+        assert g.item() == g2.item() and np.float32(g.item()) == O.tensor_scale(f32(a))
+        assert torch.equal(codes, c2) and torch.equal(scales, s2), name
+        M = a.shape[0]
+        rows = np.unique(np.r_[0:min(32, M), max(M - 32, 0):M])
+        assert rows.min() >= 0 and rows.max() < M  # checked on the host before indexing on the device
+        rc, rs = O.quantize(f32(a[torch.as_tensor(rows, device="cuda")]), np.float32(g.item()))
+        assert np.array_equal(u8(codes)[rows], rc)
+        assert np.array_equal(O.scales_from_mma(u8(scales), a.shape[0], a.shape[1])[rows], rs)
