@@ -446,11 +446,16 @@ __device__ __forceinline__ void tma_load_2d_to_leader(void* smem_dst, const void
       "l"(reinterpret_cast<uint64_t>(tmap)), "r"(remote), "r"(x), "r"(y)
       : "memory");
 }
-// Arrive on the barrier at this shared-memory offset in CTA `rank` of the cluster.
-__device__ __forceinline__ void mbar_arrive_cluster(uint64_t* bar, uint32_t rank) {
+// Arrive on the barrier at this shared-memory offset in CTA `rank` of the
+// cluster, without release semantics.  Used only to hand the accumulator back:
+// the arriving warp's TMEM loads have completed (tcgen05.wait::ld) and are
+// ordered before the arrive by tcgen05.fence::before_thread_sync; no memory
+// written by this thread is read by the waiter.  (A release.cluster arrive
+// costs about a microsecond here, which stalled the MMAs at every tile.)
+__device__ __forceinline__ void mbar_arrive_cluster_relaxed(uint64_t* bar, uint32_t rank) {
   uint32_t remote;
   asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(smem_u32(bar)), "r"(rank));
-  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(remote) : "memory");
+  asm volatile("mbarrier.arrive.relaxed.cluster.shared::cluster.b64 _, [%0];" ::"r"(remote) : "memory");
 }
 
 template <int STAGES_>
@@ -602,8 +607,7 @@ __global__ void __launch_bounds__(C::kThreads, 1)
     int local = 0;
     const uint32_t sA0 = smem_u32(sA), sB0 = smem_u32(sB);
     for (int u = pair_id; u < total_units && !abort_flag; u += n_pairs, ++local) {
-      // The peer's epilogue warps arrive on tempty with release at cluster scope.
-      if (!mbar_wait_bounded_cluster(tempty, (local & 1) ^ 1u, &abort_flag)) { fail(); break; }
+      if (!mbar_wait_bounded(tempty, (local & 1) ^ 1u, &abort_flag)) { fail(); break; }
       tc_fence_after();
       bool ok = true;
       for (int kb = 0; kb < kblocks; ++kb) {
@@ -685,7 +689,7 @@ __global__ void __launch_bounds__(C::kThreads, 1)
       tmem_ld_wait();
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive_cluster(tempty, 0);
+      if (lane == 0) mbar_arrive_cluster_relaxed(tempty, 0);
 #pragma unroll
       for (int h = 0; h < 2; ++h) {
         if (lane == 0) bulk_wait_read_all();
