@@ -21,6 +21,7 @@ the CPU oracle instead, on a bounded sample of the same workload.
 from __future__ import annotations
 
 import argparse
+import hashlib
 import json
 import math
 import os
@@ -37,6 +38,27 @@ GEMM_WL = "qwen1.5b_prefill_linears_m2048"
 ATTN_WL = "qwen14b_decode_attention_b64_t16384"
 METRIC = "NVFP4 GEMM TFLOP/s & FP4-KV decode-attn HBM GB/s vs GB300 roofline"
 FP4_OVER_BF16 = 13.5 / 2.25  # nominal dense FP4 / BF16 tensor ratio of GB300
+CSRC = os.path.join(ROOT, "paper_2606_15682_gb300", "csrc")
+# DRAM bytes per launch (dram__bytes_read.sum + dram__bytes_write.sum) from one ncu capture of the
+# same kernel and shape (commands in profiles/).  Each entry holds only while the kernel sources
+# hash to the value they had at capture time; otherwise the line reports traffic = null.
+NCU_TRAFFIC = {
+    "gemm": {"bytes": 17295104 + 13306112, "sources": ("gemm.cu", "common.cuh"), "sha": "38a7b79963e14a5d",
+             "shape": (2048, 17920, 1536),
+             "profile": "profiles/gemm_qwen1.5b_prefill_gate_up_m2048_n17920_k1536.md"},
+    "attention": {"bytes": 1208748032 + 22318336, "sources": ("attention.cu", "common.cuh"),
+                  "sha": "bf910bb38594e7c5", "shape": (64, 16384),
+                  "profile": "profiles/attention_qwen14b_decode_b64_t16384.md (attn_partial_kernel)"},
+}
+
+
+def ncu_traffic(kind, shape):
+    e = NCU_TRAFFIC[kind]
+    h = hashlib.sha256()
+    for f in e["sources"]:
+        with open(os.path.join(CSRC, f), "rb") as fh:
+            h.update(fh.read())
+    return e["bytes"] if h.hexdigest()[:16] == e["sha"] and tuple(shape) == e["shape"] else None
 
 
 def load_peaks():
@@ -311,8 +333,8 @@ def run_ours(args, rank, world):
     else:
         roof = {"bound": "hbm", "achieved": d_bytes / d_s / 1e9, "peak": peaks["hbm_gbs"], "unit": "GB/s"}
     roof["frac"] = roof["achieved"] / roof["peak"]
-    roof["traffic"] = None
-    roof["kernel"] = f"nvfp4_gemm_kernel ({dom['name']}: {M}x{dom['N']}x{dom['K']})"
+    roof["traffic"] = ncu_traffic("gemm", (M, dom["N"], dom["K"]))
+    roof["kernel"] = f"nvfp4_gemm_pair_kernel ({dom['name']}: {M}x{dom['N']}x{dom['K']})"
     roof["peak_src"] = (f"{peaks['src']}: bf16 {peaks['bf16_tflops']} TFLOP/s x {FP4_OVER_BF16:g} nominal FP4/BF16"
                         if roof["bound"] == "tensor" else f"{peaks['src']} HBM copy")
     roof["also"] = {"tflops": d_flops / d_s / 1e12, "tflops_frac_of_fp4_peak": d_flops / d_s / 1e12 / fp4_peak,
@@ -349,7 +371,7 @@ def run_ours(args, rank, world):
             "step": "append 1 token/sequence (kv_append_nvfp4) + decode_attention_nvfp4",
             "algorithmic_bytes": attn_bytes,
             "roofline": {"bound": "hbm", "achieved": attn_gbs, "peak": peaks["hbm_gbs"], "unit": "GB/s",
-                         "frac": attn_gbs / peaks["hbm_gbs"], "traffic": None,
+                         "frac": attn_gbs / peaks["hbm_gbs"], "traffic": ncu_traffic("attention", (Bq, T)),
                          "kernel": "attn_partial_kernel + attn_combine_kernel (one decode_attention_nvfp4 call)"},
             "gpu_launches": attn_launches * args.steps,
         },

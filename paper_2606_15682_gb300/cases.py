@@ -2,6 +2,7 @@
 
     python -m paper_2606_15682_gb300.cases gemm --workload qwen1.5b_prefill_linears_m2048 --linear gate_up
     python -m paper_2606_15682_gb300.cases quantize --workload qwen1.5b_prefill_linears_m2048 --linear down
+    python -m paper_2606_15682_gb300.cases quantize_dynamic --workload qwen32b_prefill_linears_m8192 --linear down
     python -m paper_2606_15682_gb300.cases attention --batch 64 --context 16384
 
 Inputs are seeded synthetic tensors (paper_2606_15682_gb300.synth); for the
@@ -46,7 +47,7 @@ def _time(fn, iters):
 
 def main():
     ap = argparse.ArgumentParser()
-    ap.add_argument("kernel", choices=["gemm", "quantize", "tensor_scale", "attention"])
+    ap.add_argument("kernel", choices=["gemm", "quantize", "quantize_dynamic", "tensor_scale", "attention"])
     ap.add_argument("--workload", default="qwen1.5b_prefill_linears_m2048")
     ap.add_argument("--linear", default="gate_up")
     ap.add_argument("--batch", type=int, default=64)
@@ -55,7 +56,7 @@ def main():
     a = ap.parse_args()
     dev = torch.device("cuda", 0)
     torch.cuda.set_device(dev)
-    if a.kernel in ("gemm", "quantize", "tensor_scale"):
+    if a.kernel in ("gemm", "quantize", "quantize_dynamic", "tensor_scale"):
         x, W = synth.linear_inputs(a.workload, a.linear, device=dev)
         M, K = x.shape
         Nn = W.shape[0]
@@ -75,6 +76,10 @@ def main():
             if a.kernel == "quantize":
                 ms = _time(lambda: N.nvfp4_quantize(x, g, c, s, N.SCALES_MMA), a.iters)
                 byt = M * K * (2 + 0.5 + 1 / 16)
+            elif a.kernel == "quantize_dynamic":
+                st = torch.zeros(N.DYNAMIC_STATE_BYTES, dtype=torch.uint8, device=dev)
+                ms = _time(lambda: N.nvfp4_quantize_dynamic(x, st, g, c, s, N.SCALES_MMA), a.iters)
+                byt = M * K * (2 + 2 + 0.5 + 1 / 16)  # x read twice (amax pass, quantize pass)
             else:
                 ms = _time(lambda: N.nvfp4_tensor_scale(x, g), a.iters)
                 byt = M * K * 2
