@@ -82,70 +82,105 @@ __global__ void tensor_scale_finalize(float* g) {
 // One thread quantizes one 16-element block: two 128-bit loads (the second
 // half of the 32 bytes is in L1 after the first load of the warp), one scale
 // computation, one 64-bit code store.  A warp covers 32 consecutive blocks.
+// Where one pass of the quantizer reads: the thread's kUnroll 16-element
+// blocks of the iteration that starts at the warp-uniform block index bidx0
+// (block bidx0 + u * stride + lane).
+struct BlockSlots {
+  uint4 v0[kUnroll], v1[kUnroll];
+  uint32_t row[kUnroll], kb[kUnroll];
+};
+
+__device__ __forceinline__ void load_blocks(const uint16_t* __restrict__ x, FastDiv kblocks_div, uint32_t total_blocks,
+                                            int64_t ld, bool dense, uint32_t bidx0, uint32_t stride, uint32_t lane,
+                                            BlockSlots& sl) {
+  const uint32_t kblocks = kblocks_div.d;
+#pragma unroll
+  for (int u = 0; u < kUnroll; ++u) {
+    const uint32_t b = bidx0 + u * stride + lane;
+    sl.row[u] = kblocks_div.div(b);
+    sl.kb[u] = b - sl.row[u] * kblocks;
+    const int64_t off = dense ? static_cast<int64_t>(b) * 16 : static_cast<int64_t>(sl.row[u]) * ld + sl.kb[u] * 16;
+    const uint4* src = reinterpret_cast<const uint4*>(x + off);
+    const bool live = b < total_blocks;
+    sl.v0[u] = live ? __ldg(src) : make_uint4(0, 0, 0, 0);
+    sl.v1[u] = live ? __ldg(src + 1) : make_uint4(0, 0, 0, 0);
+  }
+}
+
+__device__ __forceinline__ uint32_t amax_bits_of(const BlockSlots& sl) {
+  uint32_t m = 0;
+#pragma unroll
+  for (int u = 0; u < kUnroll; ++u) m = max(m, max(amax_bits_bf16x8(sl.v0[u]), amax_bits_bf16x8(sl.v1[u])));
+  return m;
+}
+
+// Quantize the loaded blocks with tensor scale g.  Every lane of the warp
+// takes part (the MMA-layout scale gather shuffles across lanes).
+template <bool kMMA>
+__device__ __forceinline__ void quantize_loaded(const BlockSlots& sl, uint32_t total_blocks, uint32_t kblocks,
+                                                uint32_t bidx0, uint32_t stride, uint32_t lane, float g, float six_g,
+                                                bool g_ok, uint2* __restrict__ codes, uint8_t* __restrict__ scales) {
+  const uint32_t kgroups = kblocks >> 2;
+#pragma unroll
+  for (int u = 0; u < kUnroll; ++u) {
+    const uint32_t b = bidx0 + u * stride + lane;
+    const bool live = b < total_blocks;
+    float xf[16];
+    unpack_bf16x8(sl.v0[u], xf);
+    unpack_bf16x8(sl.v1[u], xf + 8);
+    const float amax = __uint_as_float(max(amax_bits_bf16x8(sl.v0[u]), amax_bits_bf16x8(sl.v1[u])) << 16);
+    const BlockScale bs = block_scale(amax, g, six_g);
+    float q[16];
+#pragma unroll
+    for (int i = 0; i < 16; ++i) q[i] = __fmul_rn(xf[i], bs.mult);
+    uint2 packed = make_uint2(e2m1x8(q), e2m1x8(q + 8));
+    uint32_t sc = bs.code;
+    if (!g_ok) { packed = make_uint2(0, 0); sc = 0; }
+    if (live) codes[b] = packed;
+    if (kMMA) {
+      // Lanes 4j..4j+3 hold the four k-blocks of one MMA scale group (kblocks % 4 == 0,
+      // so a group never straddles rows): assemble them into one 32-bit store.
+      uint32_t w = sc << (8 * (lane & 3));
+      w |= __shfl_xor_sync(0xffffffffu, w, 1);
+      w |= __shfl_xor_sync(0xffffffffu, w, 2);
+      if (live && (lane & 3) == 0)
+        *reinterpret_cast<uint32_t*>(scales + mma_scale_offset(sl.row[u], sl.kb[u], kgroups)) = w;
+    } else if (live) {
+      scales[static_cast<uint64_t>(sl.row[u]) * kblocks + sl.kb[u]] = static_cast<uint8_t>(sc);
+    }
+  }
+}
+
+// Zero the MMA-layout scales of the padding rows up to the next multiple of 128.
+__device__ __forceinline__ void zero_scale_padding(uint32_t rows, uint32_t kblocks, uint8_t* __restrict__ scales) {
+  const uint32_t kgroups = kblocks >> 2;
+  const uint32_t padded = (rows + 127u) & ~127u;
+  const uint32_t pad = (padded - rows) * kblocks;
+  for (uint32_t i = blockIdx.x * blockDim.x + threadIdx.x; i < pad; i += gridDim.x * blockDim.x) {
+    const uint32_t r = rows + i / kblocks, k = i % kblocks;
+    scales[mma_scale_offset(r, k, kgroups)] = 0;
+  }
+}
+
+// One thread quantizes one 16-element block per slot: two 128-bit loads (the
+// second half of the 32 bytes is in L1 after the first load of the warp), one
+// scale computation, one 64-bit code store.  A warp covers 32 consecutive
+// blocks per slot.
 template <bool kMMA>
 __device__ __forceinline__ void quantize_blocks(const uint16_t* __restrict__ x, FastDiv kblocks_div,
                                                 uint32_t total_blocks, int64_t ld, bool dense, uint32_t rows,
                                                 float g, bool g_ok, uint2* __restrict__ codes,
                                                 uint8_t* __restrict__ scales) {
   const float six_g = __fmul_rn(6.0f, g);
-  const uint32_t kblocks = kblocks_div.d;
-  const uint32_t kgroups = kblocks >> 2;
   const uint32_t lane = threadIdx.x & 31;
   const uint32_t stride = gridDim.x * blockDim.x;
-
   // bidx0 is warp-uniform so every lane takes part in the scale gather.
   for (uint32_t bidx0 = blockIdx.x * blockDim.x + (threadIdx.x & ~31u); bidx0 < total_blocks; bidx0 += stride * kUnroll) {
-    uint4 v0[kUnroll], v1[kUnroll];
-    uint32_t row[kUnroll], kb[kUnroll];
-#pragma unroll
-    for (int u = 0; u < kUnroll; ++u) {
-      const uint32_t b = bidx0 + u * stride + lane;
-      row[u] = kblocks_div.div(b);
-      kb[u] = b - row[u] * kblocks;
-      const int64_t off = dense ? static_cast<int64_t>(b) * 16 : static_cast<int64_t>(row[u]) * ld + kb[u] * 16;
-      const uint4* src = reinterpret_cast<const uint4*>(x + off);
-      const bool live = b < total_blocks;
-      v0[u] = live ? __ldg(src) : make_uint4(0, 0, 0, 0);
-      v1[u] = live ? __ldg(src + 1) : make_uint4(0, 0, 0, 0);
-    }
-#pragma unroll
-    for (int u = 0; u < kUnroll; ++u) {
-      const uint32_t b = bidx0 + u * stride + lane;
-      const bool live = b < total_blocks;
-      float xf[16];
-      unpack_bf16x8(v0[u], xf);
-      unpack_bf16x8(v1[u], xf + 8);
-      const float amax = __uint_as_float(max(amax_bits_bf16x8(v0[u]), amax_bits_bf16x8(v1[u])) << 16);
-      const BlockScale bs = block_scale(amax, g, six_g);
-      float q[16];
-#pragma unroll
-      for (int i = 0; i < 16; ++i) q[i] = __fmul_rn(xf[i], bs.mult);
-      uint2 packed = make_uint2(e2m1x8(q), e2m1x8(q + 8));
-      uint32_t sc = bs.code;
-      if (!g_ok) { packed = make_uint2(0, 0); sc = 0; }
-      if (live) codes[b] = packed;
-      if (kMMA) {
-        // Lanes 4j..4j+3 hold the four k-blocks of one MMA scale group (kblocks % 4 == 0,
-        // so a group never straddles rows): assemble them into one 32-bit store.
-        uint32_t w = sc << (8 * (lane & 3));
-        w |= __shfl_xor_sync(0xffffffffu, w, 1);
-        w |= __shfl_xor_sync(0xffffffffu, w, 2);
-        if (live && (lane & 3) == 0)
-          *reinterpret_cast<uint32_t*>(scales + mma_scale_offset(row[u], kb[u], kgroups)) = w;
-      } else if (live) {
-        scales[static_cast<uint64_t>(row[u]) * kblocks + kb[u]] = static_cast<uint8_t>(sc);
-      }
-    }
+    BlockSlots sl;
+    load_blocks(x, kblocks_div, total_blocks, ld, dense, bidx0, stride, lane, sl);
+    quantize_loaded<kMMA>(sl, total_blocks, kblocks_div.d, bidx0, stride, lane, g, six_g, g_ok, codes, scales);
   }
-  if (kMMA) {
-    // Zero the scales of the padding rows up to the next multiple of 128.
-    const uint32_t padded = (rows + 127u) & ~127u;
-    const uint32_t pad = (padded - rows) * kblocks;
-    for (uint32_t i = blockIdx.x * blockDim.x + threadIdx.x; i < pad; i += stride) {
-      const uint32_t r = rows + i / kblocks, k = i % kblocks;
-      scales[mma_scale_offset(r, k, kgroups)] = 0;
-    }
-  }
+  if (kMMA) zero_scale_padding(rows, kblocks_div.d, scales);
 }
 
 template <bool kMMA>
@@ -180,23 +215,23 @@ __global__ void __launch_bounds__(kThreads) quantize_dynamic_kernel(
     unsigned long long* state, float* __restrict__ g_out, uint2* __restrict__ codes, uint8_t* __restrict__ scales,
     int* status) {
   griddep_wait_and_release();
-  const uint32_t kblocks = kblocks_div.d;
+  const uint32_t lane = threadIdx.x & 31;
   const uint32_t stride = gridDim.x * blockDim.x;
+  // Resident: one pass covers the tensor, so the loaded blocks stay in
+  // registers across the barrier and x is read once.
+  const bool resident = total_blocks <= stride * kUnroll;
+  const uint32_t bidx_first = blockIdx.x * blockDim.x + (threadIdx.x & ~31u);
+  BlockSlots sl;
   uint32_t m = 0;
-  for (uint32_t b0 = blockIdx.x * blockDim.x + threadIdx.x; b0 < total_blocks; b0 += stride * kUnroll) {
-    uint4 v[2 * kUnroll];
-#pragma unroll
-    for (int u = 0; u < kUnroll; ++u) {
-      const uint32_t b = b0 + u * stride;
-      const uint32_t row = kblocks_div.div(b), kb = b - row * kblocks;
-      const int64_t off = dense ? static_cast<int64_t>(b) * 16 : static_cast<int64_t>(row) * ld + kb * 16;
-      const uint4* src = reinterpret_cast<const uint4*>(x + off);
-      const bool live = b < total_blocks;
-      v[2 * u] = live ? __ldg(src) : make_uint4(0, 0, 0, 0);
-      v[2 * u + 1] = live ? __ldg(src + 1) : make_uint4(0, 0, 0, 0);
+  if (resident) {
+    load_blocks(x, kblocks_div, total_blocks, ld, dense, bidx_first, stride, lane, sl);
+    m = amax_bits_of(sl);
+  } else {
+    for (uint32_t bidx0 = bidx_first; bidx0 < total_blocks; bidx0 += stride * kUnroll) {
+      BlockSlots t;
+      load_blocks(x, kblocks_div, total_blocks, ld, dense, bidx0, stride, lane, t);
+      m = max(m, amax_bits_of(t));
     }
-#pragma unroll
-    for (int u = 0; u < 2 * kUnroll; ++u) m = max(m, amax_bits_bf16x8(v[u]));
   }
   m = __reduce_max_sync(0xffffffffu, m);
   __shared__ uint32_t warp_max[kThreads / 32];
@@ -233,7 +268,14 @@ __global__ void __launch_bounds__(kThreads) quantize_dynamic_kernel(
   const float amax = __uint_as_float(s_amax << 16);
   const float g = amax > 0.0f ? __fdiv_rn(amax, 2688.0f) : 1.0f;
   if (blockIdx.x == 0 && threadIdx.x == 0) *g_out = g;
-  quantize_blocks<kMMA>(x, kblocks_div, total_blocks, ld, dense, rows, g, true, codes, scales);
+  if (resident) {
+    if (bidx_first < total_blocks)
+      quantize_loaded<kMMA>(sl, total_blocks, kblocks_div.d, bidx_first, stride, lane, g, __fmul_rn(6.0f, g), true,
+                            codes, scales);
+    if (kMMA) zero_scale_padding(rows, kblocks_div.d, scales);
+  } else {
+    quantize_blocks<kMMA>(x, kblocks_div, total_blocks, ld, dense, rows, g, true, codes, scales);
+  }
 }
 
 // Blocks of quantize_dynamic_kernel that fit on the device at once (a
@@ -377,6 +419,9 @@ NVFP4_API nvfp4_status nvfp4_quantize_dynamic(const void* x_bf16, int64_t rows, 
   if (cap <= 0) return NVFP4_ERR_CUDA;
   const uint32_t kblocks = static_cast<uint32_t>(cols / 16);
   const uint32_t total_blocks = static_cast<uint32_t>(rows * kblocks);
+  // kUnroll blocks per thread per pass, as few CTAs as that allows (each CTA
+  // is one arrival at the grid barrier); x stays in registers across the
+  // barrier when one pass covers it.
   int grid = grid_for(total_blocks, kThreads * kUnroll);
   if (grid > cap) grid = cap;
   // Cooperative: every block is resident at once, so the grid barrier can
