@@ -310,13 +310,15 @@ __global__ void __launch_bounds__(kThreads, NVFP4_ATTN_MIN_CTAS) attn_partial_ke
           if (rv[3] >= valid) vs89_raw &= 0x00FFu;
         }
         float mx0 = fmaxf(x0, x2), mx1 = fmaxf(x1, x3);
+        // The tile maximum is needed only when some logit exceeds the running
+        // maximum by more than the lazy threshold: vote first, reduce then.
+        if (__any_sync(0xffffffffu, mx0 > m_run[0] + kRescaleLog2 || mx1 > m_run[1] + kRescaleLog2)) {
 #pragma unroll
-        for (int sh = 4; sh < 32; sh <<= 1) {
-          mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, sh));
-          mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, sh));
-        }
-        const bool up0 = mx0 > m_run[0] + kRescaleLog2, up1 = mx1 > m_run[1] + kRescaleLog2;
-        if (__any_sync(0xffffffffu, up0 || up1)) {
+          for (int sh = 4; sh < 32; sh <<= 1) {
+            mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, sh));
+            mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, sh));
+          }
+          const bool up0 = mx0 > m_run[0] + kRescaleLog2, up1 = mx1 > m_run[1] + kRescaleLog2;
           const float al0 = up0 ? fast_exp2(m_run[0] - mx0) : 1.0f;
           const float al1 = up1 ? fast_exp2(m_run[1] - mx1) : 1.0f;
           if (up0) m_run[0] = mx0;
