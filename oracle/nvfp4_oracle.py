@@ -19,7 +19,9 @@ readability, not speed:
   with quantized K and V (Sec. 2.1), in fp64;
 * the inference-time Q-FIT key shift ``K~ = R(K_pre / s) - m`` applied before
   the KV cache is quantized (Eq. 2, Appendix D.3), and the RoPE / paired scaling
-  pieces needed to state its invariances (Sec. 2.1, Eq. 2).
+  pieces needed to state its invariances (Sec. 2.1, Eq. 2);
+* the fused step RoPE -> shift -> quantize -> append, with RoPE in fp32 from a
+  (cos, sin) table in a fixed order of operations (``rope_f32``).
 
 Floating-point conventions: the quantizer's arithmetic is IEEE fp32 with
 round-to-nearest-even (numpy float32 scalars/arrays, no fused multiply-add);
@@ -375,6 +377,44 @@ def rope(x, positions, theta=1.0e6):
     c, s = np.cos(ang), np.sin(ang)
     x1, x2 = x[..., :half], x[..., half:]
     return np.concatenate([x1 * c - x2 * s, x1 * s + x2 * c], axis=-1)
+
+
+def rope_table(n_pos, head_dim=128, theta=1.0e6):
+    """RoPE (cos, sin) table, float32 [n_pos, head_dim/2, 2]: the fp64 values of
+    cos/sin(pos * theta^(-2i/d)), i < d/2, rounded once to fp32 (Sec. 2.1; the
+    rotate-half pairing of ``rope``)."""
+    half = head_dim // 2
+    inv = theta ** (-np.arange(half) * 2.0 / head_dim)
+    ang = np.arange(n_pos, dtype=np.float64)[:, None] * inv[None, :]
+    return np.stack([np.cos(ang), np.sin(ang)], axis=-1).astype(np.float32)
+
+
+def rope_f32(x_f32, positions, table):
+    """RoPE in fp32 from a (cos, sin) table, the order of operations fixed so a
+    kernel can reproduce it exactly (round-to-nearest-even, no fused multiply-add):
+        y[i]       = fl(fl(x[i] * c_i) - fl(x[i + d/2] * s_i))
+        y[i + d/2] = fl(fl(x[i] * s_i) + fl(x[i + d/2] * c_i)),   i < d/2.
+    x_f32 [n, ..., d] (one row per position), positions [n]."""
+    x = np.asarray(x_f32, dtype=np.float32)
+    half = x.shape[-1] // 2
+    cs = np.asarray(table, dtype=np.float32)[np.asarray(positions)]      # [n, d/2, 2]
+    shape = (x.shape[0],) + (1,) * (x.ndim - 2) + (half,)
+    c = cs[..., 0].reshape(shape)
+    sn = cs[..., 1].reshape(shape)
+    x1, x2 = x[..., :half], x[..., half:]
+    y1 = (x1 * c).astype(np.float32) - (x2 * sn).astype(np.float32)
+    y2 = (x1 * sn).astype(np.float32) + (x2 * c).astype(np.float32)
+    return np.concatenate([y1, y2], axis=-1).astype(np.float32)
+
+
+def kv_append_rope(k_codes, k_scales, v_codes, v_scales, k_pre, v_new, seq_idx, pos, g_k, g_v, table,
+                   k_shift=None):
+    """The fused step before decode attention: K~ = RoPE(K_pre) - m (Eq. 2 with
+    the pre-RoPE scaling s folded into the key projection), then quantize and
+    store K~ and V as ``kv_append`` does.  k_pre: float32 [n_new, kv_heads, d]
+    (bf16 values, before RoPE); RoPE and the shift in fp32 (``rope_f32``)."""
+    k = rope_f32(k_pre, pos, table)
+    kv_append(k_codes, k_scales, v_codes, v_scales, k, v_new, seq_idx, pos, g_k, g_v, k_shift)
 
 
 def qfit_transform(q_pre, k_pre, s, m, positions, theta=1.0e6):

@@ -346,3 +346,63 @@ def test_kv_append_shift_is_subtracted_before_quantization():
     c, s = O.quantize(v[1], np.float32(0.02))
     assert np.array_equal(vc[0, :, 1], c) and np.array_equal(vs[0, :, 1], s)
     assert not kc[0, :, 0].any() and not kc[0, :, 3:5].any()
+
+
+# ------------------------------------------------- RoPE from a table (fp32) ---
+
+def test_rope_table_matches_closed_form_angles():
+    t = O.rope_table(5, head_dim=8, theta=10000.0)
+    assert t.dtype == np.float32 and t.shape == (5, 4, 2)
+    assert np.array_equal(t[0, :, 0], np.ones(4, np.float32)) and np.array_equal(t[0, :, 1], np.zeros(4, np.float32))
+    # channel 0 has frequency 1: angle = position exactly
+    assert np.array_equal(t[:, 0, 0], np.cos(np.arange(5.0)).astype(np.float32))
+    assert np.array_equal(t[:, 0, 1], np.sin(np.arange(5.0)).astype(np.float32))
+    # last pair: theta^(-2*3/8) = 10000^-0.75 = 0.001
+    assert np.allclose(t[3, 3, 1], np.sin(3 * 1e-3), rtol=1e-6)
+
+
+def test_rope_f32_position_zero_is_identity_and_matches_fp64_rope():
+    rng = np.random.default_rng(21)
+    x = rng.standard_normal((6, 3, 128)).astype(np.float32)
+    pos = np.array([0, 1, 7, 100, 4095, 16383])
+    tab = O.rope_table(16384)
+    y = O.rope_f32(x, pos, tab)
+    assert np.array_equal(y[0], x[0])                       # cos = 1, sin = 0 exactly
+    ref = O.rope(np.moveaxis(x, 0, -2), pos)                # fp64 closed form, [3, 6, 128]
+    ref = np.moveaxis(ref, -2, 0)
+    # fp32 table (|error| <= 2^-25) plus three fp32 roundings: a few ulps of the inputs' scale
+    assert np.abs(y - ref).max() <= 8 * np.finfo(np.float32).eps * np.abs(x).max()
+    # a rotation: each (i, i + 64) pair keeps its length
+    n_in = x[..., :64] ** 2 + x[..., 64:] ** 2
+    n_out = y.astype(np.float64)[..., :64] ** 2 + y.astype(np.float64)[..., 64:] ** 2
+    assert np.allclose(n_out, n_in, rtol=1e-5, atol=1e-6)
+
+
+def test_rope_f32_quarter_turn_swaps_halves():
+    # A table whose angle is pi/2 exactly in fp32 terms (cos 0, sin 1): y1 = -x2, y2 = x1.
+    tab = np.zeros((1, 64, 2), np.float32); tab[..., 1] = 1.0
+    x = np.random.default_rng(3).standard_normal((1, 2, 128)).astype(np.float32)
+    y = O.rope_f32(x, np.array([0]), tab)
+    assert np.array_equal(y[..., :64], -x[..., 64:]) and np.array_equal(y[..., 64:], x[..., :64])
+
+
+def test_kv_append_rope_equals_rope_then_shifted_append():
+    rng = np.random.default_rng(8)
+    B, H, T, n = 2, 2, 16, 5
+    tab = O.rope_table(T)
+    k = (rng.standard_normal((n, H, 128)) * 3).astype(np.float32)
+    v = rng.standard_normal((n, H, 128)).astype(np.float32)
+    m = rng.standard_normal((H, 128)).astype(np.float32)
+    seq = np.array([0, 1, 1, 0, 1]); pos = np.array([3, 0, 15, 9, 4])
+    bufs = lambda: [np.zeros((B, H, T, 64), np.uint8), np.zeros((B, H, T, 8), np.uint8),
+                    np.zeros((B, H, T, 64), np.uint8), np.zeros((B, H, T, 8), np.uint8)]
+    a, b = bufs(), bufs()
+    O.kv_append_rope(*a, k, v, seq, pos, np.float32(0.01), np.float32(0.02), tab, k_shift=m)
+    O.kv_append(*b, O.rope_f32(k, pos, tab), v, seq, pos, np.float32(0.01), np.float32(0.02), k_shift=m)
+    for u, w in zip(a, b):
+        assert np.array_equal(u, w)
+    # the shift is applied after RoPE: dequantized K~ + m is close to RoPE(K)
+    kc = a[0][seq, :, pos]; ks = a[1][seq, :, pos]
+    kh = O.dequantize(kc.reshape(n * H, 64), ks.reshape(n * H, 8), np.float32(0.01)).reshape(n, H, 128)
+    ref = np.moveaxis(O.rope(np.moveaxis(k, 0, -2), pos), -2, 0) - m
+    assert np.abs(kh - ref).max() <= 0.01 * 448 * 6 / 4 + 1e-3
