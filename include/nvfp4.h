@@ -198,6 +198,35 @@ nvfp4_status kv_append_nvfp4(const nvfp4_kv_cache* cache, const void* k_bf16, co
                              const float* k_shift, void* stream);
 
 /*
+ * The fused step before decode attention (a4 with RoPE): K~ = RoPE(K_pre, pos)
+ * - m, then quantize and store K~ and V exactly as kv_append_nvfp4 does (Eq. 2:
+ * K~ = R(K_pre / s) - m, with the pre-RoPE scaling s folded into the key
+ * projection weights offline, as the paired Q/K scaling allows).
+ *   k_pre_bf16 : [n_new, num_kv_heads, 128] bf16 keys before RoPE.
+ *   rope_table : fp32 [rope_positions, 64, 2], (cos, sin) of p * theta^(-2i/128)
+ *                for position p and pair i (nvfp4_rope_table writes one);
+ *                16-B aligned; rope_positions >= cache->capacity, else SHAPE.
+ * RoPE pairs channel i with i + 64 (rotate-half form) and is evaluated in fp32
+ * as y_i = x_i c_i - x_{i+64} s_i, y_{i+64} = x_i s_i + x_{i+64} c_i, each
+ * product and sum rounded to nearest even (no fused multiply-add).  Other
+ * arguments, errors and device-side checks as kv_append_nvfp4.
+ */
+nvfp4_status kv_append_rope_nvfp4(const nvfp4_kv_cache* cache, const void* k_pre_bf16, const void* v_bf16,
+                                  const int32_t* seq_idx, const int32_t* pos, int64_t n_new,
+                                  const float* rope_table, int64_t rope_positions, const float* k_shift,
+                                  void* stream);
+
+/*
+ * RoPE (cos, sin) table for kv_append_rope_nvfp4: table[p][i] = (cos, sin) of
+ * p * theta^(-2i/head_dim), p < n_pos, i < head_dim/2 (Sec. 2.1 RoPE; the
+ * evaluated models use theta = 1e6).  The angle and both functions are
+ * evaluated in fp64 and rounded once to fp32.  table: fp32 [n_pos,
+ * head_dim/2, 2], 8-B aligned.  Errors: head_dim odd or <= 0, n_pos < 0 ->
+ * SHAPE; theta <= 1 or not finite, table NULL with n_pos > 0 -> INVALID_ARG.
+ */
+nvfp4_status nvfp4_rope_table(float* table, int64_t n_pos, int32_t head_dim, float theta, void* stream);
+
+/*
  * a5. Decode attention straight from the NVFP4 cache (Sec. 2.1):
  *   out[b, h] = softmax(softmax_scale * q[b,h] . K_hat[b,kv,t]) V_hat[b,kv,t],
  *   t < seq_lens[b], kv = h / (num_q_heads / num_kv_heads) (contiguous

@@ -1,5 +1,6 @@
 // a4: quantize new K/V rows (optionally shifted by the Q-FIT post-RoPE vector
-// m, Eq. 2) and write them into the NVFP4 KV cache.
+// m, Eq. 2) and write them into the NVFP4 KV cache; optionally rotate K by
+// RoPE first (the fused RoPE -> shift -> quantize -> append step).
 //
 // Work item = one 8-element chunk of one 128-channel row; the 16 lanes that
 // hold a row cover its 8 blocks.  Item order (token, kv head, K|V, chunk) keeps
@@ -14,12 +15,17 @@ namespace {
 
 constexpr int kThreads = 256;
 
+// kRope: K arrives before RoPE and is rotated here (rotate-half pairing,
+// channel i with i + 64) with the (cos, sin) table row of its position, in
+// fp32: y_i = x_i c_i - x_{i+64} s_i, y_{i+64} = x_i s_i + x_{i+64} c_i.
+template <bool kRope>
 __global__ void __launch_bounds__(kThreads) kv_append_kernel(
     const uint16_t* __restrict__ k_in, const uint16_t* __restrict__ v_in, const int32_t* __restrict__ seq_idx,
-    const int32_t* __restrict__ pos, const float* __restrict__ k_shift, uint32_t n_rows /* n_new*H_kv */,
-    FastDiv hkv, uint32_t batch, uint32_t capacity, uint8_t* __restrict__ kc, uint8_t* __restrict__ ks,
-    uint8_t* __restrict__ vc, uint8_t* __restrict__ vs, float gk, float gv, int* status) {
-  const uint32_t total = n_rows * 32u;  // 2 tensors x 16 chunks per row
+    const int32_t* __restrict__ pos, const float* __restrict__ k_shift, const float* __restrict__ rope,
+    uint32_t n_rows /* n_new*H_kv */, FastDiv hkv, uint32_t batch, uint32_t capacity, uint8_t* __restrict__ kc,
+    uint8_t* __restrict__ ks, uint8_t* __restrict__ vc, uint8_t* __restrict__ vs, float gk, float gv, int* status) {
+  griddep_wait_and_release();
+  const uint32_t total = n_rows * 32u;  // 2 tensors x 16 chunks per row: a multiple of the warp
   const uint32_t lane = threadIdx.x & 31;
   const float six_gk = __fmul_rn(6.0f, gk), six_gv = __fmul_rn(6.0f, gv);
   for (uint32_t c0 = blockIdx.x * blockDim.x + (threadIdx.x & ~31u); c0 < total; c0 += gridDim.x * blockDim.x) {
@@ -34,6 +40,31 @@ __global__ void __launch_bounds__(kThreads) kv_append_kernel(
     if (live) raw = __ldg(reinterpret_cast<const uint4*>((is_v ? v_in : k_in) + static_cast<uint64_t>(rr) * 128 + j * 8));
     float x[8];
     unpack_bf16x8(raw, x);
+    if (kRope) {
+      // The partner chunk (channels 64 apart) is held by lane ^ 8; the whole warp is live.
+      uint4 pr;
+      pr.x = __shfl_xor_sync(0xffffffffu, raw.x, 8);
+      pr.y = __shfl_xor_sync(0xffffffffu, raw.y, 8);
+      pr.z = __shfl_xor_sync(0xffffffffu, raw.z, 8);
+      pr.w = __shfl_xor_sync(0xffffffffu, raw.w, 8);
+      if (live && !is_v) {
+        float xp[8];
+        unpack_bf16x8(pr, xp);
+        int32_t p = __ldg(pos + tok);
+        if (p < 0 || static_cast<uint32_t>(p) >= capacity) p = 0;  // reported as CAPACITY below
+        const float4* cs = reinterpret_cast<const float4*>(rope + (static_cast<uint64_t>(p) * 64 + (j & 7u) * 8) * 2);
+        float cv[8], sv[8];
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          const float4 t = __ldg(cs + q);
+          cv[2 * q] = t.x; sv[2 * q] = t.y; cv[2 * q + 1] = t.z; sv[2 * q + 1] = t.w;
+        }
+#pragma unroll
+        for (int e = 0; e < 8; ++e)
+          x[e] = j < 8 ? __fsub_rn(__fmul_rn(x[e], cv[e]), __fmul_rn(xp[e], sv[e]))
+                       : __fadd_rn(__fmul_rn(xp[e], sv[e]), __fmul_rn(x[e], cv[e]));
+      }
+    }
     if (live && !is_v && k_shift) {
       const float4* m4 = reinterpret_cast<const float4*>(k_shift + h * 128u + j * 8u);
       const float4 m0 = __ldg(m4), m1 = __ldg(m4 + 1);
@@ -61,14 +92,8 @@ __global__ void __launch_bounds__(kThreads) kv_append_kernel(
   }
 }
 
-}  // namespace
-}  // namespace nvfp4
-
-using namespace nvfp4;
-
-NVFP4_API nvfp4_status kv_append_nvfp4(const nvfp4_kv_cache* cache, const void* k_bf16, const void* v_bf16,
-                                       const int32_t* seq_idx, const int32_t* pos, int64_t n_new,
-                                       const float* k_shift, void* stream) {
+nvfp4_status append(const nvfp4_kv_cache* cache, const void* k_bf16, const void* v_bf16, const int32_t* seq_idx,
+                    const int32_t* pos, int64_t n_new, const float* k_shift, const float* rope, void* stream) {
   if (!cache || !k_bf16 || !v_bf16 || !seq_idx || !pos) return NVFP4_ERR_INVALID_ARG;
   if (!cache->k_codes || !cache->k_scales || !cache->v_codes || !cache->v_scales) return NVFP4_ERR_INVALID_ARG;
   if (!(cache->k_gscale > 0.0f && cache->k_gscale <= FLT_MAX) || !(cache->v_gscale > 0.0f && cache->v_gscale <= FLT_MAX))
@@ -77,7 +102,8 @@ NVFP4_API nvfp4_status kv_append_nvfp4(const nvfp4_kv_cache* cache, const void* 
     return NVFP4_ERR_SHAPE;
   if (n_new * cache->num_kv_heads * 32 >= (1ll << 32)) return NVFP4_ERR_SHAPE;
   if (!aligned(k_bf16, 16) || !aligned(v_bf16, 16) || !aligned(cache->k_codes, 16) || !aligned(cache->v_codes, 16) ||
-      !aligned(cache->k_scales, 8) || !aligned(cache->v_scales, 8) || (k_shift && !aligned(k_shift, 16)))
+      !aligned(cache->k_scales, 8) || !aligned(cache->v_scales, 8) || (k_shift && !aligned(k_shift, 16)) ||
+      (rope && !aligned(rope, 16)))
     return NVFP4_ERR_ALIGN;
   if (n_new == 0) return NVFP4_OK;
   const uint32_t n_rows = static_cast<uint32_t>(n_new * cache->num_kv_heads);
@@ -85,11 +111,66 @@ NVFP4_API nvfp4_status kv_append_nvfp4(const nvfp4_kv_cache* cache, const void* 
   uint64_t grid = (items + kThreads - 1) / kThreads;
   const uint64_t cap = static_cast<uint64_t>(sm_count()) * 8;
   if (grid > cap) grid = cap;
-  if (launch_pdl(kv_append_kernel, dim3(static_cast<int>(grid)), dim3(kThreads), 0, static_cast<cudaStream_t>(stream),
-                 static_cast<const uint16_t*>(k_bf16), static_cast<const uint16_t*>(v_bf16), seq_idx, pos, k_shift,
-                 n_rows, FastDiv(static_cast<uint32_t>(cache->num_kv_heads)), static_cast<uint32_t>(cache->batch),
+  const cudaError_t e =
+      launch_pdl(rope ? kv_append_kernel<true> : kv_append_kernel<false>, dim3(static_cast<int>(grid)), dim3(kThreads),
+                 0, static_cast<cudaStream_t>(stream), static_cast<const uint16_t*>(k_bf16),
+                 static_cast<const uint16_t*>(v_bf16), seq_idx, pos, k_shift, rope, n_rows,
+                 FastDiv(static_cast<uint32_t>(cache->num_kv_heads)), static_cast<uint32_t>(cache->batch),
                  static_cast<uint32_t>(cache->capacity), cache->k_codes, cache->k_scales, cache->v_codes,
-                 cache->v_scales, cache->k_gscale, cache->v_gscale, status_word_dev()) != cudaSuccess)
+                 cache->v_scales, cache->k_gscale, cache->v_gscale, status_word_dev());
+  if (e != cudaSuccess) return NVFP4_ERR_CUDA;
+  count_launches(1);
+  return launch_status();
+}
+
+// table[p][i] = (cos, sin) of p * theta^(-2i/d): angle, sine and cosine in
+// fp64, each of the two results rounded once to fp32.
+__global__ void rope_table_kernel(float2* __restrict__ table, uint32_t n_pos, uint32_t half, double theta, double d) {
+  griddep_wait_and_release();
+  const uint64_t n = static_cast<uint64_t>(n_pos) * half;
+  for (uint64_t k = blockIdx.x * static_cast<uint64_t>(blockDim.x) + threadIdx.x; k < n;
+       k += static_cast<uint64_t>(gridDim.x) * blockDim.x) {
+    const uint32_t p = static_cast<uint32_t>(k / half), i = static_cast<uint32_t>(k % half);
+    const double inv = pow(theta, -2.0 * static_cast<double>(i) / d);
+    double sn, cs;
+    sincos(static_cast<double>(p) * inv, &sn, &cs);
+    table[k] = make_float2(static_cast<float>(cs), static_cast<float>(sn));
+  }
+}
+
+}  // namespace
+}  // namespace nvfp4
+
+using namespace nvfp4;
+
+NVFP4_API nvfp4_status kv_append_nvfp4(const nvfp4_kv_cache* cache, const void* k_bf16, const void* v_bf16,
+                                       const int32_t* seq_idx, const int32_t* pos, int64_t n_new,
+                                       const float* k_shift, void* stream) {
+  return append(cache, k_bf16, v_bf16, seq_idx, pos, n_new, k_shift, nullptr, stream);
+}
+
+NVFP4_API nvfp4_status kv_append_rope_nvfp4(const nvfp4_kv_cache* cache, const void* k_pre_bf16, const void* v_bf16,
+                                            const int32_t* seq_idx, const int32_t* pos, int64_t n_new,
+                                            const float* rope_table, int64_t rope_positions, const float* k_shift,
+                                            void* stream) {
+  if (!cache || !rope_table) return NVFP4_ERR_INVALID_ARG;
+  if (rope_positions < cache->capacity) return NVFP4_ERR_SHAPE;
+  return append(cache, k_pre_bf16, v_bf16, seq_idx, pos, n_new, k_shift, rope_table, stream);
+}
+
+NVFP4_API nvfp4_status nvfp4_rope_table(float* table, int64_t n_pos, int32_t head_dim, float theta, void* stream) {
+  if (n_pos < 0 || head_dim <= 0 || head_dim % 2 || n_pos * (head_dim / 2) >= (1ll << 40)) return NVFP4_ERR_SHAPE;
+  if (!(theta > 1.0f && theta <= FLT_MAX)) return NVFP4_ERR_INVALID_ARG;
+  if (n_pos == 0) return NVFP4_OK;
+  if (!table) return NVFP4_ERR_INVALID_ARG;
+  if (!aligned(table, 8)) return NVFP4_ERR_ALIGN;
+  const uint64_t n = static_cast<uint64_t>(n_pos) * (head_dim / 2);
+  uint64_t grid = (n + 255) / 256;
+  const uint64_t cap = static_cast<uint64_t>(sm_count()) * 8;
+  if (grid > cap) grid = cap;
+  if (launch_pdl(rope_table_kernel, dim3(static_cast<int>(grid)), dim3(256), 0, static_cast<cudaStream_t>(stream),
+                 reinterpret_cast<float2*>(table), static_cast<uint32_t>(n_pos), static_cast<uint32_t>(head_dim / 2),
+                 static_cast<double>(theta), static_cast<double>(head_dim)) != cudaSuccess)
     return NVFP4_ERR_CUDA;
   count_launches(1);
   return launch_status();

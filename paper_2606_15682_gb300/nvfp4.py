@@ -55,6 +55,9 @@ _quantize_dynamic = _sig("nvfp4_quantize_dynamic", [_p, _i64, _i64, _i64, _p, _p
 _relayout = _sig("nvfp4_scales_relayout", [_p, _p, _i64, _i64, ctypes.c_int, ctypes.c_int, _p])
 _linear = _sig("nvfp4_linear", [_p, _p, _p, _p, _p, _p, _i64, _i64, _i64, _p, _i64, _p])
 _kv_append = _sig("kv_append_nvfp4", [ctypes.POINTER(KVCacheStruct), _p, _p, _p, _p, _i64, _p, _p])
+_kv_append_rope = _sig("kv_append_rope_nvfp4",
+                       [ctypes.POINTER(KVCacheStruct), _p, _p, _p, _p, _i64, _p, _i64, _p, _p])
+_rope_table = _sig("nvfp4_rope_table", [_p, _i64, _i32, _f32, _p])
 _attn_ws = _sig("decode_attention_nvfp4_workspace_size", [_i32, _i32, _i32], _sz)
 _attn = _sig("decode_attention_nvfp4", [ctypes.POINTER(KVCacheStruct), _p, _i32, _f32, _p, _p, _sz, _p])
 _attn_static = _sig("decode_attention_nvfp4_static_scratch", [ctypes.POINTER(KVCacheStruct), _p, _i32, _f32, _p, _p])
@@ -136,6 +139,19 @@ def kv_append_nvfp4(cache, k, v, seq_idx, pos, k_shift=None, stream=None):
                                          _ptr(k_shift), _stream(stream)))
 
 
+def kv_append_rope_nvfp4(cache, k_pre, v, seq_idx, pos, rope_table, k_shift=None, stream=None):
+    """rope_table: float32 [n_pos, 64, 2] (see nvfp4_rope_table), n_pos >= cache.capacity."""
+    s = cache.struct()
+    _check("kv_append_rope_nvfp4",
+           _kv_append_rope(ctypes.byref(s), _ptr(k_pre), _ptr(v), _ptr(seq_idx), _ptr(pos), k_pre.shape[0],
+                           _ptr(rope_table), rope_table.shape[0], _ptr(k_shift), _stream(stream)))
+
+
+def nvfp4_rope_table(table, theta=1.0e6, stream=None):
+    """Fill table (float32 [n_pos, head_dim/2, 2]) with (cos, sin) of p * theta^(-2i/head_dim)."""
+    _check("nvfp4_rope_table", _rope_table(_ptr(table), table.shape[0], 2 * table.shape[1], theta, _stream(stream)))
+
+
 def decode_attention_nvfp4_workspace_size(batch, num_q_heads, capacity):
     return int(_attn_ws(batch, num_q_heads, capacity))
 
@@ -193,6 +209,6 @@ class KVCache:
 
 
 EXPORTED = ["nvfp4_scales_bytes", "nvfp4_tensor_scale", "nvfp4_quantize", "nvfp4_quantize_dynamic", "nvfp4_scales_relayout", "nvfp4_linear",
-            "kv_append_nvfp4", "decode_attention_nvfp4_workspace_size", "decode_attention_nvfp4",
+            "kv_append_nvfp4", "kv_append_rope_nvfp4", "nvfp4_rope_table", "decode_attention_nvfp4_workspace_size", "decode_attention_nvfp4",
             "decode_attention_nvfp4_static_scratch",
             "nvfp4_get_device_status", "nvfp4_status_string", "nvfp4_launch_count"]

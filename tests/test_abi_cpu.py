@@ -77,6 +77,15 @@ def test_kv_and_attention_validation():
     assert L.kv_append_nvfp4(ctypes.byref(cache(head_dim=64)), p, p, p, p, 1, None, s) == 2
     assert L.kv_append_nvfp4(ctypes.byref(cache(k_gscale=0.0)), p, p, p, p, 1, None, s) == 1
     assert L.kv_append_nvfp4(ctypes.byref(cache()), None, p, p, p, 1, None, s) == 1
+    # fused RoPE append: table required, and it must cover every cache position
+    odd = ctypes.c_void_p(0x10004)
+    assert L.kv_append_rope_nvfp4(ctypes.byref(cache()), p, p, p, p, 1, None, 64, None, s) == 1
+    assert L.kv_append_rope_nvfp4(ctypes.byref(cache()), p, p, p, p, 1, p, 63, None, s) == 2
+    assert L.kv_append_rope_nvfp4(ctypes.byref(cache()), p, p, p, p, 1, odd, 64, None, s) == 3
+    assert L.nvfp4_rope_table(p, 16, 127, ctypes.c_float(1e6), s) == 2          # odd head_dim
+    assert L.nvfp4_rope_table(p, 16, 128, ctypes.c_float(0.5), s) == 1          # theta <= 1
+    assert L.nvfp4_rope_table(None, 16, 128, ctypes.c_float(1e6), s) == 1
+    assert L.nvfp4_rope_table(None, 0, 128, ctypes.c_float(1e6), s) == 0        # empty: nothing to do
     ws = N.decode_attention_nvfp4_workspace_size(2, 4, 64)
     assert L.decode_attention_nvfp4(ctypes.byref(cache()), p, 3, ctypes.c_float(0.1), p, p, ws, s) == 2   # 3 % 2
     assert L.decode_attention_nvfp4(ctypes.byref(cache()), p, 18, ctypes.c_float(0.1), p, p, 1 << 30, s) == 2  # group 9

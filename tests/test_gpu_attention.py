@@ -187,3 +187,83 @@ def test_full_size_decode_attention_workload(N):
         assert np.array_equal(u8(cache.v_codes[b:b + 1]), rvc) and np.array_equal(u8(cache.v_scales[b:b + 1]), rvs)
         ref = O.decode_attention(f32(q[b:b + 1]), rkc, rks, rvc, rvs, [T], gk_ref, gv_ref, 1.0 / math.sqrt(128))
         assert_close(f32(out[b]), ref[0], what=f"seq {b}")
+
+
+# ----------------------------------- fused RoPE -> shift -> quantize -> append ---
+
+def test_rope_table_matches_numpy(N):
+    n_pos = 16384
+    t = torch.empty(n_pos, 64, 2, dtype=torch.float32, device="cuda")
+    N.nvfp4_rope_table(t, theta=1.0e6)
+    torch.cuda.synchronize()
+    ref = O.rope_table(n_pos)
+    got = t.cpu().numpy()
+    # both sides round an fp64 value once to fp32: equal except where the fp64
+    # results straddle a rounding boundary (then one fp32 ulp apart)
+    diff = np.abs(got.view(np.int32).astype(np.int64) - ref.view(np.int32).astype(np.int64))
+    assert diff.max() <= 1 and (diff != 0).mean() < 1e-3, (diff.max(), (diff != 0).mean())
+
+
+@pytest.mark.parametrize("shifted", [False, True])
+def test_kv_append_rope_bit_exact(N, shifted):
+    """Codes and scales equal the oracle's RoPE -> shift -> quantize on the same fp32 table."""
+    B, hkv, cap, n = 3, 8, 64, 150
+    rec = synth.KVRecipe(hkv, seed=91)
+    k, v = rec.kv(n, seed=6)                     # bf16 [n, hkv, 128], used here as pre-RoPE keys
+    rng = np.random.default_rng(11)
+    seq = rng.integers(0, B, n); pos = rng.permutation(B * cap)[:n] % cap
+    pairs = {}
+    for i in range(n):
+        pairs[(seq[i], pos[i])] = i
+    keep = np.array(sorted(pairs.values()))
+    k, v, seq, pos = k[keep], v[keep], seq[keep], pos[keep]
+    table = O.rope_table(cap)
+    krot = O.rope_f32(f32(k), pos, table)
+    shift = (krot.mean(axis=0) * 0.5).astype(np.float32) if shifted else None
+    gk = O.tensor_scale((krot - (shift if shifted else 0)).astype(np.float32))
+    gv = O.tensor_scale(f32(v))
+    cache = N.KVCache(B, hkv, cap, gk, gv)
+    N.kv_append_rope_nvfp4(cache, k.cuda(), v.cuda(), torch.as_tensor(seq, dtype=torch.int32, device="cuda"),
+                           torch.as_tensor(pos, dtype=torch.int32, device="cuda"), torch.from_numpy(table).cuda(),
+                           None if shift is None else torch.from_numpy(shift).cuda())
+    torch.cuda.synchronize()
+    assert N.nvfp4_get_device_status() == 0
+    rkc, rks, rvc, rvs = oracle_cache(B, hkv, cap)
+    O.kv_append_rope(rkc, rks, rvc, rvs, f32(k), f32(v), seq, pos, np.float32(gk), np.float32(gv), table,
+                     k_shift=shift)
+    assert np.array_equal(u8(cache.k_scales), rks) and np.array_equal(u8(cache.k_codes), rkc)
+    assert np.array_equal(u8(cache.v_codes), rvc) and np.array_equal(u8(cache.v_scales), rvs)
+
+
+def test_kv_append_rope_then_attention_matches_fp64(N):
+    """End to end: pre-RoPE keys through the fused append, then decode attention,
+    against fp64 attention on the oracle's dequantized cache."""
+    B, hq, hkv, T = 2, 10, 2, 300
+    cap = T + (T & 1)
+    rec = synth.KVRecipe(hkv, seed=12)
+    table = O.rope_table(cap)
+    cache = N.KVCache(B, hkv, cap, 1.0, 1.0)
+    ks, vs = [], []
+    for b in range(B):
+        k, v = rec.kv(T, seed=100 + b)
+        ks.append(k); vs.append(v)
+    kall = torch.cat(ks); vall = torch.cat(vs)
+    seq = np.repeat(np.arange(B), T); pos = np.tile(np.arange(T), B)
+    krot = O.rope_f32(f32(kall), pos, table)
+    gk, gv = O.tensor_scale(krot), O.tensor_scale(f32(vall))
+    cache.k_gscale, cache.v_gscale = float(gk), float(gv)
+    N.kv_append_rope_nvfp4(cache, kall.cuda(), vall.cuda(), torch.as_tensor(seq, dtype=torch.int32, device="cuda"),
+                           torch.as_tensor(pos, dtype=torch.int32, device="cuda"), torch.from_numpy(table).cuda())
+    cache.seq_lens.fill_(T)
+    q = rec.queries(B, hq, seed=7)
+    out = torch.empty(B, hq, 128, dtype=torch.bfloat16, device="cuda")
+    ws = torch.empty(N.decode_attention_nvfp4_workspace_size(B, hq, cap) // 4, dtype=torch.float32, device="cuda")
+    N.decode_attention_nvfp4(cache, q.cuda(), 1 / math.sqrt(128), out, ws)
+    torch.cuda.synchronize()
+    assert N.nvfp4_get_device_status() == 0
+    rkc, rks, rvc, rvs = oracle_cache(B, hkv, cap)
+    O.kv_append_rope(rkc, rks, rvc, rvs, f32(kall), f32(vall), seq, pos, np.float32(gk), np.float32(gv), table)
+    ref = O.decode_attention(f32(q), rkc, rks, rvc, rvs, np.full(B, T), np.float32(gk), np.float32(gv),
+                             1 / math.sqrt(128))
+    for b in range(B):
+        assert_close(f32(out)[b], ref[b], what=f"seq {b}")
