@@ -21,7 +21,9 @@ readability, not speed:
   the KV cache is quantized (Eq. 2, Appendix D.3), and the RoPE / paired scaling
   pieces needed to state its invariances (Sec. 2.1, Eq. 2);
 * the fused step RoPE -> shift -> quantize -> append, with RoPE in fp32 from a
-  (cos, sin) table in a fixed order of operations (``rope_f32``).
+  (cos, sin) table in a fixed order of operations (``rope_f32``);
+* the gate_up projection with the SwiGLU product and the NVFP4 quantization of
+  the down projection's input fused behind it (``linear_swiglu_quantize``).
 
 Floating-point conventions: the quantizer's arithmetic is IEEE fp32 with
 round-to-nearest-even (numpy float32 scalars/arrays, no fused multiply-add);
@@ -274,6 +276,38 @@ def linear(a_codes, a_scales, g_a, w_codes, w_scales, g_w):
     a = dequantize(a_codes, a_scales, g_a)
     w = dequantize(w_codes, w_scales, g_w)
     return a @ w.T
+
+
+def silu(x):
+    """SiLU(x) = x * sigmoid(x) = x / (1 + e^-x), fp64 (the SwiGLU gate of the
+    evaluated models' MLP, whose output feeds the quantized down projection)."""
+    x = np.asarray(x, dtype=np.float64)
+    return x / (1.0 + np.exp(-x))
+
+
+def interleave_gate_up(w_gate, w_up):
+    """Row order of the gate/up weight for the fused SwiGLU epilogue: blocks of
+    16 gate rows alternate with the matching 16 up rows,
+        out[32 j + t] = gate[16 j + t],  out[32 j + 16 + t] = up[16 j + t],  t < 16."""
+    g = np.asarray(w_gate); u = np.asarray(w_up)
+    I = g.shape[0]
+    out = np.empty((2 * I,) + g.shape[1:], dtype=g.dtype)
+    for j in range(I // 16):
+        out[32 * j:32 * j + 16] = g[16 * j:16 * j + 16]
+        out[32 * j + 16:32 * j + 32] = u[16 * j:16 * j + 16]
+    return out
+
+
+def linear_swiglu_quantize(a_codes, a_scales, g_a, wg_codes, wg_scales, wu_codes, wu_scales, g_w, g_out):
+    """The down projection's input, h = SiLU(A W_gate^T) * (A W_up^T), from the
+    NVFP4 operands in fp64, then NVFP4-quantized with the static scale g_out
+    (same recipe as ``quantize``, applied to h rounded to fp32).  Returns
+    (h fp64, codes, scales)."""
+    G = linear(a_codes, a_scales, g_a, wg_codes, wg_scales, g_w)
+    U = linear(a_codes, a_scales, g_a, wu_codes, wu_scales, g_w)
+    h = silu(G) * U
+    codes, scales = quantize(h.astype(np.float32), np.float32(g_out))
+    return h, codes, scales
 
 
 def linear_rows(a_codes, a_scales, g_a, w_codes, w_scales, g_w, rows):

@@ -406,3 +406,42 @@ def test_kv_append_rope_equals_rope_then_shifted_append():
     kh = O.dequantize(kc.reshape(n * H, 64), ks.reshape(n * H, 8), np.float32(0.01)).reshape(n, H, 128)
     ref = np.moveaxis(O.rope(np.moveaxis(k, 0, -2), pos), -2, 0) - m
     assert np.abs(kh - ref).max() <= 0.01 * 448 * 6 / 4 + 1e-3
+
+
+# ------------------------------------------- SwiGLU + quantize after gate_up ---
+
+def test_silu_closed_forms():
+    assert O.silu(0.0) == 0.0
+    assert np.isclose(O.silu(1.0), 1.0 / (1.0 + np.exp(-1.0)), rtol=1e-15)
+    x = np.linspace(-30, 30, 61)
+    assert np.allclose(O.silu(-x), O.silu(x) - x, atol=1e-12)       # sigmoid(-x) = 1 - sigmoid(x)
+    assert np.allclose(O.silu(np.array([50.0, 100.0])), [50.0, 100.0])
+    assert np.abs(O.silu(np.array([-50.0, -100.0]))).max() < 1e-18
+    assert np.isclose(O.silu(-1.2784645), -0.2784645, atol=1e-6)    # the minimum of x*sigmoid(x)
+
+
+def test_interleave_gate_up_row_order():
+    I, K = 48, 3
+    g = np.arange(I * K).reshape(I, K); u = -np.arange(I * K).reshape(I, K) - 1
+    w = O.interleave_gate_up(g, u)
+    assert w.shape == (2 * I, K)
+    assert np.array_equal(w[0:16], g[0:16]) and np.array_equal(w[16:32], u[0:16])
+    assert np.array_equal(w[64:80], g[32:48]) and np.array_equal(w[80:96], u[32:48])
+    assert sorted(map(tuple, w.tolist())) == sorted(map(tuple, np.concatenate([g, u]).tolist()))
+
+
+def test_linear_swiglu_quantize_brute_force():
+    rng = np.random.default_rng(4)
+    M, I, K = 3, 16, 32
+    a_c = rng.integers(0, 256, (M, K // 2)).astype(np.uint8); a_s = rng.integers(0x30, 0x40, (M, K // 16)).astype(np.uint8)
+    g_c = rng.integers(0, 256, (I, K // 2)).astype(np.uint8); g_s = rng.integers(0x30, 0x40, (I, K // 16)).astype(np.uint8)
+    u_c = rng.integers(0, 256, (I, K // 2)).astype(np.uint8); u_s = rng.integers(0x30, 0x40, (I, K // 16)).astype(np.uint8)
+    ga, gw = np.float32(0.25), np.float32(0.5)
+    h, codes, scales = O.linear_swiglu_quantize(a_c, a_s, ga, g_c, g_s, u_c, u_s, gw, np.float32(0.01))
+    A = O.dequantize(a_c, a_s, ga); Wg = O.dequantize(g_c, g_s, gw); Wu = O.dequantize(u_c, u_s, gw)
+    for m in range(M):
+        for i in range(I):
+            gs = sum(A[m, k] * Wg[i, k] for k in range(K)); us = sum(A[m, k] * Wu[i, k] for k in range(K))
+            assert np.isclose(h[m, i], gs / (1 + np.exp(-gs)) * us, rtol=1e-12, atol=1e-12)
+    rc, rs = O.quantize(h.astype(np.float32), np.float32(0.01))
+    assert np.array_equal(codes, rc) and np.array_equal(scales, rs)
