@@ -158,6 +158,42 @@ nvfp4_status nvfp4_linear(const uint8_t* a_codes, const uint8_t* a_scales, const
                           void* stream);
 
 /*
+ * a3 for the gate_up projection, with the down projection's input produced in
+ * the epilogue: h[m, i] = SiLU(G[m, i]) * U[m, i], where G and U are the gate
+ * and up halves of the block-scaled product exactly as nvfp4_linear forms them
+ * (fp32, scaled by g_a g_w, not rounded to bf16).  h is then NVFP4-quantized
+ * with the static tensor scale g_out by the recipe of nvfp4_quantize and
+ * written as the A operand of the down projection.  Every linear of the layer
+ * is quantized (Appendix D.1); the paper's Q-FIT appendix notes that SwiGLU
+ * makes the down projection's input the outlier-heavy activation.
+ *   w_codes, w_scales : the [2I, K] gate/up weight, rows interleaved in blocks
+ *                       of 16 (gate rows 16j..16j+15, then up rows 16j..16j+15;
+ *                       nvfp4_interleave_gate_up on the bf16 weights, then
+ *                       nvfp4_quantize with MMA scales).
+ *   g_out             : device float, static scale of h (e.g. calibrated).
+ *   out_codes         : [M, I/2] bytes, 16-B aligned.
+ *   out_scales        : nvfp4_scales_bytes(M, I, NVFP4_SCALES_MMA) bytes, 4-B
+ *                       aligned; padding rows are written as zeros.
+ * SiLU uses the fast exponential (__expf): h may differ from an exact SiLU by
+ * a few fp32 ulps, which can change a code only where h sits on a rounding
+ * boundary.  I % 128 == 0, K % 256 == 0, M, I, K > 0 (SHAPE).  g_out <= 0 or
+ * non-finite: zero codes and scales, INVALID_ARG set on the device.
+ */
+nvfp4_status nvfp4_linear_swiglu_quantize(const uint8_t* a_codes, const uint8_t* a_scales, const float* g_a,
+                                          const uint8_t* w_codes, const uint8_t* w_scales, const float* g_w,
+                                          int64_t M, int64_t I, int64_t K, const float* g_out,
+                                          uint8_t* out_codes, uint8_t* out_scales, void* stream);
+
+/*
+ * Row order for nvfp4_linear_swiglu_quantize: w_out row 32j + t = w_gate row
+ * 16j + t and w_out row 32j + 16 + t = w_up row 16j + t (t < 16).  w_gate,
+ * w_up: [I, *] rows of row_bytes bytes; w_out: [2I, *].  I % 16 == 0,
+ * row_bytes % 16 == 0 (SHAPE); pointers 16-B aligned (ALIGN).
+ */
+nvfp4_status nvfp4_interleave_gate_up(const void* w_gate, const void* w_up, int64_t I, int64_t row_bytes,
+                                      void* w_out, void* stream);
+
+/*
  * NVFP4 KV cache (W4A4KV4; the B200 deployment uses a native 4-bit KV cache,
  * Appendix D.3).  One row per (sequence, KV head, position); the 16-element
  * blocks run along head_dim, so an appended token never touches older rows.

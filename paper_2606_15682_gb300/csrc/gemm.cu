@@ -30,6 +30,7 @@
 #include <mutex>
 
 #include "common.cuh"
+#include "nvfp4_quant.cuh"
 
 namespace nvfp4 {
 namespace {
@@ -150,6 +151,10 @@ struct GemmArgs {
   int M, N, K;
   int tiles_m, tiles_n;
   int* status;
+  // Fused SwiGLU + quantization epilogue (pair kernel, kSwiGLU): outputs.
+  uint8_t* q_codes;   // [M, N/4] bytes: N/2 SwiGLU outputs per row
+  uint8_t* q_scales;  // MMA layout for [M, N/2]
+  const float* g_out;
 };
 
 template <class C>
@@ -480,7 +485,7 @@ struct PairCfg {
   static_assert(kSmemBytes <= 227 * 1024, "shared memory budget");
 };
 
-template <class C>
+template <class C, bool kSwiGLU>
 __global__ void __launch_bounds__(C::kThreads, 1)
     nvfp4_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_constant__ CUtensorMap tmap_b,
                            const __grid_constant__ CUtensorMap tmap_sfa, const __grid_constant__ CUtensorMap tmap_sfb,
@@ -662,6 +667,76 @@ __global__ void __launch_bounds__(C::kThreads, 1)
     }
     tc_commit_pair(drain_cp, 0x1);
     mbar_wait_bounded(drain_cp, 0, nullptr);
+  } else if (kSwiGLU && warp >= 2 + C::kCopyWarps) {
+    // ------------------------------------- epilogue: SwiGLU + NVFP4 output ---
+    // W rows are interleaved in blocks of 16 (gate, then the matching up), so
+    // each 32-column TMEM load gives a thread 16 gate and 16 up values of its
+    // row: one 16-element block of h = SiLU(gate) * up, quantized here with
+    // the static scale g_out by the library's recipe.  A warp's 128 columns
+    // are 64 outputs = 4 blocks = 32 code bytes and one 32-bit scale word.
+    constexpr int kEpi0 = 2 + C::kCopyWarps;
+    const int quarter = warp & 3;
+    const int colbase = ((warp - kEpi0) >> 2) * 128;
+    const float scale = __fmul_rn(__ldg(args.ga), __ldg(args.gb));
+    const float g_in = __ldg(args.g_out);
+    const bool g_ok = g_in > 0.0f && g_in <= FLT_MAX;
+    if (!g_ok && blockIdx.x == 0 && threadIdx.x == 32 * kEpi0) set_status(args.status, NVFP4_ERR_INVALID_ARG);
+    const float g = g_ok ? g_in : 1.0f, six_g = __fmul_rn(6.0f, g);
+    const uint32_t q_cols = static_cast<uint32_t>(args.N) >> 1;  // SwiGLU outputs per row
+    const uint32_t q_kgroups = q_cols >> 6;
+    int local = 0;
+    for (int u = pair_id; u < total_units; u += n_pairs, ++local) {
+      int ms, nb;
+      unit_coords(u, msup, args.tiles_n, &ms, &nb);
+      const int mb = ms * 2 + static_cast<int>(rank);  // mb >= tiles_m: nothing is stored
+      int ok = 1;
+      if (lane == 0) {
+        ok = !abort_flag && mbar_wait_bounded(tfull, local & 1, &abort_flag);
+        if (!ok && !abort_flag) fail();
+      }
+      if (!__shfl_sync(0xffffffffu, ok, 0)) break;
+      tc_fence_after();
+      uint32_t r[128];
+      const uint32_t taddr = tmem + (static_cast<uint32_t>(quarter * 32) << 16) + colbase;
+#pragma unroll
+      for (int c = 0; c < 4; ++c) tmem_ld32(taddr + c * 32, r + 32 * c);
+      tmem_ld_wait();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive_cluster_relaxed(tempty, 0);
+      // The MMAs of the next tile run while this warp computes and stores.
+      const uint32_t row = static_cast<uint32_t>(mb * BM + quarter * 32 + lane);
+      const uint32_t oc0 = static_cast<uint32_t>(nb) * (BN / 2) + static_cast<uint32_t>(colbase / 2);
+      uint32_t codes[8], sc = 0;
+#pragma unroll
+      for (int c = 0; c < 4; ++c) {
+        float h[16];
+        float amax = 0.0f;
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+          const float gt = __uint_as_float(r[32 * c + i]) * scale;
+          const float up = __uint_as_float(r[32 * c + 16 + i]) * scale;
+          h[i] = gt * __frcp_rn(1.0f + __expf(-gt)) * up;
+          amax = fmaxf(amax, fabsf(h[i]));
+        }
+        const BlockScale bs = block_scale(amax, g, six_g);
+#pragma unroll
+        for (int i = 0; i < 16; ++i) h[i] = __fmul_rn(h[i], bs.mult);
+        codes[2 * c] = g_ok ? e2m1x8(h) : 0u;
+        codes[2 * c + 1] = g_ok ? e2m1x8(h + 8) : 0u;
+        sc |= (g_ok ? bs.code : 0u) << (8 * c);
+      }
+      if (mb < args.tiles_m) {
+        // Scales for every row of the 128-row tile (rows past M hold zeros: A's
+        // missing rows load as zeros), codes for rows < M.
+        *reinterpret_cast<uint32_t*>(args.q_scales + mma_scale_offset(row, oc0 / 16, q_kgroups)) = sc;
+        if (row < static_cast<uint32_t>(args.M)) {
+          uint4* dst = reinterpret_cast<uint4*>(args.q_codes + static_cast<uint64_t>(row) * (q_cols / 2) + oc0 / 2);
+          dst[0] = make_uint4(codes[0], codes[1], codes[2], codes[3]);
+          dst[1] = make_uint4(codes[4], codes[5], codes[6], codes[7]);
+        }
+      }
+    }
   } else if (warp >= 2 + C::kCopyWarps) {
     // --------------------------------------------------------- epilogue ---
     constexpr int kEpi0 = 2 + C::kCopyWarps;
@@ -862,7 +937,7 @@ nvfp4_status launch(const uint8_t* a_codes, const uint8_t* a_scales, const float
   return launch_status();
 }
 
-template <class C>
+template <class C, bool kSwiGLU>
 int resident_pairs() {
   static std::mutex mu;
   static std::map<int, int> cache;
@@ -871,7 +946,7 @@ int resident_pairs() {
   std::lock_guard<std::mutex> lock(mu);
   auto it = cache.find(d);
   if (it != cache.end()) return it->second;
-  if (cudaFuncSetAttribute(nvfp4_gemm_pair_kernel<C>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  if (cudaFuncSetAttribute(nvfp4_gemm_pair_kernel<C, kSwiGLU>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                            static_cast<int>(C::kSmemBytes)) != cudaSuccess)
     return 0;
   cudaLaunchConfig_t cfg = {};
@@ -888,7 +963,8 @@ int resident_pairs() {
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   int clusters = 0;
-  if (cudaOccupancyMaxActiveClusters(&clusters, nvfp4_gemm_pair_kernel<C>, &cfg) != cudaSuccess || clusters <= 0) {
+  if (cudaOccupancyMaxActiveClusters(&clusters, nvfp4_gemm_pair_kernel<C, kSwiGLU>, &cfg) != cudaSuccess ||
+      clusters <= 0) {
     cudaGetLastError();
     return 0;
   }
@@ -896,21 +972,25 @@ int resident_pairs() {
   return clusters;
 }
 
-template <class C>
+// kSwiGLU: out_bf16 is unused (no output map); the fused outputs go through
+// args.q_codes / q_scales / g_out, which the caller fills in `extra`.
+template <class C, bool kSwiGLU = false>
 nvfp4_status launch_pair(const uint8_t* a_codes, const uint8_t* a_scales, const float* g_a, const uint8_t* w_codes,
                          const uint8_t* w_scales, const float* g_w, int64_t M, int64_t N, int64_t K, void* out_bf16,
-                         int64_t ldo, cudaStream_t stream) {
+                         int64_t ldo, cudaStream_t stream, const GemmArgs* extra = nullptr) {
   const int64_t tiles_m = (M + BM - 1) / BM, tiles_n = N / C::BN;
   const int64_t units = ((tiles_m + 1) / 2) * tiles_n;
   if (units >= (1ll << 31)) return NVFP4_ERR_SHAPE;
   CUtensorMap ma, mb, msa, msb, mo;
   if (!make_code_map(&ma, a_codes, M, K, BM) || !make_code_map(&mb, w_codes, N, K, 128) ||
-      !make_scale_map(&msa, a_scales, M, K) || !make_scale_map(&msb, w_scales, N, K) ||
-      !make_out_map(&mo, out_bf16, M, N, ldo))
+      !make_scale_map(&msa, a_scales, M, K) || !make_scale_map(&msb, w_scales, N, K))
     return NVFP4_ERR_CUDA;
-  const int pairs_max = resident_pairs<C>();
+  if (kSwiGLU) mo = ma;  // not read by the fused epilogue
+  else if (!make_out_map(&mo, out_bf16, M, N, ldo)) return NVFP4_ERR_CUDA;
+  const int pairs_max = resident_pairs<C, kSwiGLU>();
   if (pairs_max <= 0) return NVFP4_ERR_CUDA;
-  GemmArgs args;
+  GemmArgs args = {};
+  if (extra) args = *extra;
   args.sfa = a_scales;
   args.sfb = w_scales;
   args.ga = g_a;
@@ -936,7 +1016,7 @@ nvfp4_status launch_pair(const uint8_t* a_codes, const uint8_t* a_scales, const 
   cfg.stream = stream;
   cfg.attrs = attr;
   cfg.numAttrs = 2;
-  if (cudaLaunchKernelEx(&cfg, nvfp4_gemm_pair_kernel<C>, ma, mb, msa, msb, mo, args) != cudaSuccess)
+  if (cudaLaunchKernelEx(&cfg, nvfp4_gemm_pair_kernel<C, kSwiGLU>, ma, mb, msa, msb, mo, args) != cudaSuccess)
     return NVFP4_ERR_CUDA;
   count_launches(1);
   return launch_status();
@@ -986,4 +1066,58 @@ NVFP4_API nvfp4_status nvfp4_linear(const uint8_t* a_codes, const uint8_t* a_sca
   if (cm == 2) NVFP4_LAUNCH(128, 5, 2);
   NVFP4_LAUNCH(128, 5, 1);
 #undef NVFP4_LAUNCH
+}
+
+NVFP4_API nvfp4_status nvfp4_linear_swiglu_quantize(const uint8_t* a_codes, const uint8_t* a_scales, const float* g_a,
+                                                    const uint8_t* w_codes, const uint8_t* w_scales, const float* g_w,
+                                                    int64_t M, int64_t I, int64_t K, const float* g_out,
+                                                    uint8_t* out_codes, uint8_t* out_scales, void* stream) {
+  if (!a_codes || !a_scales || !g_a || !w_codes || !w_scales || !g_w || !g_out || !out_codes || !out_scales)
+    return NVFP4_ERR_INVALID_ARG;
+  if (M <= 0 || I <= 0 || K <= 0 || K % BK || I % 128) return NVFP4_ERR_SHAPE;
+  if (M >= (1ll << 31) || 2 * I >= (1ll << 31) || K >= (1ll << 31)) return NVFP4_ERR_SHAPE;
+  if (!aligned(a_codes, 16) || !aligned(w_codes, 16) || !aligned(a_scales, 16) || !aligned(w_scales, 16) ||
+      !aligned(out_codes, 16) || !aligned(out_scales, 4) || !aligned(g_a, 4) || !aligned(g_w, 4) || !aligned(g_out, 4))
+    return NVFP4_ERR_ALIGN;
+  GemmArgs extra = {};
+  extra.q_codes = out_codes;
+  extra.q_scales = out_scales;
+  extra.g_out = g_out;
+  return launch_pair<PairCfg<NVFP4_GEMM_PAIR_STAGES>, true>(a_codes, a_scales, g_a, w_codes, w_scales, g_w, M, 2 * I,
+                                                           K, nullptr, 0, static_cast<cudaStream_t>(stream), &extra);
+}
+
+namespace nvfp4 {
+namespace {
+// out row 32j + t = gate row 16j + t, out row 32j + 16 + t = up row 16j + t
+// (t < 16); one thread moves 16 bytes.
+__global__ void interleave_gate_up_kernel(const uint4* __restrict__ gate, const uint4* __restrict__ up,
+                                          uint4* __restrict__ out, uint64_t row_chunks, uint64_t n) {
+  griddep_wait_and_release();
+  for (uint64_t k = blockIdx.x * static_cast<uint64_t>(blockDim.x) + threadIdx.x; k < n;
+       k += static_cast<uint64_t>(gridDim.x) * blockDim.x) {
+    const uint64_t orow = k / row_chunks, c = k - orow * row_chunks;
+    const uint64_t j = orow >> 5, t = orow & 31u;
+    const uint64_t irow = 16 * j + (t & 15u);
+    out[k] = __ldg((t < 16 ? gate : up) + irow * row_chunks + c);
+  }
+}
+}  // namespace
+}  // namespace nvfp4
+
+NVFP4_API nvfp4_status nvfp4_interleave_gate_up(const void* w_gate, const void* w_up, int64_t I, int64_t row_bytes,
+                                                void* w_out, void* stream) {
+  if (!w_gate || !w_up || !w_out) return NVFP4_ERR_INVALID_ARG;
+  if (I <= 0 || I % 16 || row_bytes <= 0 || row_bytes % 16) return NVFP4_ERR_SHAPE;
+  if (!aligned(w_gate, 16) || !aligned(w_up, 16) || !aligned(w_out, 16)) return NVFP4_ERR_ALIGN;
+  const uint64_t row_chunks = static_cast<uint64_t>(row_bytes) / 16, n = 2 * static_cast<uint64_t>(I) * row_chunks;
+  uint64_t grid = (n + 255) / 256;
+  const uint64_t cap = static_cast<uint64_t>(sm_count()) * 8;
+  if (grid > cap) grid = cap;
+  if (launch_pdl(interleave_gate_up_kernel, dim3(static_cast<int>(grid)), dim3(256), 0,
+                 static_cast<cudaStream_t>(stream), static_cast<const uint4*>(w_gate), static_cast<const uint4*>(w_up),
+                 static_cast<uint4*>(w_out), row_chunks, n) != cudaSuccess)
+    return NVFP4_ERR_CUDA;
+  count_launches(1);
+  return launch_status();
 }

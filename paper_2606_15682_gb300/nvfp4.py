@@ -54,6 +54,8 @@ _quantize = _sig("nvfp4_quantize", [_p, _i64, _i64, _i64, _p, _p, _p, ctypes.c_i
 _quantize_dynamic = _sig("nvfp4_quantize_dynamic", [_p, _i64, _i64, _i64, _p, _p, _p, _p, ctypes.c_int, _p])
 _relayout = _sig("nvfp4_scales_relayout", [_p, _p, _i64, _i64, ctypes.c_int, ctypes.c_int, _p])
 _linear = _sig("nvfp4_linear", [_p, _p, _p, _p, _p, _p, _i64, _i64, _i64, _p, _i64, _p])
+_linear_swiglu = _sig("nvfp4_linear_swiglu_quantize", [_p, _p, _p, _p, _p, _p, _i64, _i64, _i64, _p, _p, _p, _p])
+_interleave = _sig("nvfp4_interleave_gate_up", [_p, _p, _i64, _i64, _p, _p])
 _kv_append = _sig("kv_append_nvfp4", [ctypes.POINTER(KVCacheStruct), _p, _p, _p, _p, _i64, _p, _p])
 _kv_append_rope = _sig("kv_append_rope_nvfp4",
                        [ctypes.POINTER(KVCacheStruct), _p, _p, _p, _p, _i64, _p, _i64, _p, _p])
@@ -133,6 +135,19 @@ def nvfp4_linear(a_codes, a_scales, g_a, w_codes, w_scales, g_w, out, M, N, K, l
                                    _ptr(g_w), M, N, K, _ptr(out), N if ldo is None else ldo, _stream(stream)))
 
 
+def nvfp4_linear_swiglu_quantize(a_codes, a_scales, g_a, w_codes, w_scales, g_w, M, I, K, g_out,
+                                 out_codes, out_scales, stream=None):
+    _check("nvfp4_linear_swiglu_quantize",
+           _linear_swiglu(_ptr(a_codes), _ptr(a_scales), _ptr(g_a), _ptr(w_codes), _ptr(w_scales), _ptr(g_w),
+                          M, I, K, _ptr(g_out), _ptr(out_codes), _ptr(out_scales), _stream(stream)))
+
+
+def nvfp4_interleave_gate_up(w_gate, w_up, w_out, stream=None):
+    _check("nvfp4_interleave_gate_up",
+           _interleave(_ptr(w_gate), _ptr(w_up), w_gate.shape[0], w_gate.shape[1] * w_gate.element_size(),
+                       _ptr(w_out), _stream(stream)))
+
+
 def kv_append_nvfp4(cache, k, v, seq_idx, pos, k_shift=None, stream=None):
     s = cache.struct()
     _check("kv_append_nvfp4", _kv_append(ctypes.byref(s), _ptr(k), _ptr(v), _ptr(seq_idx), _ptr(pos), k.shape[0],
@@ -209,6 +224,7 @@ class KVCache:
 
 
 EXPORTED = ["nvfp4_scales_bytes", "nvfp4_tensor_scale", "nvfp4_quantize", "nvfp4_quantize_dynamic", "nvfp4_scales_relayout", "nvfp4_linear",
+            "nvfp4_linear_swiglu_quantize", "nvfp4_interleave_gate_up",
             "kv_append_nvfp4", "kv_append_rope_nvfp4", "nvfp4_rope_table", "decode_attention_nvfp4_workspace_size", "decode_attention_nvfp4",
             "decode_attention_nvfp4_static_scratch",
             "nvfp4_get_device_status", "nvfp4_status_string", "nvfp4_launch_count"]

@@ -53,6 +53,13 @@ def test_argument_validation_before_launch():
     assert L.nvfp4_linear(odd, p, p, p, p, p, 128, 128, 256, p, 128, s) == 3
     assert L.nvfp4_quantize(odd, 4, 64, 64, p, p, p, 1, s) == 3
     assert L.nvfp4_quantize(p, 4, 64, 68, p, p, p, 1, s) == 3            # ld % 8
+    # fused gate_up + SwiGLU + quantize: I % 128, K % 256, null g_out
+    assert L.nvfp4_linear_swiglu_quantize(p, p, p, p, p, p, 256, 192, 512, p, p, p, s) == 2
+    assert L.nvfp4_linear_swiglu_quantize(p, p, p, p, p, p, 256, 256, 384, p, p, p, s) == 2
+    assert L.nvfp4_linear_swiglu_quantize(p, p, p, p, p, p, 256, 256, 512, None, p, p, s) == 1
+    assert L.nvfp4_linear_swiglu_quantize(p, p, p, p, p, p, 256, 256, 512, p, odd, p, s) == 3
+    assert L.nvfp4_interleave_gate_up(p, p, 24, 64, p, s) == 2                # I % 16
+    assert L.nvfp4_interleave_gate_up(p, p, 32, 40, p, s) == 2                # row bytes % 16
     st = ctypes.c_void_p(0x20000)
     assert L.nvfp4_quantize_dynamic(p, 4, 64, 64, None, p, p, p, 1, s) == 1   # no state
     assert L.nvfp4_quantize_dynamic(p, 4, 64, 64, st, None, p, p, 1, s) == 1  # no g

@@ -136,3 +136,86 @@ def test_workload_linears(N, workload):
         got = f32(out[torch.as_tensor(rows, device="cuda")][:, torch.as_tensor(cols, device="cuda")])
         report.append((name,) + assert_close(got, ref, what=f"{workload}/{name}"))
     print(workload, report)
+
+
+# ------------------------------------ gate_up with SwiGLU + quantize fused ---
+
+def test_interleave_gate_up_matches_oracle(N):
+    gen = torch.Generator().manual_seed(12)
+    I, K = 96, 200
+    g = torch.randn(I, K, generator=gen).to(torch.bfloat16)
+    u = torch.randn(I, K, generator=gen).to(torch.bfloat16)
+    out = torch.empty(2 * I, K, dtype=torch.bfloat16, device="cuda")
+    N.nvfp4_interleave_gate_up(g.cuda(), u.cuda(), out)
+    torch.cuda.synchronize()
+    ref = O.interleave_gate_up(g.view(torch.int16).numpy(), u.view(torch.int16).numpy())
+    assert np.array_equal(out.cpu().view(torch.int16).numpy(), ref)
+
+
+def swiglu_case(N, M, I, K, seed, rows=None):
+    gen = torch.Generator().manual_seed(seed)
+    a_c, a_s = random_operand(M, K, gen)
+    wg_c, wg_s = random_operand(I, K, gen, 0x30, 0x40)
+    wu_c, wu_s = random_operand(I, K, gen, 0x30, 0x40)
+    g_a, g_w = np.float32(0.0173), np.float32(0.0021)
+    rows = np.arange(M) if rows is None else rows
+    G = O.linear_rows(a_c, a_s, g_a, wg_c, wg_s, g_w, rows)
+    U = O.linear_rows(a_c, a_s, g_a, wu_c, wu_s, g_w, rows)
+    h = O.silu(G) * U
+    g_out = O.tensor_scale(h.astype(np.float32))            # a calibrated static scale
+    w_c = O.interleave_gate_up(wg_c, wu_c)
+    w_s = O.interleave_gate_up(wg_s, wu_s)
+    dev = "cuda"
+    out_c = torch.full((M, I // 2), 0xEE, dtype=torch.uint8, device=dev)
+    out_s = torch.full((N.nvfp4_scales_bytes(M, I, 1),), 0xEE, dtype=torch.uint8, device=dev)
+    N.nvfp4_linear_swiglu_quantize(torch.from_numpy(a_c).to(dev), torch.from_numpy(O.scales_to_mma(a_s)).to(dev),
+                                   torch.tensor([g_a], device=dev), torch.from_numpy(w_c).to(dev),
+                                   torch.from_numpy(O.scales_to_mma(w_s)).to(dev), torch.tensor([g_w], device=dev),
+                                   M, I, K, torch.tensor([g_out], device=dev), out_c, out_s)
+    torch.cuda.synchronize()
+    assert N.nvfp4_get_device_status() == 0
+    return h, g_out, rows, u8(out_c), u8(out_s)
+
+
+@pytest.mark.parametrize("M,I,K", [(256, 128, 256), (129, 384, 512), (300, 256, 1024), (640, 512, 768)])
+def test_linear_swiglu_quantize(N, M, I, K):
+    """h = SiLU(gate) * up from the fp32 accumulators, quantized with a static scale:
+    scales within one E4M3 step of the oracle's, elements within the quantization
+    error bound of the fp64 h, almost all codes identical, padding scales zero."""
+    h, g_out, rows, out_c, out_s = swiglu_case(N, M, I, K, seed=M + I + K)
+    rc, rs = O.quantize(h.astype(np.float32), g_out)
+    gs = O.scales_from_mma(out_s, M, I)
+    assert np.abs(gs.astype(int) - rs.astype(int)).max() <= 1
+    assert (gs == rs).mean() > 0.99
+    assert (out_c == rc).mean() > 0.99
+    deq = O.dequantize(out_c, gs, g_out)
+    S = O.e4m3_decode(gs).repeat(16, axis=1)
+    assert np.all(np.abs(deq - h) <= 1.5 * S * np.float64(g_out) + 1e-6 * np.abs(h))
+    pad = np.setdiff1d(np.arange(O.mma_scale_bytes(M, I)), O._mma_offsets(M, I // 16).ravel())
+    assert not out_s[pad].any(), "padding rows of the output scales must be zero"
+
+
+def test_linear_swiglu_quantize_prefill_shape_then_down(N):
+    """The 1.5B-prefill MLP shape (M=2048, I=8960, K=1536) checked on sampled rows,
+    then fed to the down projection as its A operand."""
+    M, I, K, Hd = 2048, 8960, 1536, 1536
+    rows = np.sort(np.r_[np.random.default_rng(2).choice(M, 48, replace=False), M - 1])
+    h, g_out, rows, out_c, out_s = swiglu_case(N, M, I, K, seed=99, rows=rows)
+    gs = O.scales_from_mma(out_s, M, I)[rows]
+    rc, rs = O.quantize(h.astype(np.float32), g_out)
+    assert np.abs(gs.astype(int) - rs.astype(int)).max() <= 1 and (out_c[rows] == rc).mean() > 0.99
+    deq = O.dequantize(out_c[rows], gs, g_out)
+    S = O.e4m3_decode(gs).repeat(16, axis=1)
+    assert np.all(np.abs(deq - h) <= 1.5 * S * np.float64(g_out) + 1e-6 * np.abs(h))
+    # down projection straight from the fused output
+    gen = torch.Generator().manual_seed(7)
+    wd_c, wd_s = random_operand(Hd, I, gen)
+    g_wd = np.float32(0.003)
+    out = torch.empty(M, Hd, dtype=torch.bfloat16, device="cuda")
+    N.nvfp4_linear(torch.from_numpy(out_c).cuda(), torch.from_numpy(out_s).cuda(),
+                   torch.tensor([g_out], device="cuda"), torch.from_numpy(wd_c).cuda(),
+                   torch.from_numpy(O.scales_to_mma(wd_s)).cuda(), torch.tensor([g_wd], device="cuda"), out, M, Hd, I)
+    torch.cuda.synchronize()
+    assert N.nvfp4_get_device_status() == 0
+    ref = O.linear_rows(out_c, O.scales_from_mma(out_s, M, I), g_out, wd_c, wd_s, g_wd, rows)
+    assert_close(f32(out[torch.as_tensor(rows, device="cuda")]), ref, what="down(swiglu)")
