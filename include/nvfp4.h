@@ -174,9 +174,9 @@ nvfp4_status nvfp4_linear(const uint8_t* a_codes, const uint8_t* a_scales, const
  *   out_codes         : [M, I/2] bytes, 16-B aligned.
  *   out_scales        : nvfp4_scales_bytes(M, I, NVFP4_SCALES_MMA) bytes, 4-B
  *                       aligned; padding rows are written as zeros.
- * SiLU uses the fast exponential (__expf): h may differ from an exact SiLU by
- * a few fp32 ulps, which can change a code only where h sits on a rounding
- * boundary.  I % 128 == 0, K % 256 == 0, M, I, K > 0 (SHAPE).  g_out <= 0 or
+ * SiLU is evaluated as x/2 (1 + tanh(x/2)) with the hardware tanh
+ * approximation (relative error ~2^-11): h may differ from an exact SiLU by
+ * that much, which changes a code only where h sits near a rounding boundary.  I % 128 == 0, K % 256 == 0, M, I, K > 0 (SHAPE).  g_out <= 0 or
  * non-finite: zero codes and scales, INVALID_ARG set on the device.
  */
 nvfp4_status nvfp4_linear_swiglu_quantize(const uint8_t* a_codes, const uint8_t* a_scales, const float* g_a,

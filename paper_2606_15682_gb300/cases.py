@@ -4,6 +4,7 @@
     python -m paper_2606_15682_gb300.cases quantize --workload qwen1.5b_prefill_linears_m2048 --linear down
     python -m paper_2606_15682_gb300.cases quantize_dynamic --workload qwen32b_prefill_linears_m8192 --linear down
     python -m paper_2606_15682_gb300.cases attention --batch 64 --context 16384
+    python -m paper_2606_15682_gb300.cases gemm_swiglu --workload qwen32b_prefill_linears_m8192
 
 Inputs are seeded synthetic tensors (paper_2606_15682_gb300.synth); for the
 attention case the cache is filled with seeded random codes and scales
@@ -47,7 +48,8 @@ def _time(fn, iters):
 
 def main():
     ap = argparse.ArgumentParser()
-    ap.add_argument("kernel", choices=["gemm", "quantize", "quantize_dynamic", "tensor_scale", "attention"])
+    ap.add_argument("kernel", choices=["gemm", "gemm_swiglu", "quantize", "quantize_dynamic", "tensor_scale",
+                                       "attention"])
     ap.add_argument("--workload", default="qwen1.5b_prefill_linears_m2048")
     ap.add_argument("--linear", default="gate_up")
     ap.add_argument("--batch", type=int, default=64)
@@ -56,7 +58,36 @@ def main():
     a = ap.parse_args()
     dev = torch.device("cuda", 0)
     torch.cuda.set_device(dev)
-    if a.kernel in ("gemm", "quantize", "quantize_dynamic", "tensor_scale"):
+    if a.kernel == "gemm_swiglu":
+        # gate_up of the workload with SwiGLU + NVFP4 quantization of the down
+        # projection's input in the epilogue, against the same GEMM with bf16
+        # output followed by the one-launch quantizer on an [M, I] tensor.
+        x, W = synth.linear_inputs(a.workload, "gate_up", device=dev)
+        M, K = x.shape
+        I = W.shape[0] // 2
+        Wi = torch.empty_like(W)
+        N.nvfp4_interleave_gate_up(W[:I].contiguous(), W[I:].contiguous(), Wi)
+        del W
+        ac, asf, ga = _quantized(x)
+        wc, wsf, gw = _quantized(Wi)
+        del Wi
+        g_out = torch.tensor([0.05], dtype=torch.float32, device=dev)
+        qc = torch.empty(M, I // 2, dtype=torch.uint8, device=dev)
+        qs = torch.empty(N.nvfp4_scales_bytes(M, I, N.SCALES_MMA), dtype=torch.uint8, device=dev)
+        ms_f = _time(lambda: N.nvfp4_linear_swiglu_quantize(ac, asf, ga, wc, wsf, gw, M, I, K, g_out, qc, qs), a.iters)
+        out = torch.empty(M, 2 * I, dtype=torch.bfloat16, device=dev)
+        h = out[:, :I].contiguous()
+        st = torch.zeros(N.DYNAMIC_STATE_BYTES, dtype=torch.uint8, device=dev)
+        g_h = torch.empty(1, dtype=torch.float32, device=dev)
+
+        def unfused():
+            N.nvfp4_linear(ac, asf, ga, wc, wsf, gw, out, M, 2 * I, K)
+            N.nvfp4_quantize_dynamic(h, st, g_h, qc, qs, N.SCALES_MMA)
+        ms_u = _time(unfused, a.iters)
+        print(f"gemm_swiglu {a.workload} {M}x{2 * I}x{K}: fused {ms_f * 1e3:.1f} us "
+              f"({2 * M * 2 * I * K / ms_f / 1e9:.1f} TFLOP/s); bf16 GEMM + quantize of h {ms_u * 1e3:.1f} us "
+              f"(SwiGLU itself not included)")
+    elif a.kernel in ("gemm", "quantize", "quantize_dynamic", "tensor_scale"):
         x, W = synth.linear_inputs(a.workload, a.linear, device=dev)
         M, K = x.shape
         Nn = W.shape[0]
