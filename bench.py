@@ -240,12 +240,32 @@ def run_ours(args, rank, world):
     h2d = sum(t.numel() * t.element_size() for t in host_a)
     d2h = sum(t.numel() * t.element_size() for t in host_o)
 
+    # Copies run on their own streams so each layer's H2D, compute and D2H
+    # overlap the others' (the two copy directions also run concurrently).
+    s_in, s_out = torch.cuda.Stream(device=dev), torch.cuda.Stream(device=dev)
+    ev_fork = torch.cuda.Event()
+    ev_in = [torch.cuda.Event() for _ in layers]
+    ev_c = [torch.cuda.Event() for _ in layers]
+    ev_join = torch.cuda.Event()
+
     def e2e_step():
-        for L, ha in zip(layers, host_a):
-            L["a"].copy_(ha, non_blocking=True)
-        gemm_step(False)
-        for L, ho in zip(layers, host_o):
-            ho.copy_(L["out"], non_blocking=True)
+        ev_fork.record(stream)
+        s_in.wait_event(ev_fork)
+        s_out.wait_event(ev_fork)
+        with torch.cuda.stream(s_in):
+            for L, ha, e in zip(layers, host_a, ev_in):
+                L["a"].copy_(ha, non_blocking=True)
+                e.record(s_in)
+        for L, ho, ei, ec in zip(layers, host_o, ev_in, ev_c):
+            stream.wait_event(ei)
+            N.nvfp4_quantize_dynamic(L["a"], L["qstate"], L["ga"], L["ac"], L["asf"], N.SCALES_MMA)
+            N.nvfp4_linear(L["ac"], L["asf"], L["ga"], L["wc"], L["ws"], L["gw"], L["out"], M, L["N"], L["K"])
+            ec.record(stream)
+            s_out.wait_event(ec)
+            with torch.cuda.stream(s_out):
+                ho.copy_(L["out"], non_blocking=True)
+        ev_join.record(s_out)
+        stream.wait_event(ev_join)
 
     e2e_ms = timed_loop(e2e_step, max(3, min(args.steps, 50)), args.warmup)
 
