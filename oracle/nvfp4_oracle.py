@@ -23,7 +23,8 @@ readability, not speed:
 * the fused step RoPE -> shift -> quantize -> append, with RoPE in fp32 from a
   (cos, sin) table in a fixed order of operations (``rope_f32``);
 * the gate_up projection with the SwiGLU product and the NVFP4 quantization of
-  the down projection's input fused behind it (``linear_swiglu_quantize``).
+  the down projection's input fused behind it (``linear_swiglu_quantize``);
+* the E1M2 element grid for the KV cache (``e1m2_*``, ``element="e1m2"``).
 
 Floating-point conventions: the quantizer's arithmetic is IEEE fp32 with
 round-to-nearest-even (numpy float32 scalars/arrays, no fused multiply-add);
@@ -145,6 +146,38 @@ def _e4m3_code_of_value(val):
 # NVFP4 tensor quantization.
 # ---------------------------------------------------------------------------
 
+# ---------------------------------------------------------------------------
+# E1M2 elements: the 4-bit KV-cache element of the paper's QAT runs (the
+# Q-FIT section uses E1M2 for the KV cache; the paper names the format but not
+# its bias).  Reading: 1 sign bit, 1 exponent bit with bias 0, 2 mantissa
+# bits, so  e == 0: m/2 (subnormal), e == 1: 2 + m/2  -- the uniform grid
+# 0, 0.5, ..., 3.5.  A magnitude is then k/2 with k = 0..7.
+# Storage in this library's KV cache: the two's-complement nibble of
+# n = sign * k (n in -7..7; the pattern of -8 is never written).
+# ---------------------------------------------------------------------------
+
+E1M2_MAX = 3.5
+
+
+def e1m2_decode(nib):
+    """Value of stored E1M2 nibbles (array of ints 0..15): n/2, n = nib as a
+    4-bit two's-complement integer."""
+    nib = np.asarray(nib, dtype=np.int64)
+    n = np.where(nib >= 8, nib - 16, nib)
+    return n.astype(np.float64) / 2.0
+
+
+def e1m2_encode(v):
+    """Round values onto E1M2: k = RNE(2|v|) (ties to even k, i.e. to an even
+    mantissa), saturated at 7 (3.5); stored as the nibble of sign * k.  A
+    negative value that rounds to zero is stored as 0 (one zero in two's
+    complement)."""
+    v = np.asarray(v, dtype=np.float64)
+    k = np.minimum(np.rint(np.abs(v) * 2.0), 7).astype(np.int64)
+    n = np.where(np.signbit(v), -k, k)
+    return (n & 0xF).astype(np.uint8)
+
+
 BLOCK = 16                    # elements per E4M3 block scale (Appendix A)
 TENSOR_SCALE_DIV = np.float32(6.0 * 448.0)   # largest E2M1 magnitude x largest E4M3 scale
 
@@ -168,8 +201,10 @@ def tensor_scale(x_f32):
     return np.float32(amax / TENSOR_SCALE_DIV)
 
 
-def quantize(x_f32, g):
+def quantize(x_f32, g, element="e2m1"):
     """NVFP4-quantize a [rows, cols] tensor along its rows (cols % 16 == 0).
+    element="e1m2" swaps the element grid for the E1M2 KV variant (step 2
+    then divides by 3.5 g instead of 6 g and step 4 rounds onto E1M2).
 
     Reading of the format (the paper gives the format, not the recipe), per
     block b of 16 consecutive elements of a row, all fp32 RNE:
@@ -191,7 +226,8 @@ def quantize(x_f32, g):
         raise ValueError("tensor scale must be positive and finite")
     xb = x.reshape(rows, cols // BLOCK, BLOCK)
     amax = np.max(np.abs(xb), axis=2)                               # exact
-    six_g = np.float32(np.float32(6.0) * g)
+    qmax = np.float32(6.0) if element == "e2m1" else np.float32(E1M2_MAX)
+    six_g = np.float32(qmax * g)
     with np.errstate(over="ignore", divide="ignore"):
         s_f = (amax / six_g).astype(np.float32)
     S = e4m3_encode_nonneg(s_f)                                      # uint8 [rows, cols/16]
@@ -202,7 +238,7 @@ def quantize(x_f32, g):
         r = np.where(zero_scale, np.float32(0.0), np.float32(1.0) / np.where(zero_scale, np.float32(1.0), d))
     r = r.astype(np.float32)
     v = (xb * r[:, :, None]).astype(np.float32)                     # zero scale -> signed zeros
-    codes = e2m1_encode(v).reshape(rows, cols)
+    codes = (e2m1_encode(v) if element == "e2m1" else e1m2_encode(v)).reshape(rows, cols)
     packed = (codes[:, 0::2] | (codes[:, 1::2] << 4)).astype(np.uint8)
     return packed, S
 
@@ -216,10 +252,10 @@ def unpack_codes(packed):
     return out
 
 
-def dequantize(packed, scales, g):
-    """x_hat = e2m1(code) * e4m3(S) * g, evaluated in fp64 (exact)."""
+def dequantize(packed, scales, g, element="e2m1"):
+    """x_hat = e2m1(code) * e4m3(S) * g (or e1m2(code) ...), evaluated in fp64 (exact)."""
     codes = unpack_codes(packed)
-    vals = e2m1_decode(codes)
+    vals = e2m1_decode(codes) if element == "e2m1" else e1m2_decode(codes)
     rows, cols = codes.shape[-2], codes.shape[-1]
     s = e4m3_decode(scales).astype(np.float64)
     s = np.repeat(s, BLOCK, axis=-1)
@@ -327,7 +363,8 @@ def linear_rows(a_codes, a_scales, g_a, w_codes, w_scales, g_w, rows):
 # ---------------------------------------------------------------------------
 
 
-def kv_append(k_codes, k_scales, v_codes, v_scales, k_new, v_new, seq_idx, pos, g_k, g_v, k_shift=None):
+def kv_append(k_codes, k_scales, v_codes, v_scales, k_new, v_new, seq_idx, pos, g_k, g_v, k_shift=None,
+              element="e2m1"):
     """Quantize and store new K/V rows in place.
 
     k_new, v_new: float32 [n_new, kv_heads, head_dim] (bf16 values, post-RoPE K).
@@ -339,8 +376,8 @@ def kv_append(k_codes, k_scales, v_codes, v_scales, k_new, v_new, seq_idx, pos, 
     n_new, hkv, d = k.shape
     if k_shift is not None:
         k = (k - np.asarray(k_shift, dtype=np.float32)[None, :, :]).astype(np.float32)
-    kc, ks = quantize(k.reshape(n_new * hkv, d), g_k)
-    vc, vs = quantize(v.reshape(n_new * hkv, d), g_v)
+    kc, ks = quantize(k.reshape(n_new * hkv, d), g_k, element)
+    vc, vs = quantize(v.reshape(n_new * hkv, d), g_v, element)
     kc = kc.reshape(n_new, hkv, d // 2); ks = ks.reshape(n_new, hkv, d // BLOCK)
     vc = vc.reshape(n_new, hkv, d // 2); vs = vs.reshape(n_new, hkv, d // BLOCK)
     for i in range(n_new):
@@ -350,7 +387,7 @@ def kv_append(k_codes, k_scales, v_codes, v_scales, k_new, v_new, seq_idx, pos, 
 
 
 def decode_attention(q_f32, k_codes, k_scales, v_codes, v_scales, seq_lens, g_k, g_v, softmax_scale,
-                     batches=None, heads=None):
+                     batches=None, heads=None, element="e2m1"):
     """fp64 decode attention over the NVFP4 cache (Sec. 2.1).
 
     For query head h of sequence b, with KV head kv = h // (H_q / H_kv)
@@ -379,8 +416,8 @@ def decode_attention(q_f32, k_codes, k_scales, v_codes, v_scales, seq_lens, g_k,
         for j, h in enumerate(heads):
             kv = h // group
             if kv not in cache:
-                cache[kv] = (dequantize(k_codes[b, kv, :T], k_scales[b, kv, :T], g_k),
-                             dequantize(v_codes[b, kv, :T], v_scales[b, kv, :T], g_v))
+                cache[kv] = (dequantize(k_codes[b, kv, :T], k_scales[b, kv, :T], g_k, element),
+                             dequantize(v_codes[b, kv, :T], v_scales[b, kv, :T], g_v, element))
             K, V = cache[kv]
             out[i, j] = attention_fp64(q[b, h], K, V, scale)
     return out
@@ -442,13 +479,13 @@ def rope_f32(x_f32, positions, table):
 
 
 def kv_append_rope(k_codes, k_scales, v_codes, v_scales, k_pre, v_new, seq_idx, pos, g_k, g_v, table,
-                   k_shift=None):
+                   k_shift=None, element="e2m1"):
     """The fused step before decode attention: K~ = RoPE(K_pre) - m (Eq. 2 with
     the pre-RoPE scaling s folded into the key projection), then quantize and
     store K~ and V as ``kv_append`` does.  k_pre: float32 [n_new, kv_heads, d]
     (bf16 values, before RoPE); RoPE and the shift in fp32 (``rope_f32``)."""
     k = rope_f32(k_pre, pos, table)
-    kv_append(k_codes, k_scales, v_codes, v_scales, k, v_new, seq_idx, pos, g_k, g_v, k_shift)
+    kv_append(k_codes, k_scales, v_codes, v_scales, k, v_new, seq_idx, pos, g_k, g_v, k_shift, element)
 
 
 def qfit_transform(q_pre, k_pre, s, m, positions, theta=1.0e6):

@@ -445,3 +445,42 @@ def test_linear_swiglu_quantize_brute_force():
             assert np.isclose(h[m, i], gs / (1 + np.exp(-gs)) * us, rtol=1e-12, atol=1e-12)
     rc, rs = O.quantize(h.astype(np.float32), np.float32(0.01))
     assert np.array_equal(codes, rc) and np.array_equal(scales, rs)
+
+
+# ------------------------------------------------------- E1M2 KV elements ---
+
+def test_e1m2_decode_exhaustive_table():
+    # two's-complement nibbles 0..7 -> 0..3.5, 8 -> -4 (never written), 9..15 -> -3.5..-0.5
+    want = [0, .5, 1, 1.5, 2, 2.5, 3, 3.5, -4, -3.5, -3, -2.5, -2, -1.5, -1, -.5]
+    assert np.array_equal(O.e1m2_decode(np.arange(16)), np.array(want))
+
+
+def test_e1m2_grid_is_the_bias0_minifloat():
+    # 1 exponent bit (bias 0), 2 mantissa bits: e=0 -> m/2, e=1 -> 2 + m/2
+    mags = [(m / 2.0 if e == 0 else 2.0 + m / 2.0) for e in (0, 1) for m in range(4)]
+    assert np.array_equal(np.sort(np.unique(np.abs(O.e1m2_decode(np.arange(16)))))[:8], np.array(mags))
+
+
+def test_e1m2_encode_ties_saturation_and_roundtrip():
+    # ties of 2|v| go to the even integer; beyond 3.5 saturates
+    v = np.array([0.25, 0.75, 1.25, 1.75, 2.25, 3.25, 3.75, 100.0, -0.25, -0.75, -1e-9, 0.0])
+    got = O.e1m2_decode(O.e1m2_encode(v))
+    assert np.array_equal(got, [0.0, 1.0, 1.0, 2.0, 2.0, 3.0, 3.5, 3.5, 0.0, -1.0, 0.0, 0.0])
+    codes = np.array([c for c in range(16) if c != 8])
+    assert np.array_equal(O.e1m2_encode(O.e1m2_decode(codes)), codes.astype(np.uint8))
+
+
+def test_e1m2_quantize_scale_closed_form_and_error_bound():
+    rng = np.random.default_rng(14)
+    x = (rng.standard_normal((40, 64)) * np.exp2(rng.integers(-4, 4, (40, 1)))).astype(np.float32)
+    g = np.float32(np.abs(x).max() / (3.5 * 448))
+    codes, S = O.quantize(x, g, "e1m2")
+    blocks = np.abs(x).reshape(40, 4, 16).max(axis=2)
+    # the block scale is the E4M3 rounding of amax / (3.5 g)
+    want = O.e4m3_encode_nonneg((blocks / np.float32(np.float32(3.5) * g)).astype(np.float32))
+    assert np.array_equal(S, want)
+    xh = O.dequantize(codes, S, g, "e1m2")
+    Sv = np.repeat(O.e4m3_decode(S), 16, axis=1) * np.float64(g)
+    # uniform grid with step 0.5: error <= 0.25 scale units inside the range, plus E4M3's
+    # rounding of the scale below amax (at most 1/16 of 3.5 units) at the block maximum
+    assert np.all(np.abs(xh - x) <= (0.25 + 3.5 / 16) * Sv + 1e-12)
