@@ -193,6 +193,19 @@ nvfp4_status nvfp4_linear_swiglu_quantize(const uint8_t* a_codes, const uint8_t*
 nvfp4_status nvfp4_interleave_gate_up(const void* w_gate, const void* w_up, int64_t I, int64_t row_bytes,
                                       void* w_out, void* stream);
 
+/* Element grid of the KV cache (the block scales are E4M3 per 16 either way). */
+typedef enum {
+  /* E2M1, the NVFP4 element {0, 0.5, 1, 1.5, 2, 3, 4, 6} (the B200 deployment's
+   * native 4-bit KV cache, Appendix D.3).  Nibble = sign | E2M1 magnitude.  */
+  NVFP4_KV_E2M1 = 0,
+  /* E1M2, the KV element of the paper's QAT runs (Q-FIT section): read as the
+   * bias-0 grid {0, 0.5, ..., 3.5}; block scale E4M3(amax / (3.5 g)), element
+   * RNE(2|v|) saturated at 7, stored as the two's-complement nibble of
+   * sign * k.  Decode attention reads it through integer tricks (no hardware
+   * conversion), so it is slower than E2M1.                                 */
+  NVFP4_KV_E1M2 = 1
+} nvfp4_kv_format;
+
 /*
  * NVFP4 KV cache (W4A4KV4; the B200 deployment uses a native 4-bit KV cache,
  * Appendix D.3).  One row per (sequence, KV head, position); the 16-element
@@ -203,7 +216,10 @@ nvfp4_status nvfp4_interleave_gate_up(const void* w_gate, const void* w_up, int6
  *                        (maintained by the caller; read by attention).
  *   k_gscale, v_gscale : static per-layer FP32 tensor scales (an append-only
  *                        cache cannot re-scale rows it already holds).
- * head_dim must be 128.  Buffers 16-B aligned.
+ *   kv_format          : nvfp4_kv_format of both K and V (0 = E2M1 when a
+ *                        caller zero-initializes the struct).
+ * head_dim must be 128.  Buffers 16-B aligned.  A kv_format other than the
+ * enum's values -> INVALID_ARG in every call that takes the cache.
  */
 typedef struct {
   uint8_t* k_codes;
@@ -217,6 +233,7 @@ typedef struct {
   int32_t capacity;
   float k_gscale;
   float v_gscale;
+  int32_t kv_format;
 } nvfp4_kv_cache;
 
 /*

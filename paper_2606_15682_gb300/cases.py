@@ -55,6 +55,7 @@ def main():
     ap.add_argument("--batch", type=int, default=64)
     ap.add_argument("--context", type=int, default=16384)
     ap.add_argument("--iters", type=int, default=3)
+    ap.add_argument("--kv-format", choices=["e2m1", "e1m2"], default="e2m1")
     a = ap.parse_args()
     dev = torch.device("cuda", 0)
     torch.cuda.set_device(dev)
@@ -119,7 +120,8 @@ def main():
         B, hq, hkv, T = a.batch, 40, 8, a.context
         gen = torch.Generator(device=dev)
         gen.manual_seed(5)
-        cache = N.KVCache(B, hkv, T, 0.01, 0.01, device=dev)
+        cache = N.KVCache(B, hkv, T, 0.01, 0.01, device=dev,
+                          kv_format=N.KV_E1M2 if a.kv_format == "e1m2" else N.KV_E2M1)
         for t in (cache.k_codes, cache.v_codes):
             t.copy_(torch.randint(0, 256, t.shape, generator=gen, device=dev, dtype=torch.int32).to(torch.uint8))
         for t in (cache.k_scales, cache.v_scales):
@@ -130,7 +132,7 @@ def main():
         out = torch.empty(B, hq, 128, dtype=torch.bfloat16, device=dev)
         ms = _time(lambda: N.decode_attention_nvfp4(cache, q, 1 / math.sqrt(128), out, ws), a.iters)
         byt = B * hkv * T * 144
-        print(f"attention B={B} T={T}: {ms * 1e3:.1f} us, {byt / ms / 1e6:.0f} GB/s (K/V codes+scales)")
+        print(f"attention {a.kv_format} B={B} T={T}: {ms * 1e3:.1f} us, {byt / ms / 1e6:.0f} GB/s (K/V codes+scales)")
     assert N.nvfp4_get_device_status() == 0
 
 

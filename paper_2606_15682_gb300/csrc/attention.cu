@@ -71,6 +71,28 @@ __device__ __forceinline__ void e2m1x8_to_f16x2(uint32_t w, uint32_t h[4]) {
       : "r"(w));
 }
 
+// Four bytes of E1M2 nibbles (two's complement n, value n/2) -> four f16x2
+// holding n (low nibble -> low half); the 1/2 goes into the block scale.  The
+// nibble XOR 8 in the low mantissa bits of 1024.0 (0x6400) reads as 1032 + n.
+__device__ __forceinline__ uint32_t hsub2(uint32_t a, uint32_t b) {
+  uint32_t d;
+  asm("sub.rn.f16x2 %0, %1, %2;" : "=r"(d) : "r"(a), "r"(b));
+  return d;
+}
+__device__ __forceinline__ void e1m2x8_to_f16x2(uint32_t w, uint32_t h[4]) {
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    const uint32_t x = w >> (8 * j);
+    h[j] = hsub2(((x & 0xFu) | ((x & 0xF0u) << 12)) ^ 0x64086408u, 0x64086408u);
+  }
+}
+
+template <bool kE1M2>
+__device__ __forceinline__ void decode8(uint32_t w, uint32_t h[4]) {
+  if (kE1M2) e1m2x8_to_f16x2(w, h);
+  else e2m1x8_to_f16x2(w, h);
+}
+
 // Two E4M3 bytes (low byte -> low half) -> f16x2, exact.
 __device__ __forceinline__ uint32_t e4m3x2_to_f16x2(uint32_t two_bytes) {
   uint32_t h;
@@ -144,6 +166,8 @@ struct Params {
   float logit_mult;  // softmax_scale * g_K * log2(e)
 };
 
+// kE1M2: the cache holds E1M2 elements (decoded to n, the scale carries 1/2).
+template <bool kE1M2>
 __global__ void __launch_bounds__(kThreads, NVFP4_ATTN_MIN_CTAS) attn_partial_kernel(const Params p) {
   extern __shared__ __align__(128) uint8_t smem[];
   uint8_t* ring = smem;
@@ -275,8 +299,9 @@ __global__ void __launch_bounds__(kThreads, NVFP4_ATTN_MIN_CTAS) attn_partial_ke
         // ---- S^T = K_hat Q^T: 8 k-steps of 16 channels ---------------------
         const uint4 ka = *reinterpret_cast<const uint4*>(st + kOffKc + (r0 + rk0) * 64 + 16 * t);
         const uint4 kb = *reinterpret_cast<const uint4*>(st + kOffKc + (r0 + rk1) * 64 + 16 * t);
-        const uint32_t ksa = e4m3x2_to_f16x2(*reinterpret_cast<const uint16_t*>(st + kOffKs + (r0 + rk0) * 8 + 2 * t));
-        const uint32_t ksb = e4m3x2_to_f16x2(*reinterpret_cast<const uint16_t*>(st + kOffKs + (r0 + rk1) * 8 + 2 * t));
+        uint32_t ksa = e4m3x2_to_f16x2(*reinterpret_cast<const uint16_t*>(st + kOffKs + (r0 + rk0) * 8 + 2 * t));
+        uint32_t ksb = e4m3x2_to_f16x2(*reinterpret_cast<const uint16_t*>(st + kOffKs + (r0 + rk1) * 8 + 2 * t));
+        if (kE1M2) { ksa = hmul2(ksa, 0x38003800u); ksb = hmul2(ksb, 0x38003800u); }  // times 1/2, exact
         const uint32_t sa_lo = bcast_lo(ksa), sa_hi = bcast_hi(ksa);
         const uint32_t sb_lo = bcast_lo(ksb), sb_hi = bcast_hi(ksb);
         float s[4] = {0.0f, 0.0f, 0.0f, 0.0f};
@@ -285,8 +310,8 @@ __global__ void __launch_bounds__(kThreads, NVFP4_ATTN_MIN_CTAS) attn_partial_ke
 #pragma unroll
         for (int w = 0; w < 4; ++w) {
           uint32_t ha[4], hb[4];
-          e2m1x8_to_f16x2(kaw[w], ha);
-          e2m1x8_to_f16x2(kbw[w], hb);
+          decode8<kE1M2>(kaw[w], ha);
+          decode8<kE1M2>(kbw[w], hb);
           const uint32_t sa = w < 2 ? sa_lo : sa_hi, sb = w < 2 ? sb_lo : sb_hi;
 #pragma unroll
           for (int h = 0; h < 2; ++h) {  // k-step j = 2w + h uses bytes 2j and 2j+1
@@ -343,7 +368,8 @@ __global__ void __launch_bounds__(kThreads, NVFP4_ATTN_MIN_CTAS) attn_partial_ke
         const uint32_t pb1 = movmatrix_trans(f32x2_to_f16x2(p2, p3));
 
         // ---- O^T += V_hat^T P^T: 8 m-tiles, m-tile i = channels 16g+2i, 16g+2i+1
-        const uint32_t vs01 = e4m3x2_to_f16x2(vs01_raw), vs89 = e4m3x2_to_f16x2(vs89_raw);
+        uint32_t vs01 = e4m3x2_to_f16x2(vs01_raw), vs89 = e4m3x2_to_f16x2(vs89_raw);
+        if (kE1M2) { vs01 = hmul2(vs01, 0x38003800u); vs89 = hmul2(vs89, 0x38003800u); }
         const uint2 va = *reinterpret_cast<const uint2*>(st + kOffVc + (r0 + rv[0]) * 64 + 8 * g);
         const uint2 vb = *reinterpret_cast<const uint2*>(st + kOffVc + (r0 + rv[1]) * 64 + 8 * g);
         const uint2 vc = *reinterpret_cast<const uint2*>(st + kOffVc + (r0 + rv[2]) * 64 + 8 * g);
@@ -358,10 +384,10 @@ __global__ void __launch_bounds__(kThreads, NVFP4_ATTN_MIN_CTAS) attn_partial_ke
           const uint32_t lo_cd = (wc & 0x0F0F0F0Fu) | ((wd << 4) & 0xF0F0F0F0u);
           const uint32_t hi_cd = ((wc >> 4) & 0x0F0F0F0Fu) | (wd & 0xF0F0F0F0u);
           uint32_t f_lo_ab[4], f_hi_ab[4], f_lo_cd[4], f_hi_cd[4];
-          e2m1x8_to_f16x2(lo_ab, f_lo_ab);
-          e2m1x8_to_f16x2(hi_ab, f_hi_ab);
-          e2m1x8_to_f16x2(lo_cd, f_lo_cd);
-          e2m1x8_to_f16x2(hi_cd, f_hi_cd);
+          decode8<kE1M2>(lo_ab, f_lo_ab);
+          decode8<kE1M2>(hi_ab, f_hi_ab);
+          decode8<kE1M2>(lo_cd, f_lo_cd);
+          decode8<kE1M2>(hi_cd, f_hi_cd);
 #pragma unroll
           for (int k = 0; k < 4; ++k) {
             const uint32_t a[4] = {hmul2(f_lo_ab[k], vs01), hmul2(f_hi_ab[k], vs01), hmul2(f_lo_cd[k], vs89),
@@ -450,6 +476,7 @@ int splits_for(int capacity) { return (capacity + kChunk - 1) / kChunk; }
 constexpr size_t kSmemBytes =
     kStages * kStageBytes + (kConsumers * 8 * kD + 2 * kConsumers * 8) * sizeof(float) + 2 * kStages * 8;
 
+template <bool kE1M2>
 int resident_ctas() {
   static std::mutex mu;
   static std::map<int, int> cache;
@@ -458,16 +485,28 @@ int resident_ctas() {
   std::lock_guard<std::mutex> lock(mu);
   auto it = cache.find(d);
   if (it != cache.end()) return it->second;
-  if (cudaFuncSetAttribute(attn_partial_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  if (cudaFuncSetAttribute(attn_partial_kernel<kE1M2>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                            static_cast<int>(kSmemBytes)) != cudaSuccess)
     return 0;
   int per_sm = 0;
-  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, attn_partial_kernel, kThreads, kSmemBytes) !=
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, attn_partial_kernel<kE1M2>, kThreads, kSmemBytes) !=
           cudaSuccess ||
       per_sm <= 0)
     return 0;
   cache[d] = per_sm * sm_count();
   return cache[d];
+}
+
+// The partial kernel for the cache's element format, and its resident CTAs.
+using PartialKernel = void (*)(const Params);
+PartialKernel partial_kernel(const nvfp4_kv_cache* cache) {
+  return cache->kv_format == NVFP4_KV_E1M2 ? attn_partial_kernel<true> : attn_partial_kernel<false>;
+}
+int resident_ctas(const nvfp4_kv_cache* cache) {
+  return cache->kv_format == NVFP4_KV_E1M2 ? resident_ctas<true>() : resident_ctas<false>();
+}
+bool kv_format_ok(const nvfp4_kv_cache* cache) {
+  return cache->kv_format == NVFP4_KV_E2M1 || cache->kv_format == NVFP4_KV_E1M2;
 }
 
 }  // namespace
@@ -485,6 +524,7 @@ NVFP4_API nvfp4_status decode_attention_nvfp4(const nvfp4_kv_cache* cache, const
                                               size_t workspace_bytes, void* stream) {
   if (!cache || !q_bf16 || !out_bf16 || !workspace || !cache->seq_lens) return NVFP4_ERR_INVALID_ARG;
   if (!cache->k_codes || !cache->k_scales || !cache->v_codes || !cache->v_scales) return NVFP4_ERR_INVALID_ARG;
+  if (!kv_format_ok(cache)) return NVFP4_ERR_INVALID_ARG;
   if (!(cache->k_gscale > 0.0f && cache->k_gscale <= FLT_MAX) || !(cache->v_gscale > 0.0f && cache->v_gscale <= FLT_MAX) ||
       !(softmax_scale > 0.0f && softmax_scale <= FLT_MAX))
     return NVFP4_ERR_INVALID_ARG;
@@ -500,7 +540,7 @@ NVFP4_API nvfp4_status decode_attention_nvfp4(const nvfp4_kv_cache* cache, const
   if (!aligned(q_bf16, 16) || !aligned(out_bf16, 16) || !aligned(workspace, 16) || !aligned(cache->k_codes, 16) ||
       !aligned(cache->v_codes, 16) || !aligned(cache->k_scales, 16) || !aligned(cache->v_scales, 16))
     return NVFP4_ERR_ALIGN;
-  const int ctas_max = resident_ctas();
+  const int ctas_max = resident_ctas(cache);
   if (ctas_max <= 0) return NVFP4_ERR_CUDA;
   Params prm;
   prm.k_codes = cache->k_codes;
@@ -521,7 +561,7 @@ NVFP4_API nvfp4_status decode_attention_nvfp4(const nvfp4_kv_cache* cache, const
   prm.ml_ws = prm.o_ws + static_cast<size_t>(cache->batch) * num_q_heads * prm.n_splits * kD;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   const int grid = static_cast<int>(n_items < ctas_max ? n_items : ctas_max);
-  if (launch_pdl(attn_partial_kernel, dim3(grid), dim3(kThreads), kSmemBytes, s, prm) != cudaSuccess ||
+  if (launch_pdl(partial_kernel(cache), dim3(grid), dim3(kThreads), kSmemBytes, s, prm) != cudaSuccess ||
       launch_pdl(attn_combine_kernel, dim3(num_q_heads, cache->batch), dim3(kD), 0, s,
                  static_cast<const float*>(prm.o_ws), static_cast<const float*>(prm.ml_ws), prm.n_splits,
                  cache->v_gscale, static_cast<uint16_t*>(out_bf16)) != cudaSuccess)
@@ -565,6 +605,7 @@ NVFP4_API nvfp4_status decode_attention_nvfp4_static_scratch(const nvfp4_kv_cach
                                                              void* out_bf16, void* stream) {
   if (!cache || !q_bf16 || !out_bf16 || !cache->seq_lens) return NVFP4_ERR_INVALID_ARG;
   if (!cache->k_codes || !cache->k_scales || !cache->v_codes || !cache->v_scales) return NVFP4_ERR_INVALID_ARG;
+  if (!kv_format_ok(cache)) return NVFP4_ERR_INVALID_ARG;
   if (!(cache->k_gscale > 0.0f && cache->k_gscale <= FLT_MAX) || !(cache->v_gscale > 0.0f && cache->v_gscale <= FLT_MAX) ||
       !(softmax_scale > 0.0f && softmax_scale <= FLT_MAX))
     return NVFP4_ERR_INVALID_ARG;
@@ -584,7 +625,7 @@ NVFP4_API nvfp4_status decode_attention_nvfp4_static_scratch(const nvfp4_kv_cach
     return NVFP4_ERR_ALIGN;
   float* scratch = attn_static_scratch_dev();
   if (!scratch) return NVFP4_ERR_CUDA;
-  const int ctas_max = resident_ctas();
+  const int ctas_max = resident_ctas(cache);
   if (ctas_max <= 0) return NVFP4_ERR_CUDA;
   Params prm;
   prm.k_codes = cache->k_codes;
@@ -607,7 +648,7 @@ NVFP4_API nvfp4_status decode_attention_nvfp4_static_scratch(const nvfp4_kv_cach
   prm.ml_ws = prm.o_ws + static_cast<size_t>(cache->batch) * num_q_heads * prm.n_splits * kD;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   const int grid = static_cast<int>(n_items < ctas_max ? n_items : ctas_max);
-  if (launch_pdl(attn_partial_kernel, dim3(grid), dim3(kThreads), kSmemBytes, s, prm) != cudaSuccess ||
+  if (launch_pdl(partial_kernel(cache), dim3(grid), dim3(kThreads), kSmemBytes, s, prm) != cudaSuccess ||
       launch_pdl(attn_combine_kernel, dim3(num_q_heads, cache->batch), dim3(kD), 0, s,
                  static_cast<const float*>(prm.o_ws), static_cast<const float*>(prm.ml_ws), prm.n_splits,
                  cache->v_gscale, static_cast<uint16_t*>(out_bf16)) != cudaSuccess)

@@ -18,7 +18,7 @@ constexpr int kThreads = 256;
 // kRope: K arrives before RoPE and is rotated here (rotate-half pairing,
 // channel i with i + 64) with the (cos, sin) table row of its position, in
 // fp32: y_i = x_i c_i - x_{i+64} s_i, y_{i+64} = x_i s_i + x_{i+64} c_i.
-template <bool kRope>
+template <bool kRope, bool kE1M2>
 __global__ void __launch_bounds__(kThreads) kv_append_kernel(
     const uint16_t* __restrict__ k_in, const uint16_t* __restrict__ v_in, const int32_t* __restrict__ seq_idx,
     const int32_t* __restrict__ pos, const float* __restrict__ k_shift, const float* __restrict__ rope,
@@ -27,7 +27,8 @@ __global__ void __launch_bounds__(kThreads) kv_append_kernel(
   griddep_wait_and_release();
   const uint32_t total = n_rows * 32u;  // 2 tensors x 16 chunks per row: a multiple of the warp
   const uint32_t lane = threadIdx.x & 31;
-  const float six_gk = __fmul_rn(6.0f, gk), six_gv = __fmul_rn(6.0f, gv);
+  const float qmax = kE1M2 ? 3.5f : 6.0f;  // largest element magnitude of the grid
+  const float six_gk = __fmul_rn(qmax, gk), six_gv = __fmul_rn(qmax, gv);
   for (uint32_t c0 = blockIdx.x * blockDim.x + (threadIdx.x & ~31u); c0 < total; c0 += gridDim.x * blockDim.x) {
     const uint32_t c = c0 + lane;
     const bool live = c < total;
@@ -77,7 +78,7 @@ __global__ void __launch_bounds__(kThreads) kv_append_kernel(
 #pragma unroll
     for (int i = 0; i < 8; ++i) amax = fmaxf(amax, fabsf(x[i]));
     uint32_t sc;
-    const uint32_t packed = quantize8_pair(x, amax, is_v ? gv : gk, is_v ? six_gv : six_gk, &sc);
+    const uint32_t packed = quantize8_pair<kE1M2>(x, amax, is_v ? gv : gk, is_v ? six_gv : six_gk, &sc);
     if (!live) continue;
     const int32_t b = __ldg(seq_idx + tok), p = __ldg(pos + tok);
     if (b < 0 || static_cast<uint32_t>(b) >= batch || p < 0 || static_cast<uint32_t>(p) >= capacity) {
@@ -98,6 +99,7 @@ nvfp4_status append(const nvfp4_kv_cache* cache, const void* k_bf16, const void*
   if (!cache->k_codes || !cache->k_scales || !cache->v_codes || !cache->v_scales) return NVFP4_ERR_INVALID_ARG;
   if (!(cache->k_gscale > 0.0f && cache->k_gscale <= FLT_MAX) || !(cache->v_gscale > 0.0f && cache->v_gscale <= FLT_MAX))
     return NVFP4_ERR_INVALID_ARG;
+  if (cache->kv_format != NVFP4_KV_E2M1 && cache->kv_format != NVFP4_KV_E1M2) return NVFP4_ERR_INVALID_ARG;
   if (cache->head_dim != 128 || cache->batch <= 0 || cache->num_kv_heads <= 0 || cache->capacity <= 0 || n_new < 0)
     return NVFP4_ERR_SHAPE;
   if (n_new * cache->num_kv_heads * 32 >= (1ll << 32)) return NVFP4_ERR_SHAPE;
@@ -111,8 +113,11 @@ nvfp4_status append(const nvfp4_kv_cache* cache, const void* k_bf16, const void*
   uint64_t grid = (items + kThreads - 1) / kThreads;
   const uint64_t cap = static_cast<uint64_t>(sm_count()) * 8;
   if (grid > cap) grid = cap;
+  const bool e1m2 = cache->kv_format == NVFP4_KV_E1M2;
+  const auto kernel = rope ? (e1m2 ? kv_append_kernel<true, true> : kv_append_kernel<true, false>)
+                           : (e1m2 ? kv_append_kernel<false, true> : kv_append_kernel<false, false>);
   const cudaError_t e =
-      launch_pdl(rope ? kv_append_kernel<true> : kv_append_kernel<false>, dim3(static_cast<int>(grid)), dim3(kThreads),
+      launch_pdl(kernel, dim3(static_cast<int>(grid)), dim3(kThreads),
                  0, static_cast<cudaStream_t>(stream), static_cast<const uint16_t*>(k_bf16),
                  static_cast<const uint16_t*>(v_bf16), seq_idx, pos, k_shift, rope, n_rows,
                  FastDiv(static_cast<uint32_t>(cache->num_kv_heads)), static_cast<uint32_t>(cache->batch),

@@ -53,6 +53,20 @@ __device__ __forceinline__ uint32_t e2m1x8(const float v[8]) {
   return out;
 }
 
+// 8 fp32 -> 8 E1M2 elements (the KV variant), element 0 in the lowest nibble:
+// k = RNE(2|v|) saturated at 7, stored as the two's-complement nibble of
+// sign * k (a negative value that rounds to zero is stored as 0).
+__device__ __forceinline__ uint32_t e1m2x8(const float v[8]) {
+  uint32_t out = 0;
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    const int k = min(__float2int_rn(fabsf(v[i]) * 2.0f), 7);
+    const int n = signbit(v[i]) ? -k : k;
+    out |= (static_cast<uint32_t>(n) & 0xFu) << (4 * i);
+  }
+  return out;
+}
+
 // bf16 -> fp32 (exact) for the low / high half of a 32-bit pair.
 __device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
 __device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
@@ -77,15 +91,17 @@ __device__ __forceinline__ uint32_t amax_bits_bf16x8(const uint4 v) {
 // Quantize 8 fp32 values whose block partner lane holds the other 8.  All 32
 // lanes of the warp must call this together.  Returns packed codes; *scale
 // receives the block's E4M3 code (identical in both lanes).
-__device__ __forceinline__ uint32_t quantize8_pair(const float x[8], float amax_own, float g, float six_g,
+// kE1M2: E1M2 elements; qmax_g is then 3.5 g instead of 6 g.
+template <bool kE1M2 = false>
+__device__ __forceinline__ uint32_t quantize8_pair(const float x[8], float amax_own, float g, float qmax_g,
                                                    uint32_t* scale) {
   const float amax = fmaxf(amax_own, __shfl_xor_sync(0xffffffffu, amax_own, 1));
-  const BlockScale b = block_scale(amax, g, six_g);
+  const BlockScale b = block_scale(amax, g, qmax_g);
   float v[8];
 #pragma unroll
   for (int i = 0; i < 8; ++i) v[i] = __fmul_rn(x[i], b.mult);
   *scale = b.code;
-  return e2m1x8(v);
+  return kE1M2 ? e1m2x8(v) : e2m1x8(v);
 }
 
 // Byte offset of block scale (row r, k-block kb) in the tensor-core storage

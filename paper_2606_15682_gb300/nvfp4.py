@@ -39,7 +39,7 @@ _p, _i64, _i32, _f32, _sz = ctypes.c_void_p, ctypes.c_int64, ctypes.c_int32, cty
 class KVCacheStruct(ctypes.Structure):
     _fields_ = [("k_codes", _p), ("k_scales", _p), ("v_codes", _p), ("v_scales", _p), ("seq_lens", _p),
                 ("batch", _i32), ("num_kv_heads", _i32), ("head_dim", _i32), ("capacity", _i32),
-                ("k_gscale", _f32), ("v_gscale", _f32)]
+                ("k_gscale", _f32), ("v_gscale", _f32), ("kv_format", _i32)]
 
 
 def _sig(name, args, res=ctypes.c_int):
@@ -116,6 +116,7 @@ def nvfp4_quantize(x, g, codes, scales, layout=SCALES_MMA, stream=None):
 
 
 DYNAMIC_STATE_BYTES = 16
+KV_E2M1, KV_E1M2 = 0, 1
 
 
 def nvfp4_quantize_dynamic(x, state, g, codes, scales, layout=SCALES_MMA, stream=None):
@@ -207,8 +208,9 @@ def nvfp4_launch_count():
 class KVCache:
     """Caller-owned NVFP4 KV cache buffers (layout of include/nvfp4.h)."""
 
-    def __init__(self, batch, num_kv_heads, capacity, k_gscale, v_gscale, head_dim=128, device="cuda"):
+    def __init__(self, batch, num_kv_heads, capacity, k_gscale, v_gscale, head_dim=128, device="cuda", kv_format=0):
         self.batch, self.num_kv_heads, self.capacity, self.head_dim = batch, num_kv_heads, capacity, head_dim
+        self.kv_format = kv_format  # KV_E2M1 or KV_E1M2
         self.k_gscale, self.v_gscale = float(k_gscale), float(v_gscale)
         shape = (batch, num_kv_heads, capacity)
         self.k_codes = torch.zeros(shape + (head_dim // 2,), dtype=torch.uint8, device=device)
@@ -220,7 +222,7 @@ class KVCache:
     def struct(self):
         return KVCacheStruct(self.k_codes.data_ptr(), self.k_scales.data_ptr(), self.v_codes.data_ptr(),
                              self.v_scales.data_ptr(), self.seq_lens.data_ptr(), self.batch, self.num_kv_heads,
-                             self.head_dim, self.capacity, self.k_gscale, self.v_gscale)
+                             self.head_dim, self.capacity, self.k_gscale, self.v_gscale, self.kv_format)
 
 
 EXPORTED = ["nvfp4_scales_bytes", "nvfp4_tensor_scale", "nvfp4_quantize", "nvfp4_quantize_dynamic", "nvfp4_scales_relayout", "nvfp4_linear",

@@ -84,6 +84,9 @@ def test_kv_and_attention_validation():
     assert L.kv_append_nvfp4(ctypes.byref(cache(head_dim=64)), p, p, p, p, 1, None, s) == 2
     assert L.kv_append_nvfp4(ctypes.byref(cache(k_gscale=0.0)), p, p, p, p, 1, None, s) == 1
     assert L.kv_append_nvfp4(ctypes.byref(cache()), None, p, p, p, 1, None, s) == 1
+    # KV element format must be one of the enum's values
+    assert L.kv_append_nvfp4(ctypes.byref(cache(kv_format=2)), p, p, p, p, 1, None, s) == 1
+    assert L.decode_attention_nvfp4(ctypes.byref(cache(kv_format=-1)), p, 4, ctypes.c_float(0.1), p, p, 1 << 30, s) == 1
     # fused RoPE append: table required, and it must cover every cache position
     odd = ctypes.c_void_p(0x10004)
     assert L.kv_append_rope_nvfp4(ctypes.byref(cache()), p, p, p, p, 1, None, 64, None, s) == 1

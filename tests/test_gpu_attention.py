@@ -267,3 +267,71 @@ def test_kv_append_rope_then_attention_matches_fp64(N):
                              1 / math.sqrt(128))
     for b in range(B):
         assert_close(f32(out)[b], ref[b], what=f"seq {b}")
+
+
+# ------------------------------------------------------ E1M2 KV elements ---
+
+@pytest.mark.parametrize("rope", [False, True])
+def test_kv_append_e1m2_bit_exact(N, rope):
+    B, hkv, cap, n = 3, 8, 64, 140
+    rec = synth.KVRecipe(hkv, seed=33)
+    k, v = rec.kv(n, seed=9)
+    rng = np.random.default_rng(17)
+    seq = rng.integers(0, B, n); pos = rng.permutation(B * cap)[:n] % cap
+    pairs = {}
+    for i in range(n):
+        pairs[(seq[i], pos[i])] = i
+    keep = np.array(sorted(pairs.values()))
+    k, v, seq, pos = k[keep], v[keep], seq[keep], pos[keep]
+    table = O.rope_table(cap)
+    kq = O.rope_f32(f32(k), pos, table) if rope else f32(k)
+    shift = (kq.mean(axis=0) * 0.5).astype(np.float32)
+    gk = np.float32(np.abs(kq - shift).max() / (3.5 * 448))
+    gv = np.float32(np.abs(f32(v)).max() / (3.5 * 448))
+    cache = N.KVCache(B, hkv, cap, gk, gv, kv_format=N.KV_E1M2)
+    args = (k.cuda(), v.cuda(), torch.as_tensor(seq, dtype=torch.int32, device="cuda"),
+            torch.as_tensor(pos, dtype=torch.int32, device="cuda"))
+    if rope:
+        N.kv_append_rope_nvfp4(cache, *args, torch.from_numpy(table).cuda(), torch.from_numpy(shift).cuda())
+    else:
+        N.kv_append_nvfp4(cache, *args, torch.from_numpy(shift).cuda())
+    torch.cuda.synchronize()
+    assert N.nvfp4_get_device_status() == 0
+    rkc, rks, rvc, rvs = oracle_cache(B, hkv, cap)
+    if rope:
+        O.kv_append_rope(rkc, rks, rvc, rvs, f32(k), f32(v), seq, pos, gk, gv, table, k_shift=shift, element="e1m2")
+    else:
+        O.kv_append(rkc, rks, rvc, rvs, f32(k), f32(v), seq, pos, gk, gv, k_shift=shift, element="e1m2")
+    assert np.array_equal(u8(cache.k_scales), rks) and np.array_equal(u8(cache.k_codes), rkc)
+    assert np.array_equal(u8(cache.v_scales), rvs) and np.array_equal(u8(cache.v_codes), rvc)
+
+
+@pytest.mark.parametrize("B,hq,hkv,lens", [(2, 10, 2, [300, 1030]), (3, 8, 8, [17, 2049, 1])])
+def test_decode_attention_e1m2_matches_fp64(N, B, hq, hkv, lens):
+    cap = (max(lens) + 6) & ~1
+    rec = synth.KVRecipe(hkv, seed=58)
+    cache = N.KVCache(B, hkv, cap, 1.0, 1.0, kv_format=N.KV_E1M2)
+    ks, vs, seqs, poss = [], [], [], []
+    for b, T in enumerate(lens):
+        k, v = rec.kv(T, seed=300 + b)
+        ks.append(k); vs.append(v); seqs.append(np.full(T, b)); poss.append(np.arange(T))
+    kall, vall = torch.cat(ks), torch.cat(vs)
+    seq, pos = np.concatenate(seqs), np.concatenate(poss)
+    gk = np.float32(np.abs(f32(kall)).max() / (3.5 * 448)); gv = np.float32(np.abs(f32(vall)).max() / (3.5 * 448))
+    cache.k_gscale, cache.v_gscale = float(gk), float(gv)
+    N.kv_append_nvfp4(cache, kall.cuda(), vall.cuda(), torch.as_tensor(seq, dtype=torch.int32, device="cuda"),
+                      torch.as_tensor(pos, dtype=torch.int32, device="cuda"))
+    cache.seq_lens.copy_(torch.tensor(lens, dtype=torch.int32))
+    q = rec.queries(B, hq, seed=5)
+    out = torch.empty(B, hq, 128, dtype=torch.bfloat16, device="cuda")
+    ws = torch.empty(N.decode_attention_nvfp4_workspace_size(B, hq, cap) // 4, dtype=torch.float32, device="cuda")
+    N.decode_attention_nvfp4(cache, q.cuda(), 1 / math.sqrt(128), out, ws)
+    torch.cuda.synchronize()
+    assert N.nvfp4_get_device_status() == 0
+    # the oracle builds its own cache from the same inputs (the append is bit-exact, tested above)
+    rkc, rks, rvc, rvs = oracle_cache(B, hkv, cap)
+    O.kv_append(rkc, rks, rvc, rvs, f32(kall), f32(vall), seq, pos, gk, gv, element="e1m2")
+    ref = O.decode_attention(f32(q), rkc, rks, rvc, rvs, np.array(lens), gk, gv, 1 / math.sqrt(128),
+                             element="e1m2")
+    for b in range(B):
+        assert_close(f32(out)[b], ref[b], what=f"seq {b}")
