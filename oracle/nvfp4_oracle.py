@@ -24,7 +24,10 @@ readability, not speed:
   (cos, sin) table in a fixed order of operations (``rope_f32``);
 * the gate_up projection with the SwiGLU product and the NVFP4 quantization of
   the down projection's input fused behind it (``linear_swiglu_quantize``);
-* the E1M2 element grid for the KV cache (``e1m2_*``, ``element="e1m2"``).
+* the E1M2 element grid for the KV cache (``e1m2_*``, ``element="e1m2"``);
+* the Q-FIT calibration (Algorithm 1): the paired pre-RoPE scale and the
+  post-RoPE shift chosen by a grid search on the KV4 attention error
+  (``qfit_calibrate``).
 
 Floating-point conventions: the quantizer's arithmetic is IEEE fp32 with
 round-to-nearest-even (numpy float32 scalars/arrays, no fused multiply-add);
@@ -492,3 +495,93 @@ def qfit_transform(q_pre, k_pre, s, m, positions, theta=1.0e6):
     """Q~ = R(Q_pre * s), K~ = R(K_pre / s) - m  (Eq. 2), fp64."""
     s = np.asarray(s, dtype=np.float64)
     return rope(q_pre * s, positions, theta), rope(k_pre / s, positions, theta) - np.asarray(m, np.float64)
+
+
+# ---------------------------------------------------------------------------
+# Q-FIT calibration (Algorithm 1, Sec. 4 / the Q-FIT appendix): choose the
+# paired pre-RoPE scale S and the post-RoPE key shift m that minimize the MSE
+# between a reference attention and the attention over the KV4 cache.
+# Readings where the algorithm leaves a choice open:
+#   * RoPE is the fp32 table form ``rope_f32`` (tables from ``rope_table``);
+#     the scaled keys K_pre / S_K are rounded to bf16 before RoPE, as a key
+#     projection with S folded into its weights would produce them.
+#   * Attn(Q, K, V) is evaluated for the queries at positions ``q_pos``, each
+#     attending to all T cached tokens, with softmax scale 1/sqrt(d) (decode
+#     form; the calibration sequence is the cache).
+#   * Q_KV4 uses a static tensor scale per grid point: g = amax / (qmax * 448)
+#     of the tensor being cached (K~ - m, or V).
+#   * the shift template mu is the token mean of RoPE(K_pre) (unscaled keys),
+#     as written; m(alpha_m) = alpha_m * mu at every alpha_s.
+# ---------------------------------------------------------------------------
+
+
+def _bf16_round(x):
+    """Round fp32 values to bf16 (RNE) and back to fp32."""
+    b = np.asarray(x, dtype=np.float32).view(np.uint32).astype(np.uint64)
+    b = (b + 0x7FFF + ((b >> 16) & 1)) >> 16
+    return (b << 16).astype(np.uint32).view(np.float32)
+
+
+def qfit_init_scale(k_pre, eps):
+    """S_K^0[h, r] = max(max_t |K[t,h,r]|, max_t |K[t,h,r+d/2]|, eps), shared by the
+    pair (r, r + d/2) so the scaling commutes with RoPE.  k_pre [T, H_kv, d]."""
+    k = np.abs(np.asarray(k_pre, dtype=np.float64))
+    half = k.shape[-1] // 2
+    m = np.maximum(k[..., :half].max(axis=0), k[..., half:].max(axis=0))
+    s0 = np.maximum(m, eps)
+    return np.concatenate([s0, s0], axis=-1)                       # [H_kv, d]
+
+
+def qfit_attention_error(q_pre, k_pre, v, table, q_pos, s_k, s_q, m, element="e2m1"):
+    """MSE between the reference attention (RoPE'd Q and K, exact V) and the
+    attention over the KV4 cache holding Q_KV4(RoPE(K_pre / s_k) - m), Q_KV4(V)
+    for queries RoPE(Q_pre * s_q) (one grid point of Algorithm 1)."""
+    T, hkv, d = k_pre.shape
+    hq = q_pre.shape[1]
+    pos = np.arange(T)
+    qmax = 6.0 if element == "e2m1" else E1M2_MAX
+    # reference: unscaled, unshifted, unquantized
+    k0 = rope_f32(k_pre, pos, table).astype(np.float64)
+    q0 = rope_f32(q_pre[q_pos], q_pos, table).astype(np.float64)
+    scale = 1.0 / np.sqrt(d)
+    group = hq // hkv
+    y_ref = np.stack([[attention_fp64(q0[i, h], k0[:, h // group], np.asarray(v, np.float64)[:, h // group], scale)
+                       for h in range(hq)] for i in range(len(q_pos))])
+    # transformed and quantized
+    k_in = _bf16_round(np.asarray(k_pre, np.float32) / np.asarray(s_k, np.float32)[None])
+    kt = rope_f32(k_in, pos, table)
+    kt = (kt - np.asarray(m, np.float32)[None]).astype(np.float32)
+    g_k = np.float32(np.abs(kt).max() / (qmax * 448))
+    g_v = np.float32(np.abs(np.asarray(v, np.float32)).max() / (qmax * 448))
+    kc, ks = quantize(kt.reshape(T * hkv, d), g_k, element)
+    vc, vs = quantize(np.asarray(v, np.float32).reshape(T * hkv, d), g_v, element)
+    K = dequantize(kc, ks, g_k, element).reshape(T, hkv, d)
+    V = dequantize(vc, vs, g_v, element).reshape(T, hkv, d)
+    q_in = np.asarray(q_pre, np.float32)[q_pos] * np.repeat(np.asarray(s_q, np.float32), 1, axis=0)[None]
+    qt = _bf16_round(rope_f32(q_in.astype(np.float32), q_pos, table)).astype(np.float64)
+    y = np.stack([[attention_fp64(qt[i, h], K[:, h // group], V[:, h // group], scale) for h in range(hq)]
+                  for i in range(len(q_pos))])
+    return float(np.mean((y - y_ref) ** 2))
+
+
+def qfit_calibrate(q_pre, k_pre, v, table, q_pos, grid_s, grid_m, eps=1e-6, element="e2m1"):
+    """Algorithm 1: returns (s_q, s_k, m, errors[grid_s, grid_m])."""
+    hkv = k_pre.shape[1]
+    hq = q_pre.shape[1]
+    s0_k = qfit_init_scale(k_pre, eps)
+    s0_q = np.repeat(s0_k, hq // hkv, axis=0)                      # Replicate to query heads
+    mu = rope_f32(k_pre, np.arange(k_pre.shape[0]), table).astype(np.float64).mean(axis=0)
+    errors = np.full((grid_s, grid_m), np.inf)
+    best = None
+    for a in range(grid_s):
+        alpha_s = a / grid_s
+        s_k = (s0_k ** alpha_s).astype(np.float32)
+        s_q = (s0_q ** alpha_s).astype(np.float32)
+        for b in range(grid_m):
+            alpha_m = b / grid_m
+            m = (alpha_m * mu).astype(np.float32)
+            e = qfit_attention_error(q_pre, k_pre, v, table, q_pos, s_k, s_q, m, element)
+            errors[a, b] = e
+            if best is None or e < best[0]:
+                best = (e, s_q, s_k, m)
+    return best[1], best[2], best[3], errors

@@ -484,3 +484,57 @@ def test_e1m2_quantize_scale_closed_form_and_error_bound():
     # uniform grid with step 0.5: error <= 0.25 scale units inside the range, plus E4M3's
     # rounding of the scale below amax (at most 1/16 of 3.5 units) at the block maximum
     assert np.all(np.abs(xh - x) <= (0.25 + 3.5 / 16) * Sv + 1e-12)
+
+
+# -------------------------------------------------- Q-FIT calibration (Alg. 1) ---
+
+def test_qfit_init_scale_pairs_and_floor():
+    k = np.zeros((3, 1, 8)); k[0, 0, 1] = -5.0; k[2, 0, 5] = 7.0; k[1, 0, 3] = 2.0
+    s0 = O.qfit_init_scale(k, eps=0.5)
+    # pairs (r, r+4): (0,4) -> eps, (1,5) -> max(5, 7) = 7, (2,6) -> eps, (3,7) -> 2
+    assert np.array_equal(s0[0], [0.5, 7, 0.5, 2, 0.5, 7, 0.5, 2])
+
+
+def _qfit_data(T=96, hq=4, hkv=2, d=128, seed=3, offset=3.0):
+    rng = np.random.default_rng(seed)
+    spread = np.exp(rng.standard_normal((hkv, d)))                 # channel outliers (paired scaling helps)
+    k = (rng.standard_normal((T, hkv, d)) * spread + offset).astype(np.float32)   # a mean (the shift helps)
+    q = rng.standard_normal((T, hq, d)).astype(np.float32)
+    v = rng.standard_normal((T, hkv, d)).astype(np.float32)
+    return _bf(q), _bf(k), _bf(v)
+
+
+def _bf(x):
+    return O._bf16_round(x)
+
+
+def test_qfit_identity_point_and_invariance_without_quantization(monkeypatch):
+    q, k, v = _qfit_data()
+    tab = O.rope_table(k.shape[0])
+    qp = np.array([10, 50, 95])
+    # With the quantizer replaced by the identity, every grid point reproduces the
+    # reference (paired scaling and the shift leave attention unchanged), up to the
+    # bf16 rounding of the scaled inputs.
+    e_q = O.qfit_attention_error(q, k, v, tab, qp, np.ones((2, 128), np.float32), np.ones((4, 128), np.float32),
+                                 np.zeros((2, 128), np.float32))     # with the KV4 quantizer: ~4e-2
+    monkeypatch.setattr(O, "quantize", lambda x, g, element="e2m1": (np.asarray(x, np.float32), g))
+    monkeypatch.setattr(O, "dequantize", lambda c, s, g, element="e2m1": np.asarray(c, np.float64))
+    s0 = O.qfit_init_scale(k, 1e-6)
+    mu = O.rope_f32(k, np.arange(k.shape[0]), tab).astype(np.float64).mean(axis=0)
+    for alpha_s, alpha_m in [(0.0, 0.0), (0.5, 0.5), (0.8, 0.8)]:
+        e = O.qfit_attention_error(q, k, v, tab, qp, (s0 ** alpha_s).astype(np.float32),
+                                   np.repeat(s0 ** alpha_s, 2, axis=0).astype(np.float32),
+                                   (alpha_m * mu).astype(np.float32))
+        # bf16 rounding of the scaled q and k (relative 2^-9) is all that remains
+        assert e < 1e-4 and e < 1e-2 * e_q, (alpha_s, alpha_m, e, e_q)
+
+
+def test_qfit_calibration_prefers_the_shift_for_offset_keys():
+    q, k, v = _qfit_data(offset=6.0)
+    tab = O.rope_table(k.shape[0])
+    qp = np.arange(80, 96)
+    s_q, s_k, m, err = O.qfit_calibrate(q, k, v, tab, qp, grid_s=3, grid_m=4)
+    assert err.shape == (3, 4) and np.isfinite(err).all()
+    # keys with a large common offset: some shift beats none at alpha_s = 0
+    assert err[0, 1:].min() < err[0, 0]
+    assert np.isclose(err.min(), O.qfit_attention_error(q, k, v, tab, qp, s_k, s_q, m))
