@@ -219,3 +219,21 @@ def test_linear_swiglu_quantize_prefill_shape_then_down(N):
     assert N.nvfp4_get_device_status() == 0
     ref = O.linear_rows(out_c, O.scales_from_mma(out_s, M, I), g_out, wd_c, wd_s, g_wd, rows)
     assert_close(f32(out[torch.as_tensor(rows, device="cuda")]), ref, what="down(swiglu)")
+
+
+def test_linear_swiglu_quantize_invalid_g_out_zeroes_and_reports(N):
+    M, I, K = 256, 128, 256
+    gen = torch.Generator().manual_seed(3)
+    a_c, a_s = random_operand(M, K, gen)
+    w_c, w_s = random_operand(2 * I, K, gen)
+    dev = "cuda"
+    out_c = torch.full((M, I // 2), 0xEE, dtype=torch.uint8, device=dev)
+    out_s = torch.full((N.nvfp4_scales_bytes(M, I, 1),), 0xEE, dtype=torch.uint8, device=dev)
+    N.nvfp4_get_device_status()
+    N.nvfp4_linear_swiglu_quantize(torch.from_numpy(a_c).to(dev), torch.from_numpy(O.scales_to_mma(a_s)).to(dev),
+                                   torch.ones(1, device=dev), torch.from_numpy(w_c).to(dev),
+                                   torch.from_numpy(O.scales_to_mma(w_s)).to(dev), torch.ones(1, device=dev),
+                                   M, I, K, torch.tensor([-1.0], device=dev), out_c, out_s)
+    torch.cuda.synchronize()
+    assert N.nvfp4_get_device_status() == 1
+    assert not u8(out_c).any() and not u8(out_s).any()

@@ -257,3 +257,23 @@ def test_dynamic_workload_activations(N, workload):
         rc, rs = O.quantize(f32(a[torch.as_tensor(rows, device="cuda")]), np.float32(g.item()))
         assert np.array_equal(u8(codes)[rows], rc)
         assert np.array_equal(O.scales_from_mma(u8(scales), a.shape[0], a.shape[1])[rows], rs)
+
+
+def test_dynamic_barrier_wait_runs_out_and_reports_timeout(N):
+    """A state whose arrival count can never reach the grid size (a flag that
+    nothing sets): every block's bounded barrier wait expires after ~2 s, the
+    kernel returns without writing, NVFP4_ERR_TIMEOUT is reported, and the
+    device stays usable -- a zero-filled state works again afterwards."""
+    x = torch.randn(256, 1024, device="cuda").to(torch.bfloat16)
+    state = torch.zeros(N.DYNAMIC_STATE_BYTES // 8, dtype=torch.int64, device="cuda")
+    state[0] = 0x7FFFFF00          # epoch 0, an arrival count far beyond any grid
+    N.nvfp4_get_device_status()
+    codes, scales, g = dynamic(N, x, state.view(torch.uint8))
+    torch.cuda.synchronize()
+    assert N.nvfp4_get_device_status() == 6
+    assert np.isnan(g.item()), "g must stay unwritten after a timeout"
+    state.zero_()
+    codes, scales, g = dynamic(N, x, state.view(torch.uint8))
+    torch.cuda.synchronize()
+    assert N.nvfp4_get_device_status() == 0
+    assert np.float32(g.item()) == O.tensor_scale(f32(x))
