@@ -1055,13 +1055,20 @@ NVFP4_API nvfp4_status nvfp4_linear(const uint8_t* a_codes, const uint8_t* a_sca
     return NVFP4_ERR_ALIGN;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   const int64_t tiles_m = (M + BM - 1) / BM;
-  const int bn = NVFP4_GEMM_BN ? NVFP4_GEMM_BN : (N % 256 == 0 ? 256 : 128);
   // Measured on GB300: sharing W tiles by cluster multicast did not beat
   // independent CTAs on these shapes (the cluster waits for its slowest CTA),
   // so clusters are off by default; the multicast path stays selectable.
   const int cm = NVFP4_GEMM_CM ? NVFP4_GEMM_CM : 1;
-  if (NVFP4_GEMM_PAIR && N % 256 == 0 && tiles_m >= 2)
-    return launch_pair<PairCfg<NVFP4_GEMM_PAIR_STAGES>>(a_codes, a_scales, g_a, w_codes, w_scales, g_w, M, N, K, out_bf16, ldo, s);
+  // The CTA pair, unless its 256 x 256 tiles would leave most pairs idle
+  // (decode-sized M): then 128 x 128 tiles on single CTAs spread the W stream
+  // over more SMs (measured faster at M = 256 with N = 5120 or 7168, slower
+  // with N = 27648).
+  using Pair = PairCfg<NVFP4_GEMM_PAIR_STAGES>;
+  if (NVFP4_GEMM_PAIR && N % 256 == 0 && tiles_m >= 2 &&
+      2 * ((tiles_m + 1) / 2) * (N / 256) >= resident_pairs<Pair, false>())
+    return launch_pair<Pair>(a_codes, a_scales, g_a, w_codes, w_scales, g_w, M, N, K, out_bf16, ldo, s);
+  // Single CTAs: BN = 128 (measured faster than 256 at M <= 256 on GB300).
+  const int bn = NVFP4_GEMM_BN ? NVFP4_GEMM_BN : 128;
 #define NVFP4_LAUNCH(BN_, ST_, CM_) \
   return launch<Cfg<BN_, ST_, CM_>>(a_codes, a_scales, g_a, w_codes, w_scales, g_w, M, N, K, out_bf16, ldo, s)
   if (bn == 256) {

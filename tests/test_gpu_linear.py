@@ -47,8 +47,13 @@ def run_linear(N, a_codes, a_scales_rm, g_a, w_codes, w_scales_rm, g_w, M, Nn, K
 
 @pytest.mark.parametrize("M,Nn,K", [(128, 128, 256), (1, 16, 256), (16, 128, 512), (130, 144, 512),
                                     (257, 384, 1024), (300, 272, 2304), (128, 1024, 256),
-                                    # CTA-pair path (N % 256 == 0, more than one 128-row tile), odd tile counts
-                                    (256, 256, 512), (300, 512, 1024), (640, 768, 768), (129, 1280, 2048)])
+                                    # N % 256 == 0 with few 256 x 256 tiles: single CTAs
+                                    (256, 256, 512), (300, 512, 1024), (640, 768, 768), (129, 1280, 2048),
+                                    # CTA-pair path (enough 256 x 256 tiles to occupy the pairs):
+                                    # M tails with a spare CTA, odd super-tile counts, one-row tail
+                                    (256, 10240, 512), (300, 10240, 1024), (640, 5120, 768), (129, 12800, 256),
+                                    # more 256 x 256 tiles than pairs: a second round of tiles
+                                    (512, 10240, 1024), (300, 15360, 1536), (640, 7680, 1280)])
 def test_random_codes(N, M, Nn, K):
     gen = torch.Generator().manual_seed(M * 1000 + Nn * 10 + K)
     a_c, a_s = random_operand(M, K, gen)
