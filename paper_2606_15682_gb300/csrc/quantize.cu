@@ -202,13 +202,31 @@ __device__ __forceinline__ unsigned long long ld_acquire_u64(const unsigned long
   return v;
 }
 
+__device__ __forceinline__ unsigned long long atom_add_acq_rel_u64(unsigned long long* p, unsigned long long v) {
+  unsigned long long old;
+  asm volatile("atom.acq_rel.gpu.global.add.u64 %0, [%1], %2;" : "=l"(old) : "l"(p), "l"(v) : "memory");
+  return old;
+}
+__device__ __forceinline__ void red_max_u64(unsigned long long* p, unsigned long long v) {
+  asm volatile("red.relaxed.gpu.global.max.u64 [%0], %1;" ::"l"(p), "l"(v) : "memory");
+}
+__device__ __forceinline__ void st_release_u64(unsigned long long* p, unsigned long long v) {
+  asm volatile("st.release.gpu.global.u64 [%0], %1;" ::"l"(p), "l"(v) : "memory");
+}
+
 // a1 + a2 in one cooperative launch.  Phase 1 reduces amax(|x|) over the
 // same 16-element blocks phase 2 quantizes; a grid-wide barrier separates
 // them.  Caller-owned state (two 64-bit words, zero before the first call):
-//   state[0] = (call epoch << 32) | blocks arrived in this epoch
-//   state[1] = (epoch << 32) | amax bits, combined with atomicMax
+//   state[0] = (call epoch << 32) | (previous call's amax bits << 16) | blocks arrived
+//   state[1] = (epoch << 32) | amax bits, combined with a max reduction
 // A newer epoch's tag dominates any older value, so nothing is cleared
-// between calls; the last block to arrive opens the next epoch.
+// between calls.  Each block max-reduces its amax into state[1], then counts
+// itself into state[0] with an acquire-release add (the release orders the
+// reduction before the count).  The last block to arrive reads the total
+// amax (its acquire made every reduction visible) and opens the next epoch
+// with one release store that also carries the amax, so the waiting blocks
+// learn both from the load that ends their wait.  The epoch is read before
+// the loads of phase 1: it cannot change until every block has arrived.
 template <bool kMMA>
 __global__ void __launch_bounds__(kThreads) quantize_dynamic_kernel(
     const uint16_t* __restrict__ x, FastDiv kblocks_div, uint32_t total_blocks, int64_t ld, bool dense, uint32_t rows,
@@ -217,21 +235,20 @@ __global__ void __launch_bounds__(kThreads) quantize_dynamic_kernel(
   griddep_wait_and_release();
   const uint32_t lane = threadIdx.x & 31;
   const uint32_t stride = gridDim.x * blockDim.x;
+  unsigned long long epoch = 0;
+  if (threadIdx.x == 0) epoch = ld_acquire_u64(&state[0]) >> 32;
   // Resident: one pass covers the tensor, so the loaded blocks stay in
-  // registers across the barrier and x is read once.
+  // registers across the barrier and x is read once.  Otherwise the blocks
+  // of the last phase-1 iteration stay in registers and phase 2 starts with
+  // them, so only the earlier iterations are read again.
   const bool resident = total_blocks <= stride * kUnroll;
   const uint32_t bidx_first = blockIdx.x * blockDim.x + (threadIdx.x & ~31u);
   BlockSlots sl;
-  uint32_t m = 0;
-  if (resident) {
-    load_blocks(x, kblocks_div, total_blocks, ld, dense, bidx_first, stride, lane, sl);
-    m = amax_bits_of(sl);
-  } else {
-    for (uint32_t bidx0 = bidx_first; bidx0 < total_blocks; bidx0 += stride * kUnroll) {
-      BlockSlots t;
-      load_blocks(x, kblocks_div, total_blocks, ld, dense, bidx0, stride, lane, t);
-      m = max(m, amax_bits_of(t));
-    }
+  uint32_t m = 0, bidx_last = bidx_first;
+  for (uint32_t bidx0 = bidx_first; bidx0 < total_blocks || bidx0 == bidx_first; bidx0 += stride * kUnroll) {
+    load_blocks(x, kblocks_div, total_blocks, ld, dense, bidx0, stride, lane, sl);
+    m = max(m, amax_bits_of(sl));
+    bidx_last = bidx0;
   }
   m = __reduce_max_sync(0xffffffffu, m);
   __shared__ uint32_t warp_max[kThreads / 32];
@@ -243,23 +260,25 @@ __global__ void __launch_bounds__(kThreads) quantize_dynamic_kernel(
     m = threadIdx.x < kThreads / 32 ? warp_max[threadIdx.x] : 0u;
     m = __reduce_max_sync(0xffffffffu, m);
     if (threadIdx.x == 0) {
-      const unsigned long long epoch = ld_acquire_u64(&state[0]) >> 32;
-      atomicMax(&state[1], (epoch << 32) | m);
-      __threadfence();
-      const unsigned long long old = atomicAdd(&state[0], 1ull);
+      red_max_u64(&state[1], (epoch << 32) | m);
+      const unsigned long long old = atom_add_acq_rel_u64(&state[0], 1ull);
       int ok = (old >> 32) == epoch;
-      if (ok && static_cast<uint32_t>(old) == gridDim.x - 1) {
-        __threadfence();
-        atomicExch(&state[0], (epoch + 1) << 32);
+      uint32_t amax_bits = 0;
+      if (ok && static_cast<uint32_t>(old & 0xFFFFu) == gridDim.x - 1) {
+        const unsigned long long a = ld_acquire_u64(&state[1]);
+        ok = (a >> 32) == epoch;
+        amax_bits = static_cast<uint32_t>(a) & 0xFFFFu;
+        if (ok) st_release_u64(&state[0], ((epoch + 1) << 32) | (static_cast<unsigned long long>(amax_bits) << 16));
       } else if (ok) {
         const uint64_t t0 = globaltimer_ns();
-        for (uint32_t it = 0; (ld_acquire_u64(&state[0]) >> 32) == epoch; ++it)
+        unsigned long long v;
+        for (uint32_t it = 0; ((v = ld_acquire_u64(&state[0])) >> 32) == epoch; ++it)
           if ((it & 63u) == 63u && globaltimer_ns() - t0 > kWaitLimitNs) { ok = 0; break; }
+        if (ok && (v >> 32) != epoch + 1) ok = 0;
+        amax_bits = static_cast<uint32_t>(v >> 16) & 0xFFFFu;
       }
-      const unsigned long long a = ld_acquire_u64(&state[1]);
-      if (ok && (a >> 32) != epoch) ok = 0;
       if (!ok) set_status(status, NVFP4_ERR_TIMEOUT);
-      s_amax = static_cast<uint32_t>(a) & 0xFFFFu;
+      s_amax = amax_bits;
       s_ok = ok;
     }
   }
@@ -267,15 +286,18 @@ __global__ void __launch_bounds__(kThreads) quantize_dynamic_kernel(
   if (!s_ok) return;
   const float amax = __uint_as_float(s_amax << 16);
   const float g = amax > 0.0f ? __fdiv_rn(amax, 2688.0f) : 1.0f;
+  const float six_g = __fmul_rn(6.0f, g);
   if (blockIdx.x == 0 && threadIdx.x == 0) *g_out = g;
-  if (resident) {
-    if (bidx_first < total_blocks)
-      quantize_loaded<kMMA>(sl, total_blocks, kblocks_div.d, bidx_first, stride, lane, g, __fmul_rn(6.0f, g), true,
-                            codes, scales);
-    if (kMMA) zero_scale_padding(rows, kblocks_div.d, scales);
-  } else {
-    quantize_blocks<kMMA>(x, kblocks_div, total_blocks, ld, dense, rows, g, true, codes, scales);
+  if (bidx_last < total_blocks)
+    quantize_loaded<kMMA>(sl, total_blocks, kblocks_div.d, bidx_last, stride, lane, g, six_g, true, codes, scales);
+  if (!resident) {
+    for (uint32_t bidx0 = bidx_first; bidx0 < bidx_last; bidx0 += stride * kUnroll) {
+      BlockSlots t;
+      load_blocks(x, kblocks_div, total_blocks, ld, dense, bidx0, stride, lane, t);
+      quantize_loaded<kMMA>(t, total_blocks, kblocks_div.d, bidx0, stride, lane, g, six_g, true, codes, scales);
+    }
   }
+  if (kMMA) zero_scale_padding(rows, kblocks_div.d, scales);
 }
 
 // Blocks of quantize_dynamic_kernel that fit on the device at once (a
@@ -424,6 +446,7 @@ NVFP4_API nvfp4_status nvfp4_quantize_dynamic(const void* x_bf16, int64_t rows, 
   // barrier when one pass covers it.
   int grid = grid_for(total_blocks, kThreads * kUnroll);
   if (grid > cap) grid = cap;
+  if (grid > 0xFFFF) grid = 0xFFFF;  // the barrier counts arrivals in 16 bits
   // Cooperative: every block is resident at once, so the grid barrier can
   // complete.  (Without programmatic serialization: measured no faster.)
   cudaLaunchConfig_t cfg = {};
