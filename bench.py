@@ -43,11 +43,11 @@ CSRC = os.path.join(ROOT, "paper_2606_15682_gb300", "csrc")
 # same kernel and shape (commands in profiles/).  Each entry holds only while the kernel sources
 # hash to the value they had at capture time; otherwise the line reports traffic = null.
 NCU_TRAFFIC = {
-    "gemm": {"bytes": 17295872 + 13333760, "sources": ("gemm.cu", "common.cuh"), "sha": "8d4a03ae983bc8a0",
+    "gemm": {"bytes": 17293824 + 12077824, "sources": ("gemm.cu", "common.cuh"), "sha": "df869ea01e6926f0",
              "shape": (2048, 17920, 1536),
              "profile": "profiles/gemm_qwen1.5b_prefill_gate_up_m2048_n17920_k1536.md"},
-    "attention": {"bytes": 1208752896 + 22476032, "sources": ("attention.cu", "common.cuh"),
-                  "sha": "e70533c1c9c6b86b", "shape": (64, 16384),
+    "attention": {"bytes": 1208717312 + 22197760, "sources": ("attention.cu", "common.cuh"),
+                  "sha": "4dda26a3f17c55dd", "shape": (64, 16384),
                   "profile": "profiles/attention_qwen14b_decode_b64_t16384.md (attn_partial_kernel)"},
 }
 

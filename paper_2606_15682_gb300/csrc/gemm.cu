@@ -469,10 +469,21 @@ __device__ __forceinline__ void mbar_arrive_cluster_relaxed(uint64_t* bar, uint3
   asm volatile("mbarrier.arrive.relaxed.cluster.shared::cluster.b64 _, [%0];" ::"r"(remote) : "memory");
 }
 
-template <int STAGES_>
+// RES_: the W-resident form for 1024 <= K <= 1536.  A pair walks a run of
+// consecutive units that share one W tile.  The run's first unit loads the W
+// tile's codes for the whole K into shared memory and copies its block scales
+// for the whole K into TMEM (8 columns per 64-deep k group); the run's later
+// units stream only A and its scales (18 KB per k-block and CTA instead of
+// 38 KB).  The A ring keeps 4 stages.
+template <int STAGES_, bool RES_ = false>
 struct PairCfg {
   static constexpr int BN = 256;                 // MMA N (both halves of the pair)
   static constexpr int kStages = STAGES_;
+  static constexpr bool kRes = RES_;
+  static constexpr int kResKblocks = 6;                          // K <= 1536 in the resident form
+  static constexpr int kBTiles = kRes ? kResKblocks : kStages;   // W tiles held in shared memory
+  static constexpr uint32_t kSfbResCol = BN;                     // resident W scales
+  static constexpr uint32_t kSfaResCol = BN + 32 * kResKblocks;  // per-stage A scales, 16 columns each
   static constexpr int kEpiWarps = 8;            // 128 rows x 256 accumulator columns per CTA
   static constexpr int kCopyWarps = NVFP4_GEMM_COPY_WARPS;  // warps issuing the scale copies (1, 2 or 4)
   static constexpr int kThreads = 64 + 32 * kCopyWarps + 32 * kEpiWarps;
@@ -483,11 +494,12 @@ struct PairCfg {
   static constexpr uint32_t kStageBytes = kTileBytesA + kTileBytesB + kSfaBytes + kSfbBytes;
   static constexpr uint32_t kSfCols = 16 + 32;
   static constexpr uint32_t kSfTmemCol = BN;
-  static constexpr size_t kSmemBytes =
-      1024 + kStages * kStageBytes + kEpiWarps * kEpiBufBytes + 512 /*barriers*/;
+  static constexpr size_t kSmemBytes = 1024 + kStages * (kStageBytes - kTileBytesB) + kBTiles * kTileBytesB +
+                                       kEpiWarps * kEpiBufBytes + 512 /*barriers*/;
   static constexpr uint32_t kIdesc = (1u << 7) | (1u << 10) | (static_cast<uint32_t>(BN >> 3) << 17) |
                                      (static_cast<uint32_t>(256 >> 4) << 24);
-  static_assert(kSfTmemCol + kStages * kSfCols <= kTmemCols, "TMEM budget");
+  static_assert(kRes ? kSfaResCol + kStages * 16 <= kTmemCols : kSfTmemCol + kStages * kSfCols <= kTmemCols,
+                "TMEM budget");
   static_assert(kSmemBytes <= 227 * 1024, "shared memory budget");
 };
 
@@ -502,7 +514,7 @@ __global__ void __launch_bounds__(C::kThreads, 1)
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* sA = smem;
   uint8_t* sB = sA + kStages * C::kTileBytesA;
-  uint8_t* sEpi = sB + kStages * C::kTileBytesB;
+  uint8_t* sEpi = sB + C::kBTiles * C::kTileBytesB;
   uint8_t* sSFA = sEpi + C::kEpiWarps * kEpiBufBytes;
   uint8_t* sSFB = sSFA + kStages * C::kSfaBytes;
   uint64_t* full = reinterpret_cast<uint64_t*>(sSFB + kStages * C::kSfbBytes);  // codes landed
@@ -519,11 +531,33 @@ __global__ void __launch_bounds__(C::kThreads, 1)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int kblocks = args.K / BK;
   const int kgroups = args.K / 64;
+  if (C::kRes && (kblocks < kStages || kblocks > C::kResKblocks)) {
+    // Outside the resident form's K range (the host never launches it so):
+    // the whole grid returns before touching any barrier or TMEM.
+    if (blockIdx.x == 0 && threadIdx.x == 0) set_status(args.status, NVFP4_ERR_SHAPE);
+    return;
+  }
   const uint32_t rank = cluster_ctarank();
   const bool leader = rank == 0;
   const int msup = (args.tiles_m + 1) / 2;
   const int total_units = msup * args.tiles_n;
   const int pair_id = blockIdx.x / 2, n_pairs = gridDim.x / 2;
+  // Units of this pair: every n_pairs-th one, or (resident form) a
+  // contiguous run in W-tile-major order, so that consecutive units share nb.
+  const int run = C::kRes ? (total_units + n_pairs - 1) / n_pairs : 0;
+  const int u_first = C::kRes ? pair_id * run : pair_id;
+  const int u_end = C::kRes ? min(total_units, u_first + run) : total_units;
+  const int u_step = C::kRes ? 1 : n_pairs;
+  auto coords = [&](int u, int* ms, int* nb) {
+    if (C::kRes) {
+      // Within a W tile the row super-tiles start at a rotation of nb, so
+      // that the pairs running at the same time read different A tiles.
+      *nb = u / msup;
+      *ms = (u - *nb * msup + *nb) % msup;
+    } else {
+      unit_coords(u, msup, args.tiles_n, ms, nb);
+    }
+  };
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
@@ -566,9 +600,16 @@ __global__ void __launch_bounds__(C::kThreads, 1)
     uint32_t issued_parity[kStages];
     bool issued[kStages];
     for (int s = 0; s < kStages; ++s) issued[s] = false;
-    for (int u = pair_id; u < total_units && !abort_flag; u += n_pairs) {
+    int prev_nb = -1;
+    for (int u = u_first; u < u_end && !abort_flag; u += u_step) {
       int ms, nb;
-      unit_coords(u, msup, args.tiles_n, &ms, &nb);
+      coords(u, &ms, &nb);
+      // W codes and scales: every unit, or (resident form) a run's first.
+      // Resident W tile kb is rewritten only after the MMAs of k-block kb of
+      // the previous unit completed: this stage's empty barrier covers the
+      // MMAs up to kStages k-blocks back, and kblocks >= kStages.
+      const bool load_w = !C::kRes || nb != prev_nb;
+      prev_nb = nb;
       const int mb = min(ms * 2 + static_cast<int>(rank), args.tiles_m - 1);  // a spare CTA redoes the last tile
       // Scale atoms through a [bytes / 256, 256] view: one (128-row tile,
       // k-block) group of four 512-byte atoms is 8 rows of that view.
@@ -577,26 +618,31 @@ __global__ void __launch_bounds__(C::kThreads, 1)
       for (int kb = 0; kb < kblocks; ++kb) {
         if (!mbar_wait_bounded(&empty[stage], phase ^ 1u, &abort_flag)) { fail(); break; }
         uint8_t* a_dst = sA + stage * C::kTileBytesA;
-        uint8_t* b_dst = sB + stage * C::kTileBytesB;
+        uint8_t* b_dst = sB + (C::kRes ? kb : stage) * C::kTileBytesB;
         uint8_t* sfa_dst = sSFA + stage * C::kSfaBytes;
         uint8_t* sfb_dst = sSFB + stage * C::kSfbBytes;
         const int kx = kb * (BK / 2), b_row = nb * BN + static_cast<int>(rank) * 128;
         constexpr uint32_t kSfStage = C::kSfaBytes + C::kSfbBytes;
         if (leader) {
           // Both CTAs' loads land on the leader's barriers.
-          mbar_arrive_expect_tx(&sffull[stage], 2 * kSfStage);
-          mbar_arrive_expect_tx(&full[stage], 2 * (C::kStageBytes - kSfStage));
+          mbar_arrive_expect_tx(&sffull[stage], 2 * (load_w ? kSfStage : C::kSfaBytes));
+          mbar_arrive_expect_tx(&full[stage], 2 * (C::kTileBytesA + (load_w ? C::kTileBytesB : 0u)));
           tma_load_2d(sfa_dst, &tmap_sfa, &sffull[stage], 0, sfa_row + kb * 8);
-          tma_load_2d(sfb_dst, &tmap_sfb, &sffull[stage], 0, sfb_row + kb * 8);
-          tma_load_2d(sfb_dst + C::kSfaBytes, &tmap_sfb, &sffull[stage], 0, sfb_row + kgroups * 2 + kb * 8);
+          if (load_w) {
+            tma_load_2d(sfb_dst, &tmap_sfb, &sffull[stage], 0, sfb_row + kb * 8);
+            tma_load_2d(sfb_dst + C::kSfaBytes, &tmap_sfb, &sffull[stage], 0, sfb_row + kgroups * 2 + kb * 8);
+          }
           tma_load_2d(a_dst, &tmap_a, &full[stage], kx, mb * BM);
-          tma_load_2d(b_dst, &tmap_b, &full[stage], kx, b_row);
+          if (load_w) tma_load_2d(b_dst, &tmap_b, &full[stage], kx, b_row);
         } else {
           tma_load_2d_to_leader(sfa_dst, &tmap_sfa, &sffull[stage], 0, sfa_row + kb * 8);
-          tma_load_2d_to_leader(sfb_dst, &tmap_sfb, &sffull[stage], 0, sfb_row + kb * 8);
-          tma_load_2d_to_leader(sfb_dst + C::kSfaBytes, &tmap_sfb, &sffull[stage], 0, sfb_row + kgroups * 2 + kb * 8);
+          if (load_w) {
+            tma_load_2d_to_leader(sfb_dst, &tmap_sfb, &sffull[stage], 0, sfb_row + kb * 8);
+            tma_load_2d_to_leader(sfb_dst + C::kSfaBytes, &tmap_sfb, &sffull[stage], 0,
+                                  sfb_row + kgroups * 2 + kb * 8);
+          }
           tma_load_2d_to_leader(a_dst, &tmap_a, &full[stage], kx, mb * BM);
-          tma_load_2d_to_leader(b_dst, &tmap_b, &full[stage], kx, b_row);
+          if (load_w) tma_load_2d_to_leader(b_dst, &tmap_b, &full[stage], kx, b_row);
         }
         issued[stage] = true;
         issued_parity[stage] = phase;
@@ -617,7 +663,7 @@ __global__ void __launch_bounds__(C::kThreads, 1)
     uint32_t phase = 0;
     int local = 0;
     const uint32_t sA0 = smem_u32(sA), sB0 = smem_u32(sB);
-    for (int u = pair_id; u < total_units && !abort_flag; u += n_pairs, ++local) {
+    for (int u = u_first; u < u_end && !abort_flag; u += u_step, ++local) {
       if (!mbar_wait_bounded(tempty, (local & 1) ^ 1u, &abort_flag)) { fail(); break; }
       tc_fence_after();
       bool ok = true;
@@ -625,13 +671,13 @@ __global__ void __launch_bounds__(C::kThreads, 1)
         if (!mbar_wait_bounded(&full[stage], phase, &abort_flag) ||
             !mbar_wait_bounded(&sfready[stage], phase, &abort_flag)) { fail(); ok = false; break; }
         tc_fence_after();
-        const uint32_t sfa_col = tmem + C::kSfTmemCol + stage * C::kSfCols;
-        const uint32_t sfb_col = sfa_col + 16;
+        const uint32_t sfa_col = tmem + (C::kRes ? C::kSfaResCol + stage * 16 : C::kSfTmemCol + stage * C::kSfCols);
+        const uint32_t sfb_col = C::kRes ? tmem + C::kSfbResCol + kb * 32 : sfa_col + 16;
+        const uint32_t b_tile = sB0 + (C::kRes ? kb : stage) * C::kTileBytesB;
 #pragma unroll
         for (int kk = 0; kk < 4; ++kk)
-          mma_fp4_pair(tmem, desc_sw128(sA0 + stage * C::kTileBytesA + kk * 32),
-                       desc_sw128(sB0 + stage * C::kTileBytesB + kk * 32), C::kIdesc, sfa_col + kk * 4,
-                       sfb_col + kk * 8, (kb | kk) != 0);
+          mma_fp4_pair(tmem, desc_sw128(sA0 + stage * C::kTileBytesA + kk * 32), desc_sw128(b_tile + kk * 32),
+                       C::kIdesc, sfa_col + kk * 4, sfb_col + kk * 8, (kb | kk) != 0);
         tc_commit_pair(&empty[stage], 0x3);
         if (++stage == kStages) { stage = 0; phase ^= 1u; }
       }
@@ -649,21 +695,32 @@ __global__ void __launch_bounds__(C::kThreads, 1)
     int stage = 0;
     uint32_t phase = 0;
     const uint32_t sSFA0 = smem_u32(sSFA), sSFB0 = smem_u32(sSFB);
-    for (int u = pair_id; u < total_units && !abort_flag; u += n_pairs) {
+    int prev_nb = -1;
+    for (int u = u_first; u < u_end && !abort_flag; u += u_step) {
       bool ok = true;
+      int ms, nb;
+      coords(u, &ms, &nb);
+      // Resident form: a run's first unit copies the W scales for the whole
+      // K.  The copy of k-block kb's columns waited (through the producer's
+      // empty barrier) for the MMAs of the previous unit's k-block kb.
+      const bool copy_w = !C::kRes || nb != prev_nb;
+      prev_nb = nb;
       for (int kb = 0; kb < kblocks; ++kb) {
         if (!mbar_wait_bounded(&sffull[stage], phase, &abort_flag)) { fail(); ok = false; break; }
         {
           tc_fence_after();
-          const uint32_t sfa_col = tmem + C::kSfTmemCol + stage * C::kSfCols;
-          const uint32_t sfb_col = sfa_col + 16;
+          const uint32_t sfa_col =
+              tmem + (C::kRes ? C::kSfaResCol + stage * 16 : C::kSfTmemCol + stage * C::kSfCols);
+          const uint32_t sfb_col = C::kRes ? tmem + C::kSfbResCol + kb * 32 : sfa_col + 16;
 #pragma unroll
           for (int kk = kk0; kk < kk0 + kPerWarp; ++kk) {
             copy_sf_to_tmem_pair(sfa_col + kk * 4, desc_sf(sSFA0 + stage * C::kSfaBytes + kk * 512));
+            if (copy_w) {
 #pragma unroll
-            for (int j = 0; j < 2; ++j)
-              copy_sf_to_tmem_pair(sfb_col + kk * 8 + j * 4,
-                                   desc_sf(sSFB0 + stage * C::kSfbBytes + j * C::kSfaBytes + kk * 512));
+              for (int j = 0; j < 2; ++j)
+                copy_sf_to_tmem_pair(sfb_col + kk * 8 + j * 4,
+                                     desc_sf(sSFB0 + stage * C::kSfbBytes + j * C::kSfaBytes + kk * 512));
+            }
           }
           tc_commit_pair(&sfready[stage], 0x1);
         }
@@ -691,9 +748,9 @@ __global__ void __launch_bounds__(C::kThreads, 1)
     const uint32_t q_cols = static_cast<uint32_t>(args.N) >> 1;  // SwiGLU outputs per row
     const uint32_t q_kgroups = q_cols >> 6;
     int local = 0;
-    for (int u = pair_id; u < total_units; u += n_pairs, ++local) {
+    for (int u = u_first; u < u_end; u += u_step, ++local) {
       int ms, nb;
-      unit_coords(u, msup, args.tiles_n, &ms, &nb);
+      coords(u, &ms, &nb);
       const int mb = ms * 2 + static_cast<int>(rank);  // mb >= tiles_m: nothing is stored
       int ok = 1;
       if (lane == 0) {
@@ -753,9 +810,9 @@ __global__ void __launch_bounds__(C::kThreads, 1)
     const uint32_t buf = smem_u32(buf_ptr);
     const float scale = __fmul_rn(__ldg(args.ga), __ldg(args.gb));
     int local = 0;
-    for (int u = pair_id; u < total_units; u += n_pairs, ++local) {
+    for (int u = u_first; u < u_end; u += u_step, ++local) {
       int ms, nb;
-      unit_coords(u, msup, args.tiles_n, &ms, &nb);
+      coords(u, &ms, &nb);
       const int mb = ms * 2 + static_cast<int>(rank);  // mb >= tiles_m: nothing is stored
       int ok = 1;
       if (lane == 0) {
@@ -1038,6 +1095,23 @@ nvfp4_status launch_pair(const uint8_t* a_codes, const uint8_t* a_scales, const 
 #ifndef NVFP4_GEMM_PAIR
 #define NVFP4_GEMM_PAIR 1  // 0: never use the CTA-pair kernel
 #endif
+#ifndef NVFP4_GEMM_RES
+#define NVFP4_GEMM_RES 1  // 0: never use the W-resident form
+#endif
+
+using PairRes = PairCfg<4, true>;
+
+// The W-resident form pays when a pair gets runs of two or more units (more
+// units than pairs); K must fit its shared-memory and TMEM budget, and its
+// copy-after-read order needs at least as many k-blocks as ring stages.
+// Measured on GB300 (graph-replayed, L2 flushed): gate_up of the 1.5B
+// prefill (2048 x 17920 x 1536) 38.0 -> 35.7 us; with 4 k-blocks
+// (8192 x 5120 x 1024) it was slower, so it starts at 5.
+bool use_w_resident(int64_t pair_units, int64_t K, int pairs) {
+  const int64_t kblocks = K / BK;
+  return NVFP4_GEMM_RES && pairs > 0 && pair_units > pairs && kblocks >= PairRes::kStages + 1 &&
+         kblocks <= PairRes::kResKblocks;
+}
 
 }  // namespace
 }  // namespace nvfp4
@@ -1064,9 +1138,13 @@ NVFP4_API nvfp4_status nvfp4_linear(const uint8_t* a_codes, const uint8_t* a_sca
   // over more SMs (measured faster at M = 256 with N = 5120 or 7168, slower
   // with N = 27648).
   using Pair = PairCfg<NVFP4_GEMM_PAIR_STAGES>;
-  if (NVFP4_GEMM_PAIR && N % 256 == 0 && tiles_m >= 2 &&
-      2 * ((tiles_m + 1) / 2) * (N / 256) >= resident_pairs<Pair, false>())
-    return launch_pair<Pair>(a_codes, a_scales, g_a, w_codes, w_scales, g_w, M, N, K, out_bf16, ldo, s);
+  if (NVFP4_GEMM_PAIR && N % 256 == 0 && tiles_m >= 2) {
+    const int64_t pair_units = ((tiles_m + 1) / 2) * (N / 256);
+    if (use_w_resident(pair_units, K, resident_pairs<PairRes, false>()))
+      return launch_pair<PairRes>(a_codes, a_scales, g_a, w_codes, w_scales, g_w, M, N, K, out_bf16, ldo, s);
+    if (2 * pair_units >= resident_pairs<Pair, false>())
+      return launch_pair<Pair>(a_codes, a_scales, g_a, w_codes, w_scales, g_w, M, N, K, out_bf16, ldo, s);
+  }
   // Single CTAs: BN = 128 (measured faster than 256 at M <= 256 on GB300).
   const int bn = NVFP4_GEMM_BN ? NVFP4_GEMM_BN : 128;
 #define NVFP4_LAUNCH(BN_, ST_, CM_) \
@@ -1097,6 +1175,10 @@ NVFP4_API nvfp4_status nvfp4_linear_swiglu_quantize(const uint8_t* a_codes, cons
   extra.q_codes = out_codes;
   extra.q_scales = out_scales;
   extra.g_out = g_out;
+  const int64_t pair_units = ((M + 2 * BM - 1) / (2 * BM)) * (2 * I / 256);
+  if (use_w_resident(pair_units, K, resident_pairs<PairRes, true>()))
+    return launch_pair<PairRes, true>(a_codes, a_scales, g_a, w_codes, w_scales, g_w, M, 2 * I, K, nullptr, 0,
+                                      static_cast<cudaStream_t>(stream), &extra);
   return launch_pair<PairCfg<NVFP4_GEMM_PAIR_STAGES>, true>(a_codes, a_scales, g_a, w_codes, w_scales, g_w, M, 2 * I,
                                                            K, nullptr, 0, static_cast<cudaStream_t>(stream), &extra);
 }

@@ -52,7 +52,9 @@ def run_linear(N, a_codes, a_scales_rm, g_a, w_codes, w_scales_rm, g_w, M, Nn, K
                                     # CTA-pair path (enough 256 x 256 tiles to occupy the pairs):
                                     # M tails with a spare CTA, odd super-tile counts, one-row tail
                                     (256, 10240, 512), (300, 10240, 1024), (640, 5120, 768), (129, 12800, 256),
-                                    # more 256 x 256 tiles than pairs: a second round of tiles
+                                    # more 256 x 256 tiles than pairs: a second round of tiles (K = 1024), and
+                                    # the W-resident form (K = 1280, 1536): runs of two units per pair, an M
+                                    # tail, runs that cross a W tile
                                     (512, 10240, 1024), (300, 15360, 1536), (640, 7680, 1280)])
 def test_random_codes(N, M, Nn, K):
     gen = torch.Generator().manual_seed(M * 1000 + Nn * 10 + K)
