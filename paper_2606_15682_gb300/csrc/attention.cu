@@ -71,25 +71,33 @@ __device__ __forceinline__ void e2m1x8_to_f16x2(uint32_t w, uint32_t h[4]) {
       : "r"(w));
 }
 
-// Four bytes of E1M2 nibbles (two's complement n, value n/2) -> four f16x2
-// holding n (low nibble -> low half); the 1/2 goes into the block scale.  The
-// nibble XOR 8 in the low mantissa bits of 1024.0 (0x6400) reads as 1032 + n.
+// E1M2 nibbles (two's complement n, value n/2) decode to f16 n; the 1/2 goes
+// into the block scale.  The nibble XOR 8 in the low mantissa bits of 1024.0
+// (0x6400) reads as 1032 + n, and one f16x2 subtraction of 1032 leaves n.
 __device__ __forceinline__ uint32_t hsub2(uint32_t a, uint32_t b) {
   uint32_t d;
   asm("sub.rn.f16x2 %0, %1, %2;" : "=r"(d) : "r"(a), "r"(b));
   return d;
 }
-__device__ __forceinline__ void e1m2x8_to_f16x2(uint32_t w, uint32_t h[4]) {
+// K side: the eight nibbles n0..n7 of w (n0 lowest) -> h[i] = (n_i, n_{i+4}),
+// one mask-and-xor and one subtraction per pair.  The channel order inside
+// each group of eight differs from the E2M1 path; the queries are paired the
+// same way, so every logit is the same sum.
+__device__ __forceinline__ void e1m2x8_to_f16x2_paired(uint32_t w, uint32_t h[4]) {
 #pragma unroll
-  for (int j = 0; j < 4; ++j) {
-    const uint32_t x = w >> (8 * j);
-    h[j] = hsub2(((x & 0xFu) | ((x & 0xF0u) << 12)) ^ 0x64086408u, 0x64086408u);
-  }
+  for (int i = 0; i < 4; ++i) h[i] = hsub2(((w >> (4 * i)) & 0x000F000Fu) ^ 0x64086408u, 0x64086408u);
+}
+// V side: byte k of two tokens' words a and b -> lo = (a, b) of the byte's
+// low-nibble channel, hi = (a, b) of its high-nibble channel.
+__device__ __forceinline__ void e1m2_token_pair(uint32_t wa, uint32_t wb, int k, uint32_t* lo, uint32_t* hi) {
+  const uint32_t x = __byte_perm(wa, wb, 0x4400u + 0x1111u * k);  // bytes: a_k, a_k, b_k, b_k
+  *lo = hsub2((x & 0x000F000Fu) ^ 0x64086408u, 0x64086408u);
+  *hi = hsub2(((x >> 4) & 0x000F000Fu) ^ 0x64086408u, 0x64086408u);
 }
 
 template <bool kE1M2>
 __device__ __forceinline__ void decode8(uint32_t w, uint32_t h[4]) {
-  if (kE1M2) e1m2x8_to_f16x2(w, h);
+  if (kE1M2) e1m2x8_to_f16x2_paired(w, h);
   else e2m1x8_to_f16x2(w, h);
 }
 
@@ -268,7 +276,14 @@ __global__ void __launch_bounds__(kThreads, NVFP4_ATTN_MIN_CTAS) attn_partial_ke
     const float qscale = ldexpf(1.0f, -qexp);
     uint32_t qf[16];
 #pragma unroll
-    for (int i = 0; i < 16; ++i) qf[i] = f32x2_to_f16x2(qv[2 * i] * qscale, qv[2 * i + 1] * qscale);
+    for (int j = 0; j < 8; ++j) {
+      // k-step j = 2w + h.  E2M1 keys hold channel pairs (4j, 4j+1), (4j+2, 4j+3);
+      // E1M2 keys (decoded in pairs i, i+4 of each word) hold (8w+2h, 8w+2h+4), (8w+2h+1, 8w+2h+5).
+      const int c0 = kE1M2 ? 8 * (j >> 1) + 2 * (j & 1) : 4 * j;
+      const int c1 = kE1M2 ? c0 + 4 : c0 + 1, c2 = kE1M2 ? c0 + 1 : c0 + 2, c3 = kE1M2 ? c0 + 5 : c0 + 3;
+      qf[2 * j] = f32x2_to_f16x2(qv[c0] * qscale, qv[c1] * qscale);
+      qf[2 * j + 1] = f32x2_to_f16x2(qv[c2] * qscale, qv[c3] * qscale);
+    }
     const float mult_self = p.logit_mult / qscale;
     const float mult0 = __shfl_sync(0xffffffffu, mult_self, (2 * t) * 4);
     const float mult1 = __shfl_sync(0xffffffffu, mult_self, (2 * t + 1) * 4);
@@ -378,16 +393,24 @@ __global__ void __launch_bounds__(kThreads, NVFP4_ATTN_MIN_CTAS) attn_partial_ke
         for (int half = 0; half < 2; ++half) {  // bytes 0-3, then 4-7 of each token's 8-byte slice
           const uint32_t wa = half ? va.y : va.x, wb = half ? vb.y : vb.x;
           const uint32_t wc = half ? vc.y : vc.x, wd = half ? vd.y : vd.x;
-          // Pair the same channel of two tokens in one e2m1x2 byte (first token in the low nibble).
-          const uint32_t lo_ab = (wa & 0x0F0F0F0Fu) | ((wb << 4) & 0xF0F0F0F0u);
-          const uint32_t hi_ab = ((wa >> 4) & 0x0F0F0F0Fu) | (wb & 0xF0F0F0F0u);
-          const uint32_t lo_cd = (wc & 0x0F0F0F0Fu) | ((wd << 4) & 0xF0F0F0F0u);
-          const uint32_t hi_cd = ((wc >> 4) & 0x0F0F0F0Fu) | (wd & 0xF0F0F0F0u);
           uint32_t f_lo_ab[4], f_hi_ab[4], f_lo_cd[4], f_hi_cd[4];
-          decode8<kE1M2>(lo_ab, f_lo_ab);
-          decode8<kE1M2>(hi_ab, f_hi_ab);
-          decode8<kE1M2>(lo_cd, f_lo_cd);
-          decode8<kE1M2>(hi_cd, f_hi_cd);
+          if (kE1M2) {
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+              e1m2_token_pair(wa, wb, k, &f_lo_ab[k], &f_hi_ab[k]);
+              e1m2_token_pair(wc, wd, k, &f_lo_cd[k], &f_hi_cd[k]);
+            }
+          } else {
+            // Pair the same channel of two tokens in one e2m1x2 byte (first token in the low nibble).
+            const uint32_t lo_ab = (wa & 0x0F0F0F0Fu) | ((wb << 4) & 0xF0F0F0F0u);
+            const uint32_t hi_ab = ((wa >> 4) & 0x0F0F0F0Fu) | (wb & 0xF0F0F0F0u);
+            const uint32_t lo_cd = (wc & 0x0F0F0F0Fu) | ((wd << 4) & 0xF0F0F0F0u);
+            const uint32_t hi_cd = ((wc >> 4) & 0x0F0F0F0Fu) | (wd & 0xF0F0F0F0u);
+            e2m1x8_to_f16x2(lo_ab, f_lo_ab);
+            e2m1x8_to_f16x2(hi_ab, f_hi_ab);
+            e2m1x8_to_f16x2(lo_cd, f_lo_cd);
+            e2m1x8_to_f16x2(hi_cd, f_hi_cd);
+          }
 #pragma unroll
           for (int k = 0; k < 4; ++k) {
             const uint32_t a[4] = {hmul2(f_lo_ab[k], vs01), hmul2(f_hi_ab[k], vs01), hmul2(f_lo_cd[k], vs89),
