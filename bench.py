@@ -36,6 +36,9 @@ sys.path.insert(0, ROOT)
 
 GEMM_WL = "qwen1.5b_prefill_linears_m2048"
 ATTN_WL = "qwen14b_decode_attention_b64_t16384"
+# Reported beside the headline (same step form, graph-replayed, L2 flushed): the single linear, the
+# decode-batch linears with their K/V append, and the 32B prefill layer chain.
+OTHER_LINEAR_WLS = ("w4a4_linear_m16_k1536_n1536", "qwen14b_decode_linears_m256", "qwen32b_prefill_linears_m8192")
 METRIC = "NVFP4 GEMM TFLOP/s & FP4-KV decode-attn HBM GB/s vs GB300 roofline"
 FP4_OVER_BF16 = 13.5 / 2.25  # nominal dense FP4 / BF16 tensor ratio of GB300
 CSRC = os.path.join(ROOT, "paper_2606_15682_gb300", "csrc")
@@ -172,35 +175,39 @@ def run_ours(args, rank, world):
     sampler.start()
 
     # ---------------- GEMM step: prefill linears with on-the-fly activation quantization
-    w = synth.WORKLOADS[GEMM_WL]
-    M = w["M"]
-    layers = []
-    flops = 0
-    for name, (Nn, K) in w["linears"].items():
-        a, W = synth.linear_inputs(GEMM_WL, name, device=dev)
-        gw = torch.empty(1, dtype=torch.float32, device=dev)
-        wc = torch.empty(Nn, K // 2, dtype=torch.uint8, device=dev)
-        ws = torch.empty(N.nvfp4_scales_bytes(Nn, K, N.SCALES_MMA), dtype=torch.uint8, device=dev)
-        N.nvfp4_tensor_scale(W, gw)
-        N.nvfp4_quantize(W, gw, wc, ws, N.SCALES_MMA)
-        del W
-        L = dict(name=name, N=Nn, K=K, a=a, wc=wc, ws=ws, gw=gw,
-                 ga=torch.empty(1, dtype=torch.float32, device=dev),
-                 qstate=torch.zeros(N.DYNAMIC_STATE_BYTES, dtype=torch.uint8, device=dev),
-                 ac=torch.empty(M, K // 2, dtype=torch.uint8, device=dev),
-                 asf=torch.empty(N.nvfp4_scales_bytes(M, K, N.SCALES_MMA), dtype=torch.uint8, device=dev),
-                 out=torch.empty(M, Nn, dtype=torch.bfloat16, device=dev),
-                 ev=[torch.cuda.Event(enable_timing=True) for _ in range(2)])
-        layers.append(L)
-        flops += 2 * M * Nn * K
-    torch.cuda.synchronize()
+    def build_layers(wl):
+        """The workload's linears: bf16 activations, weights quantized once (MMA scales)."""
+        Mw = synth.WORKLOADS[wl]["M"]
+        out_layers, out_flops = [], 0
+        for name, (Nn, K) in synth.WORKLOADS[wl]["linears"].items():
+            a, W = synth.linear_inputs(wl, name, device=dev)
+            gw = torch.empty(1, dtype=torch.float32, device=dev)
+            wc = torch.empty(Nn, K // 2, dtype=torch.uint8, device=dev)
+            ws = torch.empty(N.nvfp4_scales_bytes(Nn, K, N.SCALES_MMA), dtype=torch.uint8, device=dev)
+            N.nvfp4_tensor_scale(W, gw)
+            N.nvfp4_quantize(W, gw, wc, ws, N.SCALES_MMA)
+            del W
+            out_layers.append(dict(name=name, N=Nn, K=K, a=a, wc=wc, ws=ws, gw=gw,
+                                   ga=torch.empty(1, dtype=torch.float32, device=dev),
+                                   qstate=torch.zeros(N.DYNAMIC_STATE_BYTES, dtype=torch.uint8, device=dev),
+                                   ac=torch.empty(Mw, K // 2, dtype=torch.uint8, device=dev),
+                                   asf=torch.empty(N.nvfp4_scales_bytes(Mw, K, N.SCALES_MMA), dtype=torch.uint8,
+                                                   device=dev),
+                                   out=torch.empty(Mw, Nn, dtype=torch.bfloat16, device=dev),
+                                   ev=[torch.cuda.Event(enable_timing=True) for _ in range(2)]))
+            out_flops += 2 * Mw * Nn * K
+        torch.cuda.synchronize()
+        return Mw, out_layers, out_flops
 
-    def gemm_step(record_gemm_events):
-        for L in layers:
+    M, layers, flops = build_layers(GEMM_WL)
+
+    def gemm_step(record_gemm_events, layer_list=None, Mw=None):
+        for L in (layers if layer_list is None else layer_list):
             N.nvfp4_quantize_dynamic(L["a"], L["qstate"], L["ga"], L["ac"], L["asf"], N.SCALES_MMA)
             if record_gemm_events:
                 L["ev"][0].record()
-            N.nvfp4_linear(L["ac"], L["asf"], L["ga"], L["wc"], L["ws"], L["gw"], L["out"], M, L["N"], L["K"])
+            N.nvfp4_linear(L["ac"], L["asf"], L["ga"], L["wc"], L["ws"], L["gw"], L["out"], M if Mw is None else Mw,
+                           L["N"], L["K"])
             if record_gemm_events:
                 L["ev"][1].record()
 
@@ -289,6 +296,77 @@ def run_ours(args, rank, world):
 
     e2e_ms = timed_loop(e2e_step, max(3, min(args.steps, 50)), args.warmup)
 
+    # ---------------- the other linear workloads (reported beside the headline, not in it)
+    def gemm_bytes(Mm, Nn, K):
+        # Algorithmic bytes: codes 0.5 B/elem, scales 1/16 B/elem, bf16 output 2 B/elem, each operand once.
+        return Mm * K * (0.5 + 1 / 16) + Nn * K * (0.5 + 1 / 16) + Mm * Nn * 2
+
+    fp4_peak = peaks["bf16_tflops"] * FP4_OVER_BF16
+
+    def graph_of(fn):
+        with torch.cuda.stream(stream):
+            fn()
+            stream.synchronize()
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, stream=stream):
+                fn()
+        torch.cuda.synchronize()
+        return g
+
+    def roofline_of(flop, byt, ms):
+        s_ = ms * 1e-3
+        t_mem, t_cmp = byt / (peaks["hbm_gbs"] * 1e9), flop / (fp4_peak * 1e12)
+        if t_cmp >= t_mem:
+            return {"bound": "tensor", "achieved": flop / s_ / 1e12, "peak": fp4_peak, "unit": "TFLOP/s",
+                    "frac": flop / s_ / 1e12 / fp4_peak}
+        return {"bound": "hbm", "achieved": byt / s_ / 1e9, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                "frac": byt / s_ / 1e9 / peaks["hbm_gbs"]}
+
+    other_steps = min(args.steps, 10)
+    other = {}
+    for wl in OTHER_LINEAR_WLS:
+        Mw, lw, fw = build_layers(wl)
+        g = graph_of(lambda lw=lw, Mw=Mw: gemm_step(False, lw, Mw))
+        ms_w = statistics.mean(timed_loop(g.replay, other_steps, args.warmup))
+        per = {}
+        with torch.cuda.stream(stream):
+            for _ in range(3):
+                flush_buf.zero_()
+                torch.cuda._sleep(2_000_000)
+                gemm_step(True, lw, Mw)
+                stream.synchronize()
+                for L in lw:
+                    per.setdefault(L["name"], []).append(L["ev"][0].elapsed_time(L["ev"][1]))
+        byt = sum(gemm_bytes(Mw, L["N"], L["K"]) for L in lw)
+        entry = {"step": "per linear: tensor scale + quantize activation (one launch) + NVFP4 GEMM",
+                 "ms_per_step": ms_w, "tflops": fw / (ms_w * 1e-3) / 1e12,
+                 "gemm_us": {k: 1e3 * statistics.median(v) for k, v in per.items()},
+                 "gemm_roofline": {k: roofline_of(2 * Mw * L["N"] * L["K"], gemm_bytes(Mw, L["N"], L["K"]),
+                                                  statistics.median(per[L["name"]])) for k, L in
+                                   ((L["name"], L) for L in lw)},
+                 "algorithmic_gemm_bytes": byt}
+        kva = synth.WORKLOADS[wl].get("kv_append")
+        if kva:
+            # One new token for each of n_new sequences, K and V quantized and appended.
+            n_new, hk = kva["n_new"], kva["num_kv_heads"]
+            gen = torch.Generator(device=dev)
+            gen.manual_seed(synth.seed_for(wl, "kv_append") % (1 << 62))
+            kn = torch.randn(n_new, hk, 128, generator=gen, device=dev).to(torch.bfloat16)
+            vn = torch.randn(n_new, hk, 128, generator=gen, device=dev).to(torch.bfloat16)
+            c3_cache = N.KVCache(n_new, hk, 16, float(kn.float().abs().max()) / 2688,
+                                 float(vn.float().abs().max()) / 2688, device=dev)
+            seq_a = torch.arange(n_new, dtype=torch.int32, device=dev)
+            pos_a = torch.full((n_new,), 7, dtype=torch.int32, device=dev)
+            ga_ = graph_of(lambda: N.kv_append_nvfp4(c3_cache, kn, vn, seq_a, pos_a))
+            ms_a = statistics.mean(timed_loop(ga_.replay, other_steps, args.warmup))
+            a_bytes = n_new * hk * 2 * (256 + 72)
+            entry["kv_append"] = {"rows": n_new * hk, "us": 1e3 * ms_a, "algorithmic_bytes": a_bytes,
+                                  "gbs": a_bytes / (ms_a * 1e-3) / 1e9}
+            del c3_cache, kn, vn
+        other[wl] = entry
+        del lw, g
+        torch.cuda.empty_cache()
+
     # ---------------- decode attention over the NVFP4 cache
     aw = synth.WORKLOADS[ATTN_WL]
     Bq, hq, hkv, T = aw["batch"], aw["num_q_heads"], aw["num_kv_heads"], aw["context"]
@@ -356,10 +434,6 @@ def run_ours(args, rank, world):
     ms_step, ms_e2e, ms_attn_step, ms_attn_kernel = reduce_max_over_ranks(
         [ms_step, ms_e2e, ms_attn_step, ms_attn_kernel], world)
 
-    # Algorithmic bytes: codes 0.5 B/elem, scales 1/16 B/elem, bf16 output 2 B/elem, each operand once.
-    def gemm_bytes(Mm, Nn, K):
-        return Mm * K * (0.5 + 1 / 16) + Nn * K * (0.5 + 1 / 16) + Mm * Nn * 2
-    fp4_peak = peaks["bf16_tflops"] * FP4_OVER_BF16
     dom = max(layers, key=lambda L: gemm_mean[L["name"]])
     d_flops = 2 * M * dom["N"] * dom["K"]
     d_bytes = gemm_bytes(M, dom["N"], dom["K"])
@@ -412,6 +486,7 @@ def run_ours(args, rank, world):
                          "kernel": "attn_partial_kernel + attn_combine_kernel (one decode_attention_nvfp4 call)"},
             "gpu_launches": attn_launches * args.steps,
         },
+        "other_workloads": other,
         "clocks": sampler.summary(),
     }
     if rank == 0 and not args.no_cpu_baseline:
