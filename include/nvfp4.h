@@ -303,6 +303,27 @@ nvfp4_status decode_attention_nvfp4(const nvfp4_kv_cache* cache, const void* q_b
                                     void* workspace, size_t workspace_bytes, void* stream);
 
 /*
+ * Decode attention whose output is written as the output projection's NVFP4
+ * A operand (every linear of the layer, the o projection included, runs
+ * W4A4: Appendix D.1).  The same attention as decode_attention_nvfp4; its
+ * bf16 output o, viewed as the [batch, num_q_heads * 128] matrix, is then
+ * quantized with the static tensor scale g_out by the recipe of
+ * nvfp4_quantize (MMA scale layout).  codes and scales are bit-identical to
+ * decode_attention_nvfp4 followed by nvfp4_quantize(o, g_out, MMA layout);
+ * the bf16 o itself is never stored.
+ *   g_out      : device float, static scale of o (e.g. calibrated).
+ *   out_codes  : [batch, num_q_heads * 64] bytes, 16-B aligned.
+ *   out_scales : nvfp4_scales_bytes(batch, num_q_heads * 128, NVFP4_SCALES_MMA)
+ *                bytes, 4-B aligned; padding rows are written as zeros.
+ *   workspace, errors: as decode_attention_nvfp4.  g_out <= 0 or non-finite:
+ *   zero codes and scales, INVALID_ARG set on the device.
+ */
+nvfp4_status decode_attention_nvfp4_quantize(const nvfp4_kv_cache* cache, const void* q_bf16,
+                                             int32_t num_q_heads, float softmax_scale, const float* g_out,
+                                             uint8_t* out_codes, uint8_t* out_scales, void* workspace,
+                                             size_t workspace_bytes, void* stream);
+
+/*
  * Decode attention without a caller workspace (no counterpart in the paper).
  *
  * Same computation and arguments as decode_attention_nvfp4, but the split-KV

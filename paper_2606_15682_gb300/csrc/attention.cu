@@ -32,6 +32,7 @@
 #include <mutex>
 
 #include "common.cuh"
+#include "nvfp4_quant.cuh"
 
 namespace nvfp4 {
 namespace {
@@ -472,9 +473,25 @@ __global__ void __launch_bounds__(kThreads, NVFP4_ATTN_MIN_CTAS) attn_partial_ke
 }
 
 // out[b, h] = g_V * sum_s 2^(m_s - M) O_s / sum_s 2^(m_s - M) l_s
+// Where the combine kernel puts o: bf16 [batch, heads, 128], or (kQuant) the
+// NVFP4 A operand of the output projection: the bf16-rounded o of each query
+// head's 128 channels quantized in 8 blocks of 16 with the static tensor scale
+// g_out by the library's recipe, codes [batch, heads * 64] bytes and MMA-layout
+// scales of the [batch, heads * 128] matrix (padding rows zero).
+struct CombineOut {
+  uint16_t* bf16;
+  uint8_t* codes;
+  uint8_t* scales;
+  const float* g_out;
+  int* status;
+  int rows;
+  uint32_t kgroups;
+};
+
+template <bool kQuant>
 __global__ void __launch_bounds__(kD) attn_combine_kernel(const float* __restrict__ o_ws,
                                                          const float* __restrict__ ml_ws, int n_splits, float gv,
-                                                         uint16_t* __restrict__ out) {
+                                                         const CombineOut out) {
   griddep_wait_and_release();
   const size_t bh = static_cast<size_t>(blockIdx.y) * gridDim.x + blockIdx.x;
   const float* ml = ml_ws + bh * n_splits * 2;
@@ -491,7 +508,39 @@ __global__ void __launch_bounds__(kD) attn_combine_kernel(const float* __restric
   const float r = L > 0.0f ? __fdiv_rn(acc, L) * gv : 0.0f;
   uint16_t bits;
   asm("cvt.rn.bf16.f32 %0, %1;" : "=h"(bits) : "f"(r));
-  out[bh * kD + threadIdx.x] = bits;
+  if (!kQuant) {
+    out.bf16[bh * kD + threadIdx.x] = bits;
+    return;
+  }
+  // Lanes 16j..16j+15 of a warp hold one 16-channel block of this head.
+  const float g_in = __ldg(out.g_out);
+  const bool g_ok = g_in > 0.0f && g_in <= FLT_MAX;
+  if (!g_ok && bh == 0 && threadIdx.x == 0) set_status(out.status, NVFP4_ERR_INVALID_ARG);
+  const float g = g_ok ? g_in : 1.0f;
+  const float x = __uint_as_float(static_cast<uint32_t>(bits) << 16);
+  float amax = fabsf(x);
+#pragma unroll
+  for (int sh = 1; sh < 16; sh <<= 1) amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, sh));
+  const BlockScale bs = block_scale(amax, g, __fmul_rn(6.0f, g));
+  // Lane pairs (2i, 2i+1) form one code byte, element 2i in the low nibble.
+  const float mine = __fmul_rn(x, bs.mult);
+  const float other = __shfl_xor_sync(0xffffffffu, mine, 1);
+  uint32_t pair;  // the first source of the conversion goes to the high nibble
+  asm("{\n .reg .b8 t;\n cvt.rn.satfinite.e2m1x2.f32 t, %1, %2;\n cvt.u32.u8 %0, t;\n}"
+      : "=r"(pair)
+      : "f"(other), "f"(mine));
+  const uint32_t row = blockIdx.y, head = blockIdx.x, c = threadIdx.x;
+  if ((c & 1) == 0)
+    out.codes[static_cast<size_t>(row) * (gridDim.x * (kD / 2)) + head * (kD / 2) + c / 2] =
+        g_ok ? static_cast<uint8_t>(pair & 0xFFu) : 0;
+  const uint32_t kb = head * (kD / 16) + c / 16;
+  if ((c & 15) == 0) out.scales[mma_scale_offset(row, kb, out.kgroups)] = g_ok ? static_cast<uint8_t>(bs.code) : 0;
+  // Rows from batch up to the next multiple of 128 hold zero scales.
+  if (row == 0 && c < kD / 16) {
+    const uint32_t padded = (static_cast<uint32_t>(out.rows) + 127u) & ~127u;
+    for (uint32_t pr = out.rows; pr < padded; ++pr)
+      out.scales[mma_scale_offset(pr, head * (kD / 16) + c, out.kgroups)] = 0;
+  }
 }
 
 int splits_for(int capacity) { return (capacity + kChunk - 1) / kChunk; }
@@ -542,10 +591,14 @@ NVFP4_API size_t decode_attention_nvfp4_workspace_size(int32_t batch, int32_t nu
   return static_cast<size_t>(batch) * num_q_heads * splits_for(capacity) * (kD + 2) * sizeof(float);
 }
 
-NVFP4_API nvfp4_status decode_attention_nvfp4(const nvfp4_kv_cache* cache, const void* q_bf16, int32_t num_q_heads,
-                                              float softmax_scale, void* out_bf16, void* workspace,
-                                              size_t workspace_bytes, void* stream) {
-  if (!cache || !q_bf16 || !out_bf16 || !workspace || !cache->seq_lens) return NVFP4_ERR_INVALID_ARG;
+namespace nvfp4 {
+namespace {
+
+// Checks shared by the decode-attention entry points (all but the output
+// buffers and the split-KV partials).
+nvfp4_status attention_validate(const nvfp4_kv_cache* cache, const void* q_bf16, int32_t num_q_heads,
+                                float softmax_scale) {
+  if (!cache || !q_bf16 || !cache->seq_lens) return NVFP4_ERR_INVALID_ARG;
   if (!cache->k_codes || !cache->k_scales || !cache->v_codes || !cache->v_scales) return NVFP4_ERR_INVALID_ARG;
   if (!kv_format_ok(cache)) return NVFP4_ERR_INVALID_ARG;
   if (!(cache->k_gscale > 0.0f && cache->k_gscale <= FLT_MAX) || !(cache->v_gscale > 0.0f && cache->v_gscale <= FLT_MAX) ||
@@ -558,36 +611,94 @@ NVFP4_API nvfp4_status decode_attention_nvfp4(const nvfp4_kv_cache* cache, const
   if (static_cast<int64_t>(cache->batch) > 65535 || num_q_heads > 65535) return NVFP4_ERR_SHAPE;
   const int64_t n_items = static_cast<int64_t>(cache->batch) * cache->num_kv_heads * splits_for(cache->capacity);
   if (n_items >= (1ll << 31)) return NVFP4_ERR_SHAPE;
-  if (workspace_bytes < decode_attention_nvfp4_workspace_size(cache->batch, num_q_heads, cache->capacity))
-    return NVFP4_ERR_SHAPE;
-  if (!aligned(q_bf16, 16) || !aligned(out_bf16, 16) || !aligned(workspace, 16) || !aligned(cache->k_codes, 16) ||
-      !aligned(cache->v_codes, 16) || !aligned(cache->k_scales, 16) || !aligned(cache->v_scales, 16))
+  return NVFP4_OK;
+}
+
+// Alignment of the query and cache arrays, then the partial kernel's
+// parameters with its partials at `partials` and its grid size.
+nvfp4_status attention_params(const nvfp4_kv_cache* cache, const void* q_bf16, int32_t num_q_heads,
+                              float softmax_scale, float* partials, Params* prm, int* grid) {
+  if (!aligned(q_bf16, 16) || !aligned(cache->k_codes, 16) || !aligned(cache->v_codes, 16) ||
+      !aligned(cache->k_scales, 16) || !aligned(cache->v_scales, 16))
     return NVFP4_ERR_ALIGN;
   const int ctas_max = resident_ctas(cache);
   if (ctas_max <= 0) return NVFP4_ERR_CUDA;
+  const int64_t n_items = static_cast<int64_t>(cache->batch) * cache->num_kv_heads * splits_for(cache->capacity);
+  prm->k_codes = cache->k_codes;
+  prm->k_scales = cache->k_scales;
+  prm->v_codes = cache->v_codes;
+  prm->v_scales = cache->v_scales;
+  prm->seq_lens = cache->seq_lens;
+  prm->q = static_cast<const uint16_t*>(q_bf16);
+  prm->status = status_word_dev();
+  prm->hkv = cache->num_kv_heads;
+  prm->capacity = cache->capacity;
+  prm->hq = num_q_heads;
+  prm->group = num_q_heads / cache->num_kv_heads;
+  prm->n_splits = splits_for(cache->capacity);
+  prm->n_items = static_cast<int>(n_items);
+  prm->logit_mult = softmax_scale * cache->k_gscale * kLog2e;
+  // Every record the combine kernel reads is written by the partial kernel of
+  // the same call, so nothing left from an earlier call needs clearing.
+  prm->o_ws = partials;
+  prm->ml_ws = prm->o_ws + static_cast<size_t>(cache->batch) * num_q_heads * prm->n_splits * kD;
+  *grid = static_cast<int>(n_items < ctas_max ? n_items : ctas_max);
+  return NVFP4_OK;
+}
+
+}  // namespace
+}  // namespace nvfp4
+
+NVFP4_API nvfp4_status decode_attention_nvfp4(const nvfp4_kv_cache* cache, const void* q_bf16, int32_t num_q_heads,
+                                              float softmax_scale, void* out_bf16, void* workspace,
+                                              size_t workspace_bytes, void* stream) {
+  if (!out_bf16 || !workspace) return NVFP4_ERR_INVALID_ARG;
+  nvfp4_status st = attention_validate(cache, q_bf16, num_q_heads, softmax_scale);
+  if (st != NVFP4_OK) return st;
+  if (workspace_bytes < decode_attention_nvfp4_workspace_size(cache->batch, num_q_heads, cache->capacity))
+    return NVFP4_ERR_SHAPE;
+  if (!aligned(out_bf16, 16) || !aligned(workspace, 16)) return NVFP4_ERR_ALIGN;
   Params prm;
-  prm.k_codes = cache->k_codes;
-  prm.k_scales = cache->k_scales;
-  prm.v_codes = cache->v_codes;
-  prm.v_scales = cache->v_scales;
-  prm.seq_lens = cache->seq_lens;
-  prm.q = static_cast<const uint16_t*>(q_bf16);
-  prm.status = status_word_dev();
-  prm.hkv = cache->num_kv_heads;
-  prm.capacity = cache->capacity;
-  prm.hq = num_q_heads;
-  prm.group = num_q_heads / cache->num_kv_heads;
-  prm.n_splits = splits_for(cache->capacity);
-  prm.n_items = static_cast<int>(n_items);
-  prm.logit_mult = softmax_scale * cache->k_gscale * kLog2e;
-  prm.o_ws = static_cast<float*>(workspace);
-  prm.ml_ws = prm.o_ws + static_cast<size_t>(cache->batch) * num_q_heads * prm.n_splits * kD;
+  int grid = 0;
+  st = attention_params(cache, q_bf16, num_q_heads, softmax_scale, static_cast<float*>(workspace), &prm, &grid);
+  if (st != NVFP4_OK) return st;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  const int grid = static_cast<int>(n_items < ctas_max ? n_items : ctas_max);
   if (launch_pdl(partial_kernel(cache), dim3(grid), dim3(kThreads), kSmemBytes, s, prm) != cudaSuccess ||
-      launch_pdl(attn_combine_kernel, dim3(num_q_heads, cache->batch), dim3(kD), 0, s,
+      launch_pdl(attn_combine_kernel<false>, dim3(num_q_heads, cache->batch), dim3(kD), 0, s,
                  static_cast<const float*>(prm.o_ws), static_cast<const float*>(prm.ml_ws), prm.n_splits,
-                 cache->v_gscale, static_cast<uint16_t*>(out_bf16)) != cudaSuccess)
+                 cache->v_gscale, CombineOut{static_cast<uint16_t*>(out_bf16)}) != cudaSuccess)
+    return NVFP4_ERR_CUDA;
+  count_launches(2);
+  return launch_status();
+}
+
+NVFP4_API nvfp4_status decode_attention_nvfp4_quantize(const nvfp4_kv_cache* cache, const void* q_bf16,
+                                                       int32_t num_q_heads, float softmax_scale, const float* g_out,
+                                                       uint8_t* out_codes, uint8_t* out_scales, void* workspace,
+                                                       size_t workspace_bytes, void* stream) {
+  if (!g_out || !out_codes || !out_scales || !workspace) return NVFP4_ERR_INVALID_ARG;
+  nvfp4_status st = attention_validate(cache, q_bf16, num_q_heads, softmax_scale);
+  if (st != NVFP4_OK) return st;
+  if (workspace_bytes < decode_attention_nvfp4_workspace_size(cache->batch, num_q_heads, cache->capacity))
+    return NVFP4_ERR_SHAPE;
+  if (!aligned(out_codes, 16) || !aligned(out_scales, 4) || !aligned(g_out, 4) || !aligned(workspace, 16))
+    return NVFP4_ERR_ALIGN;
+  Params prm;
+  int grid = 0;
+  st = attention_params(cache, q_bf16, num_q_heads, softmax_scale, static_cast<float*>(workspace), &prm, &grid);
+  if (st != NVFP4_OK) return st;
+  CombineOut o{};
+  o.codes = out_codes;
+  o.scales = out_scales;
+  o.g_out = g_out;
+  o.status = status_word_dev();
+  o.rows = cache->batch;
+  o.kgroups = static_cast<uint32_t>(num_q_heads) * (kD / 64);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (launch_pdl(partial_kernel(cache), dim3(grid), dim3(kThreads), kSmemBytes, s, prm) != cudaSuccess ||
+      launch_pdl(attn_combine_kernel<true>, dim3(num_q_heads, cache->batch), dim3(kD), 0, s,
+                 static_cast<const float*>(prm.o_ws), static_cast<const float*>(prm.ml_ws), prm.n_splits,
+                 cache->v_gscale, o) != cudaSuccess)
     return NVFP4_ERR_CUDA;
   count_launches(2);
   return launch_status();
@@ -626,55 +737,25 @@ float* attn_static_scratch_dev() {
 NVFP4_API nvfp4_status decode_attention_nvfp4_static_scratch(const nvfp4_kv_cache* cache, const void* q_bf16,
                                                              int32_t num_q_heads, float softmax_scale,
                                                              void* out_bf16, void* stream) {
-  if (!cache || !q_bf16 || !out_bf16 || !cache->seq_lens) return NVFP4_ERR_INVALID_ARG;
-  if (!cache->k_codes || !cache->k_scales || !cache->v_codes || !cache->v_scales) return NVFP4_ERR_INVALID_ARG;
-  if (!kv_format_ok(cache)) return NVFP4_ERR_INVALID_ARG;
-  if (!(cache->k_gscale > 0.0f && cache->k_gscale <= FLT_MAX) || !(cache->v_gscale > 0.0f && cache->v_gscale <= FLT_MAX) ||
-      !(softmax_scale > 0.0f && softmax_scale <= FLT_MAX))
-    return NVFP4_ERR_INVALID_ARG;
-  if (cache->head_dim != kD || cache->batch <= 0 || cache->num_kv_heads <= 0 || cache->capacity <= 0 ||
-      cache->capacity % 2 || num_q_heads <= 0 || num_q_heads % cache->num_kv_heads ||
-      num_q_heads / cache->num_kv_heads > 8)
-    return NVFP4_ERR_SHAPE;
-  if (static_cast<int64_t>(cache->batch) > 65535 || num_q_heads > 65535) return NVFP4_ERR_SHAPE;
-  const int64_t n_items = static_cast<int64_t>(cache->batch) * cache->num_kv_heads * splits_for(cache->capacity);
-  if (n_items >= (1ll << 31)) return NVFP4_ERR_SHAPE;
+  if (!out_bf16) return NVFP4_ERR_INVALID_ARG;
+  nvfp4_status st = attention_validate(cache, q_bf16, num_q_heads, softmax_scale);
+  if (st != NVFP4_OK) return st;
   // The partials must fit in the static scratch; larger problems are refused.
   if (decode_attention_nvfp4_workspace_size(cache->batch, num_q_heads, cache->capacity) >
       NVFP4_ATTN_STATIC_SCRATCH_BYTES)
     return NVFP4_ERR_SHAPE;
-  if (!aligned(q_bf16, 16) || !aligned(out_bf16, 16) || !aligned(cache->k_codes, 16) ||
-      !aligned(cache->v_codes, 16) || !aligned(cache->k_scales, 16) || !aligned(cache->v_scales, 16))
-    return NVFP4_ERR_ALIGN;
+  if (!aligned(out_bf16, 16)) return NVFP4_ERR_ALIGN;
   float* scratch = attn_static_scratch_dev();
   if (!scratch) return NVFP4_ERR_CUDA;
-  const int ctas_max = resident_ctas(cache);
-  if (ctas_max <= 0) return NVFP4_ERR_CUDA;
   Params prm;
-  prm.k_codes = cache->k_codes;
-  prm.k_scales = cache->k_scales;
-  prm.v_codes = cache->v_codes;
-  prm.v_scales = cache->v_scales;
-  prm.seq_lens = cache->seq_lens;
-  prm.q = static_cast<const uint16_t*>(q_bf16);
-  prm.status = status_word_dev();
-  prm.hkv = cache->num_kv_heads;
-  prm.capacity = cache->capacity;
-  prm.hq = num_q_heads;
-  prm.group = num_q_heads / cache->num_kv_heads;
-  prm.n_splits = splits_for(cache->capacity);
-  prm.n_items = static_cast<int>(n_items);
-  prm.logit_mult = softmax_scale * cache->k_gscale * kLog2e;
-  // Every record the combine kernel reads is written by the partial kernel of
-  // the same call, so nothing left from an earlier call needs clearing.
-  prm.o_ws = scratch;
-  prm.ml_ws = prm.o_ws + static_cast<size_t>(cache->batch) * num_q_heads * prm.n_splits * kD;
+  int grid = 0;
+  st = attention_params(cache, q_bf16, num_q_heads, softmax_scale, scratch, &prm, &grid);
+  if (st != NVFP4_OK) return st;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  const int grid = static_cast<int>(n_items < ctas_max ? n_items : ctas_max);
   if (launch_pdl(partial_kernel(cache), dim3(grid), dim3(kThreads), kSmemBytes, s, prm) != cudaSuccess ||
-      launch_pdl(attn_combine_kernel, dim3(num_q_heads, cache->batch), dim3(kD), 0, s,
+      launch_pdl(attn_combine_kernel<false>, dim3(num_q_heads, cache->batch), dim3(kD), 0, s,
                  static_cast<const float*>(prm.o_ws), static_cast<const float*>(prm.ml_ws), prm.n_splits,
-                 cache->v_gscale, static_cast<uint16_t*>(out_bf16)) != cudaSuccess)
+                 cache->v_gscale, CombineOut{static_cast<uint16_t*>(out_bf16)}) != cudaSuccess)
     return NVFP4_ERR_CUDA;
   count_launches(2);
   return launch_status();

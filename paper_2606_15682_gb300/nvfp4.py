@@ -62,6 +62,8 @@ _kv_append_rope = _sig("kv_append_rope_nvfp4",
 _rope_table = _sig("nvfp4_rope_table", [_p, _i64, _i32, _f32, _p])
 _attn_ws = _sig("decode_attention_nvfp4_workspace_size", [_i32, _i32, _i32], _sz)
 _attn = _sig("decode_attention_nvfp4", [ctypes.POINTER(KVCacheStruct), _p, _i32, _f32, _p, _p, _sz, _p])
+_attn_quant = _sig("decode_attention_nvfp4_quantize",
+                   [ctypes.POINTER(KVCacheStruct), _p, _i32, _f32, _p, _p, _p, _p, _sz, _p])
 _attn_static = _sig("decode_attention_nvfp4_static_scratch", [ctypes.POINTER(KVCacheStruct), _p, _i32, _f32, _p, _p])
 _get_status = _sig("nvfp4_get_device_status", [ctypes.POINTER(_i32), _p])
 _status_string = _sig("nvfp4_status_string", [ctypes.c_int], ctypes.c_char_p)
@@ -182,6 +184,15 @@ def decode_attention_nvfp4(cache, q, softmax_scale, out, workspace, stream=None)
 ATTN_STATIC_SCRATCH_BYTES = 24 << 20
 
 
+def decode_attention_nvfp4_quantize(cache, q, softmax_scale, g_out, out_codes, out_scales, workspace, stream=None):
+    """out_codes [batch, H_q*64] uint8, out_scales MMA layout for [batch, H_q*128]."""
+    s = cache.struct()
+    _check("decode_attention_nvfp4_quantize",
+           _attn_quant(ctypes.byref(s), _ptr(q), q.shape[1], softmax_scale, _ptr(g_out), _ptr(out_codes),
+                       _ptr(out_scales), _ptr(workspace), workspace.numel() * workspace.element_size(),
+                       _stream(stream)))
+
+
 def decode_attention_nvfp4_static_scratch(cache, q, softmax_scale, out, stream=None):
     """Decode attention whose partials live in the library's own device scratch (no workspace)."""
     s = cache.struct()
@@ -228,5 +239,6 @@ class KVCache:
 EXPORTED = ["nvfp4_scales_bytes", "nvfp4_tensor_scale", "nvfp4_quantize", "nvfp4_quantize_dynamic", "nvfp4_scales_relayout", "nvfp4_linear",
             "nvfp4_linear_swiglu_quantize", "nvfp4_interleave_gate_up",
             "kv_append_nvfp4", "kv_append_rope_nvfp4", "nvfp4_rope_table", "decode_attention_nvfp4_workspace_size", "decode_attention_nvfp4",
+            "decode_attention_nvfp4_quantize",
             "decode_attention_nvfp4_static_scratch",
             "nvfp4_get_device_status", "nvfp4_status_string", "nvfp4_launch_count"]

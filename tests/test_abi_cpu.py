@@ -103,3 +103,11 @@ def test_kv_and_attention_validation():
     assert L.decode_attention_nvfp4(ctypes.byref(cache()), p, 4, ctypes.c_float(-1.0), p, p, ws, s) == 1
     ws_odd = N.decode_attention_nvfp4_workspace_size(2, 4, 63)
     assert L.decode_attention_nvfp4(ctypes.byref(cache(capacity=63)), p, 4, ctypes.c_float(0.1), p, p, ws_odd, s) == 2
+    # attention with the output quantized for the o projection
+    f = ctypes.c_float(0.1)
+    assert L.decode_attention_nvfp4_quantize(ctypes.byref(cache()), p, 4, f, None, p, p, p, ws, s) == 1     # no g_out
+    assert L.decode_attention_nvfp4_quantize(ctypes.byref(cache()), p, 4, f, p, None, p, p, ws, s) == 1     # no codes
+    assert L.decode_attention_nvfp4_quantize(ctypes.byref(cache()), p, 3, f, p, p, p, p, ws, s) == 2        # 3 % 2
+    assert L.decode_attention_nvfp4_quantize(ctypes.byref(cache()), p, 4, f, p, p, p, p, ws - 16, s) == 2   # workspace
+    assert L.decode_attention_nvfp4_quantize(ctypes.byref(cache()), p, 4, f, p, odd, p, p, ws, s) == 3      # codes align
+    assert L.decode_attention_nvfp4_quantize(ctypes.byref(cache(kv_format=5)), p, 4, f, p, p, p, p, ws, s) == 1

@@ -189,6 +189,80 @@ def test_full_size_decode_attention_workload(N):
         assert_close(f32(out[b]), ref[0], what=f"seq {b}")
 
 
+# ------------------------- attention output quantized for the o projection ---
+
+@pytest.mark.parametrize("B,hq,hkv,lens", [(3, 40, 8, [1000, 15, 2049]), (2, 8, 1, [0, 300]), (130, 8, 2, None)])
+def test_decode_attention_quantize(N, B, hq, hkv, lens):
+    """decode_attention_nvfp4_quantize: codes and scales bit-identical to the
+    bf16 attention followed by nvfp4_quantize on the GPU; against the oracle
+    (fp64 attention rounded to bf16, then the oracle's quantizer) the scales
+    are within one E4M3 step, almost all codes equal, every element within the
+    quantization error bound of the fp64 output, and padding scales zero."""
+    if lens is None:
+        lens = [int(x) for x in np.random.default_rng(B).integers(1, 65, B)]
+    cap = (max(max(lens), 1) + 6) & ~1
+    rec = synth.KVRecipe(hkv, seed=B * 7 + hq)
+    T = sum(lens)
+    k, v = rec.kv(max(T, 1), seed=13)
+    seq = np.concatenate([np.full(l, b) for b, l in enumerate(lens)]).astype(np.int64)
+    pos = np.concatenate([np.arange(l) for l in lens]).astype(np.int64)
+    k, v = k[:T], v[:T]
+    gk, gv = O.tensor_scale(f32(k)), O.tensor_scale(f32(v))
+    cache = N.KVCache(B, hkv, cap, gk, gv)
+    fill(N, cache, k, v, seq, pos)
+    cache.seq_lens.copy_(torch.tensor(lens, dtype=torch.int32))
+    q = rec.queries(B, hq, seed=14)
+    scale = 1.0 / math.sqrt(128)
+    rkc, rks, rvc, rvs = oracle_cache(B, hkv, cap)
+    O.kv_append(rkc, rks, rvc, rvs, f32(k), f32(v), seq, pos, np.float32(gk), np.float32(gv))
+    ref = O.decode_attention(f32(q), rkc, rks, rvc, rvs, lens, gk, gv, scale).reshape(B, hq * 128)
+    g_out = O.tensor_scale(ref.astype(np.float32))          # a calibrated static scale, from the oracle
+    g_dev = torch.tensor([g_out], dtype=torch.float32, device="cuda")
+    cols = hq * 128
+    codes = torch.full((B, cols // 2), 0xEE, dtype=torch.uint8, device="cuda")
+    scales = torch.full((N.nvfp4_scales_bytes(B, cols, 1),), 0xEE, dtype=torch.uint8, device="cuda")
+    ws = torch.empty(N.decode_attention_nvfp4_workspace_size(B, hq, cap) // 4, dtype=torch.float32, device="cuda")
+    N.decode_attention_nvfp4_quantize(cache, q.cuda(), scale, g_dev, codes, scales, ws)
+    out = run_attention(N, cache, q, scale)
+    c2 = torch.empty_like(codes)
+    s2 = torch.empty_like(scales)
+    N.nvfp4_quantize(out.view(B, cols), g_dev, c2, s2, 1)
+    torch.cuda.synchronize()
+    assert N.nvfp4_get_device_status() == 0
+    assert torch.equal(codes, c2) and torch.equal(scales, s2), "differs from attention + nvfp4_quantize"
+    rc, rs = O.quantize(O._bf16_round(ref.astype(np.float32)), g_out)
+    gs = O.scales_from_mma(u8(scales), B, cols)
+    assert np.abs(gs.astype(int) - rs.astype(int)).max() <= 1
+    assert (gs == rs).mean() > 0.99 and (u8(codes) == rc).mean() > 0.99
+    deq = O.dequantize(u8(codes), gs, g_out)
+    S = O.e4m3_decode(gs).repeat(16, axis=1)
+    tol = 2e-3 * np.abs(ref).max(axis=1, keepdims=True)    # the attention's own tolerance, per sequence
+    assert np.all(np.abs(deq - ref) <= 1.5 * S * np.float64(g_out) + tol)
+    for b, l in enumerate(lens):
+        if l == 0:
+            assert not u8(codes)[b].any() and not gs[b].any(), "an empty sequence gives zero codes and scales"
+    pad = np.setdiff1d(np.arange(O.mma_scale_bytes(B, cols)), O._mma_offsets(B, cols // 16).ravel())
+    assert not u8(scales)[pad].any(), "padding rows of the output scales must be zero"
+
+
+def test_decode_attention_quantize_invalid_g_out(N):
+    B, hq, hkv, cap = 1, 8, 8, 64
+    rec = synth.KVRecipe(hkv, seed=5)
+    k, v = rec.kv(cap, seed=1)
+    cache = N.KVCache(B, hkv, cap, O.tensor_scale(f32(k)), O.tensor_scale(f32(v)))
+    fill(N, cache, k, v, np.zeros(cap, np.int64), np.arange(cap))
+    cache.seq_lens.fill_(cap)
+    q = rec.queries(B, hq, seed=2)
+    codes = torch.full((B, hq * 64), 0xEE, dtype=torch.uint8, device="cuda")
+    scales = torch.full((N.nvfp4_scales_bytes(B, hq * 128, 1),), 0xEE, dtype=torch.uint8, device="cuda")
+    ws = torch.empty(N.decode_attention_nvfp4_workspace_size(B, hq, cap) // 4, dtype=torch.float32, device="cuda")
+    N.nvfp4_get_device_status()
+    N.decode_attention_nvfp4_quantize(cache, q.cuda(), 0.088, torch.tensor([0.0], device="cuda"), codes, scales, ws)
+    torch.cuda.synchronize()
+    assert N.nvfp4_get_device_status() == 1
+    assert not u8(codes).any() and not u8(scales).any()
+
+
 # ----------------------------------- fused RoPE -> shift -> quantize -> append ---
 
 def test_rope_table_matches_numpy(N):
