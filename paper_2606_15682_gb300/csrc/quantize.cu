@@ -231,7 +231,10 @@ template <bool kMMA>
 __global__ void __launch_bounds__(kThreads) quantize_dynamic_kernel(
     const uint16_t* __restrict__ x, FastDiv kblocks_div, uint32_t total_blocks, int64_t ld, bool dense, uint32_t rows,
     unsigned long long* state, float* __restrict__ g_out, uint2* __restrict__ codes, uint8_t* __restrict__ scales,
-    int* status) {
+    int* status, int stash_iters) {
+  // Shared-memory stash: the blocks of the first stash_iters phase-1
+  // iterations, [iteration * kUnroll + slot][half][thread] as 16-byte words.
+  extern __shared__ uint4 stash[];
   griddep_wait_and_release();
   const uint32_t lane = threadIdx.x & 31;
   const uint32_t stride = gridDim.x * blockDim.x;
@@ -239,15 +242,23 @@ __global__ void __launch_bounds__(kThreads) quantize_dynamic_kernel(
   if (threadIdx.x == 0) epoch = ld_acquire_u64(&state[0]) >> 32;
   // Resident: one pass covers the tensor, so the loaded blocks stay in
   // registers across the barrier and x is read once.  Otherwise the blocks
-  // of the last phase-1 iteration stay in registers and phase 2 starts with
-  // them, so only the earlier iterations are read again.
-  const bool resident = total_blocks <= stride * kUnroll;
+  // of the last phase-1 iteration stay in registers, those of the first
+  // stash_iters iterations in shared memory, and phase 2 reads from x again
+  // only the iterations in between.
   const uint32_t bidx_first = blockIdx.x * blockDim.x + (threadIdx.x & ~31u);
   BlockSlots sl;
   uint32_t m = 0, bidx_last = bidx_first;
-  for (uint32_t bidx0 = bidx_first; bidx0 < total_blocks || bidx0 == bidx_first; bidx0 += stride * kUnroll) {
+  int it = 0;
+  for (uint32_t bidx0 = bidx_first; bidx0 < total_blocks || bidx0 == bidx_first; bidx0 += stride * kUnroll, ++it) {
     load_blocks(x, kblocks_div, total_blocks, ld, dense, bidx0, stride, lane, sl);
     m = max(m, amax_bits_of(sl));
+    if (it < stash_iters) {
+#pragma unroll
+      for (int u = 0; u < kUnroll; ++u) {
+        stash[((it * kUnroll + u) * 2) * kThreads + threadIdx.x] = sl.v0[u];
+        stash[((it * kUnroll + u) * 2 + 1) * kThreads + threadIdx.x] = sl.v1[u];
+      }
+    }
     bidx_last = bidx0;
   }
   m = __reduce_max_sync(0xffffffffu, m);
@@ -290,36 +301,59 @@ __global__ void __launch_bounds__(kThreads) quantize_dynamic_kernel(
   if (blockIdx.x == 0 && threadIdx.x == 0) *g_out = g;
   if (bidx_last < total_blocks)
     quantize_loaded<kMMA>(sl, total_blocks, kblocks_div.d, bidx_last, stride, lane, g, six_g, true, codes, scales);
-  if (!resident) {
-    for (uint32_t bidx0 = bidx_first; bidx0 < bidx_last; bidx0 += stride * kUnroll) {
-      BlockSlots t;
+  it = 0;
+  for (uint32_t bidx0 = bidx_first; bidx0 < bidx_last; bidx0 += stride * kUnroll, ++it) {
+    BlockSlots t;
+    if (it < stash_iters) {
+      const uint32_t kblocks = kblocks_div.d;
+#pragma unroll
+      for (int u = 0; u < kUnroll; ++u) {
+        const uint32_t b = bidx0 + u * stride + lane;
+        t.row[u] = kblocks_div.div(b);
+        t.kb[u] = b - t.row[u] * kblocks;
+        t.v0[u] = stash[((it * kUnroll + u) * 2) * kThreads + threadIdx.x];
+        t.v1[u] = stash[((it * kUnroll + u) * 2 + 1) * kThreads + threadIdx.x];
+      }
+    } else {
       load_blocks(x, kblocks_div, total_blocks, ld, dense, bidx0, stride, lane, t);
-      quantize_loaded<kMMA>(t, total_blocks, kblocks_div.d, bidx0, stride, lane, g, six_g, true, codes, scales);
     }
+    quantize_loaded<kMMA>(t, total_blocks, kblocks_div.d, bidx0, stride, lane, g, six_g, true, codes, scales);
   }
   if (kMMA) zero_scale_padding(rows, kblocks_div.d, scales);
 }
 
 // Blocks of quantize_dynamic_kernel that fit on the device at once (a
 // cooperative launch must not exceed it).
+// Shared-memory stash per block for one phase-1 iteration (kUnroll slots of
+// two 16-byte words per thread), and the most iterations stashed.
+constexpr size_t kStashIterBytes = static_cast<size_t>(kUnroll) * 2 * kThreads * 16;
+constexpr int kMaxStashIters = 2;
+
 template <bool kMMA>
-int dynamic_capacity() {
+int dynamic_capacity(int stash_iters) {
   static std::mutex mu;
-  static std::map<int, int> cache;
+  static std::map<std::pair<int, int>, int> cache;
   int d = 0;
   if (cudaGetDevice(&d) != cudaSuccess) return 0;
   std::lock_guard<std::mutex> lock(mu);
-  auto it = cache.find(d);
+  auto it = cache.find({d, stash_iters});
   if (it != cache.end()) return it->second;
+  const size_t smem = stash_iters * kStashIterBytes;
+  if (smem > 48 * 1024 &&
+      cudaFuncSetAttribute(quantize_dynamic_kernel<kMMA>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           static_cast<int>(kMaxStashIters * kStashIterBytes)) != cudaSuccess) {
+    cudaGetLastError();
+    return 0;
+  }
   int per_sm = 0;
-  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, quantize_dynamic_kernel<kMMA>, kThreads, 0) !=
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, quantize_dynamic_kernel<kMMA>, kThreads, smem) !=
           cudaSuccess ||
       per_sm <= 0) {
     cudaGetLastError();
     return 0;
   }
-  cache[d] = per_sm * sm_count();
-  return cache[d];
+  cache[{d, stash_iters}] = per_sm * sm_count();
+  return cache[{d, stash_iters}];
 }
 
 template <bool kToMMA>
@@ -437,14 +471,25 @@ NVFP4_API nvfp4_status nvfp4_quantize_dynamic(const void* x_bf16, int64_t rows, 
   if (!codes || !scales) return NVFP4_ERR_INVALID_ARG;
   if (!aligned(codes, 8)) return NVFP4_ERR_ALIGN;
   const bool mma = layout == NVFP4_SCALES_MMA;
-  const int cap = mma ? dynamic_capacity<true>() : dynamic_capacity<false>();
-  if (cap <= 0) return NVFP4_ERR_CUDA;
   const uint32_t kblocks = static_cast<uint32_t>(cols / 16);
   const uint32_t total_blocks = static_cast<uint32_t>(rows * kblocks);
   // kUnroll blocks per thread per pass, as few CTAs as that allows (each CTA
   // is one arrival at the grid barrier); x stays in registers across the
-  // barrier when one pass covers it.
+  // barrier when one pass covers it, and up to kMaxStashIters more passes
+  // wait in shared memory.
   int grid = grid_for(total_blocks, kThreads * kUnroll);
+  int cap = mma ? dynamic_capacity<true>(0) : dynamic_capacity<false>(0);
+  if (cap <= 0) return NVFP4_ERR_CUDA;
+  int stash_iters = 0;
+  if (grid > cap) {
+    const int cap_stash = mma ? dynamic_capacity<true>(kMaxStashIters) : dynamic_capacity<false>(kMaxStashIters);
+    if (cap_stash > 0) {
+      const uint64_t per_iter = static_cast<uint64_t>(cap_stash) * kThreads * kUnroll;
+      const uint64_t iters = (total_blocks + per_iter - 1) / per_iter;
+      stash_iters = static_cast<int>(iters - 1 < kMaxStashIters ? iters - 1 : kMaxStashIters);
+      cap = cap_stash;
+    }
+  }
   if (grid > cap) grid = cap;
   if (grid > 0xFFFF) grid = 0xFFFF;  // the barrier counts arrivals in 16 bits
   // Cooperative: every block is resident at once, so the grid barrier can
@@ -455,7 +500,7 @@ NVFP4_API nvfp4_status nvfp4_quantize_dynamic(const void* x_bf16, int64_t rows, 
   attr[0].val.cooperative = 1;
   cfg.gridDim = dim3(grid);
   cfg.blockDim = dim3(kThreads);
-  cfg.dynamicSmemBytes = 0;
+  cfg.dynamicSmemBytes = stash_iters * kStashIterBytes;
   cfg.stream = static_cast<cudaStream_t>(stream);
   cfg.attrs = attr;
   cfg.numAttrs = 1;
@@ -463,7 +508,7 @@ NVFP4_API nvfp4_status nvfp4_quantize_dynamic(const void* x_bf16, int64_t rows, 
       cudaLaunchKernelEx(&cfg, mma ? quantize_dynamic_kernel<true> : quantize_dynamic_kernel<false>,
                          static_cast<const uint16_t*>(x_bf16), FastDiv(kblocks), total_blocks, ld, ld == cols,
                          static_cast<uint32_t>(rows), static_cast<unsigned long long*>(state_dev), g_dev,
-                         reinterpret_cast<uint2*>(codes), scales, status_word_dev());
+                         reinterpret_cast<uint2*>(codes), scales, status_word_dev(), stash_iters);
   if (e != cudaSuccess) return NVFP4_ERR_CUDA;
   count_launches(1);
   return launch_status();
