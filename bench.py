@@ -49,8 +49,8 @@ NCU_TRAFFIC = {
     "gemm": {"bytes": 17293824 + 12077824, "sources": ("gemm.cu", "common.cuh"), "sha": "df869ea01e6926f0",
              "shape": (2048, 17920, 1536),
              "profile": "profiles/gemm_qwen1.5b_prefill_gate_up_m2048_n17920_k1536.md"},
-    "attention": {"bytes": 1208723712 + 22171648, "sources": ("attention.cu", "common.cuh"),
-                  "sha": "1567a570bf179aaf", "shape": (64, 16384),
+    "attention": {"bytes": 1208721408 + 22182656, "sources": ("attention.cu", "common.cuh"),
+                  "sha": "47bada2c82109b77", "shape": (64, 16384),
                   "profile": "profiles/attention_qwen14b_decode_b64_t16384.md (attn_partial_kernel)"},
 }
 
