@@ -193,6 +193,53 @@ nvfp4_status nvfp4_linear_swiglu_quantize(const uint8_t* a_codes, const uint8_t*
 nvfp4_status nvfp4_interleave_gate_up(const void* w_gate, const void* w_up, int64_t I, int64_t row_bytes,
                                       void* w_out, void* stream);
 
+/*
+ * MXFP4 format variant (Appendix A, table "Quantization configurations of
+ * MXFP4 and NVFP4"): E2M1 elements, one E8M0 (power-of-two) scale per block
+ * of 32 elements, no global scale; Sec. 5 evaluates MXFP4 W4A4 deployments.
+ *
+ * Bytes of an MXFP4 scale buffer for a [rows, cols] tensor: ROWMAJOR holds
+ * one E8M0 byte per 32-element block ([rows, cols/32]); MMA holds the byte
+ * order nvfp4_linear reads (nvfp4_scales_bytes(rows, cols, MMA) bytes), with
+ * each block's scale stored for both of its 16-element halves.
+ */
+size_t mxfp4_scales_bytes(int64_t rows, int64_t cols, nvfp4_scale_layout layout);
+
+/*
+ * MXFP4-quantize a [rows, cols] bf16 tensor along its rows.  Per block of 32
+ * consecutive elements (the paper fixes the format; the recipe is the OCP
+ * Microscaling rule it cites):
+ *   e = floor(log2(max |x_i|)) - 2, clamped to [-127, 127] (-127 for an
+ *   all-zero block); scale code = e + 127;
+ *   code_i = E2M1_RNE_satfinite(x_i / 2^e), sign kept (also for a value that
+ *   rounds to zero); values in [6, 8) 2^e saturate to 6 2^e.
+ * rotate = 1 first multiplies every 32-element block by H_32 / sqrt(32)
+ * (Sylvester-Hadamard; the block-wise rotation applied before MXFP4
+ * quantization, Sec. 4), computed in fp32 as butterflies (a + b, a - b) at
+ * strides 1, 2, 4, 8, 16 and one multiplication by fp32(1/sqrt(32)); rotate
+ * W's K dimension the same way so that the linear's product is unchanged.
+ *   codes  : [rows, cols/2] bytes, element 2j in the low nibble of byte j,
+ *            16-B aligned.
+ *   scales : mxfp4_scales_bytes(rows, cols, layout) bytes; MMA padding rows
+ *            are written as zeros.
+ * cols % 32 == 0 (ROWMAJOR) or cols % 64 == 0 (MMA), else SHAPE; x 16-B
+ * aligned and ld % 8 == 0 (ALIGN); rotate not 0/1 -> INVALID_ARG.
+ * rows*cols == 0 is a no-op.  Inputs must be finite.
+ */
+nvfp4_status mxfp4_quantize(const void* x_bf16, int64_t rows, int64_t cols, int64_t ld, int rotate,
+                            uint8_t* codes, uint8_t* scales, nvfp4_scale_layout layout, void* stream);
+
+/*
+ * a3 with MXFP4 operands: out[m, n] = bf16_rne( sum_k a[m,k] * w[n,k] ), a
+ * and w the dequantized MXFP4 values (e2m1 * 2^e), accumulated in fp32 by the
+ * tensor core (block-scaled MMA with UE8M0 scales).  Operands as
+ * nvfp4_linear with MMA-layout MXFP4 scales (mxfp4_quantize(..., MMA)) and
+ * no g.  Same shape and alignment rules as nvfp4_linear.
+ */
+nvfp4_status mxfp4_linear(const uint8_t* a_codes, const uint8_t* a_scales, const uint8_t* w_codes,
+                          const uint8_t* w_scales, int64_t M, int64_t N, int64_t K, void* out_bf16,
+                          int64_t ldo, void* stream);
+
 /* Element grid of the KV cache (the block scales are E4M3 per 16 either way). */
 typedef enum {
   /* E2M1, the NVFP4 element {0, 0.5, 1, 1.5, 2, 3, 4, 6} (the B200 deployment's

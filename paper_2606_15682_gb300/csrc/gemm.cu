@@ -149,6 +149,9 @@ __device__ __forceinline__ void unit_coords(int u, int msup, int tiles_n, int* m
   *nb = r / rows;
 }
 
+// Scale-format bit of the block-scaled MMA instruction descriptor (bit 23: UE8M0).
+constexpr uint32_t kScaleE8M0 = 1u << 23;
+
 struct GemmArgs {
   const uint8_t* sfa;
   const uint8_t* sfb;
@@ -157,6 +160,10 @@ struct GemmArgs {
   int M, N, K;
   int tiles_m, tiles_n;
   int* status;
+  // OR-ed into the MMA instruction descriptor: 0 for UE4M3 block scales
+  // (NVFP4), kScaleE8M0 for UE8M0 (MXFP4).  With ga == nullptr the epilogue
+  // applies no global scale (MXFP4 has none).
+  uint32_t idesc_fmt;
   // Fused SwiGLU + quantization epilogue (pair kernel, kSwiGLU): outputs.
   uint8_t* q_codes;   // [M, N/4] bytes: N/2 SwiGLU outputs per row
   uint8_t* q_scales;  // MMA layout for [M, N/2]
@@ -296,7 +303,7 @@ __global__ void __launch_bounds__(C::kThreads, 1)
 #pragma unroll
         for (int kk = 0; kk < 4; ++kk) {
           mma_fp4(d_tmem, desc_sw128(sA0 + stage * C::kTileBytesA + kk * 32),
-                  desc_sw128(sB0 + stage * C::kTileBytesB + kk * 32), C::kIdesc, sfa_col + kk * 4,
+                  desc_sw128(sB0 + stage * C::kTileBytesB + kk * 32), C::kIdesc | args.idesc_fmt, sfa_col + kk * 4,
                   sfb_col + kk * C::kSfbColsPerMma, (kb | kk) != 0);
         }
         if (CM > 1) tc_commit_mc(&empty[stage], cluster_mask);
@@ -344,7 +351,7 @@ __global__ void __launch_bounds__(C::kThreads, 1)
     const int colbase = ((warp - 3) >> 2) * 128;  // accumulator columns this warp drains
     uint8_t* buf_ptr = sEpi + (warp - 3) * kEpiBufBytes;
     const uint32_t buf = smem_u32(buf_ptr);
-    const float scale = __fmul_rn(__ldg(args.ga), __ldg(args.gb));
+    const float scale = args.ga ? __fmul_rn(__ldg(args.ga), __ldg(args.gb)) : 1.0f;
     int local = 0;
     for (int u = cluster_id; u < total_units; u += n_clusters, ++local) {
       int ms, nb;
@@ -677,7 +684,7 @@ __global__ void __launch_bounds__(C::kThreads, 1)
 #pragma unroll
         for (int kk = 0; kk < 4; ++kk)
           mma_fp4_pair(tmem, desc_sw128(sA0 + stage * C::kTileBytesA + kk * 32), desc_sw128(b_tile + kk * 32),
-                       C::kIdesc, sfa_col + kk * 4, sfb_col + kk * 8, (kb | kk) != 0);
+                       C::kIdesc | args.idesc_fmt, sfa_col + kk * 4, sfb_col + kk * 8, (kb | kk) != 0);
         tc_commit_pair(&empty[stage], 0x3);
         if (++stage == kStages) { stage = 0; phase ^= 1u; }
       }
@@ -740,7 +747,7 @@ __global__ void __launch_bounds__(C::kThreads, 1)
     constexpr int kEpi0 = 2 + C::kCopyWarps;
     const int quarter = warp & 3;
     const int colbase = ((warp - kEpi0) >> 2) * 128;
-    const float scale = __fmul_rn(__ldg(args.ga), __ldg(args.gb));
+    const float scale = args.ga ? __fmul_rn(__ldg(args.ga), __ldg(args.gb)) : 1.0f;
     const float g_in = __ldg(args.g_out);
     const bool g_ok = g_in > 0.0f && g_in <= FLT_MAX;
     if (!g_ok && blockIdx.x == 0 && threadIdx.x == 32 * kEpi0) set_status(args.status, NVFP4_ERR_INVALID_ARG);
@@ -808,7 +815,7 @@ __global__ void __launch_bounds__(C::kThreads, 1)
     const int colbase = ((warp - kEpi0) >> 2) * 128;
     uint8_t* buf_ptr = sEpi + (warp - kEpi0) * kEpiBufBytes;
     const uint32_t buf = smem_u32(buf_ptr);
-    const float scale = __fmul_rn(__ldg(args.ga), __ldg(args.gb));
+    const float scale = args.ga ? __fmul_rn(__ldg(args.ga), __ldg(args.gb)) : 1.0f;
     int local = 0;
     for (int u = u_first; u < u_end; u += u_step, ++local) {
       int ms, nb;
@@ -960,7 +967,7 @@ int resident_clusters() {
 template <class C>
 nvfp4_status launch(const uint8_t* a_codes, const uint8_t* a_scales, const float* g_a, const uint8_t* w_codes,
                     const uint8_t* w_scales, const float* g_w, int64_t M, int64_t N, int64_t K, void* out_bf16,
-                    int64_t ldo, cudaStream_t stream) {
+                    int64_t ldo, cudaStream_t stream, uint32_t idesc_fmt) {
   const int64_t tiles_m = (M + BM - 1) / BM, tiles_n = (N + C::BN - 1) / C::BN;
   const int64_t units = ((tiles_m + C::CM - 1) / C::CM) * tiles_n;
   if (units >= (1ll << 31)) return NVFP4_ERR_SHAPE;
@@ -970,7 +977,8 @@ nvfp4_status launch(const uint8_t* a_codes, const uint8_t* a_scales, const float
     return NVFP4_ERR_CUDA;
   const int clusters_max = resident_clusters<C>();
   if (clusters_max <= 0) return NVFP4_ERR_CUDA;
-  GemmArgs args;
+  GemmArgs args = {};
+  args.idesc_fmt = idesc_fmt;
   args.sfa = a_scales;
   args.sfb = w_scales;
   args.ga = g_a;
@@ -1041,7 +1049,8 @@ int resident_pairs() {
 template <class C, bool kSwiGLU = false>
 nvfp4_status launch_pair(const uint8_t* a_codes, const uint8_t* a_scales, const float* g_a, const uint8_t* w_codes,
                          const uint8_t* w_scales, const float* g_w, int64_t M, int64_t N, int64_t K, void* out_bf16,
-                         int64_t ldo, cudaStream_t stream, const GemmArgs* extra = nullptr) {
+                         int64_t ldo, cudaStream_t stream, const GemmArgs* extra = nullptr,
+                         uint32_t idesc_fmt = 0) {
   const int64_t tiles_m = (M + BM - 1) / BM, tiles_n = N / C::BN;
   const int64_t units = ((tiles_m + 1) / 2) * tiles_n;
   if (units >= (1ll << 31)) return NVFP4_ERR_SHAPE;
@@ -1055,6 +1064,7 @@ nvfp4_status launch_pair(const uint8_t* a_codes, const uint8_t* a_scales, const 
   if (pairs_max <= 0) return NVFP4_ERR_CUDA;
   GemmArgs args = {};
   if (extra) args = *extra;
+  args.idesc_fmt = idesc_fmt;
   args.sfa = a_scales;
   args.sfb = w_scales;
   args.ga = g_a;
@@ -1118,16 +1128,12 @@ bool use_w_resident(int64_t pair_units, int64_t K, int pairs) {
 
 using namespace nvfp4;
 
-NVFP4_API nvfp4_status nvfp4_linear(const uint8_t* a_codes, const uint8_t* a_scales, const float* g_a,
-                                    const uint8_t* w_codes, const uint8_t* w_scales, const float* g_w, int64_t M,
-                                    int64_t N, int64_t K, void* out_bf16, int64_t ldo, void* stream) {
-  if (!a_codes || !a_scales || !g_a || !w_codes || !w_scales || !g_w || !out_bf16) return NVFP4_ERR_INVALID_ARG;
-  if (M <= 0 || N <= 0 || K <= 0 || K % BK || N % 16 || ldo < N || ldo % 8) return NVFP4_ERR_SHAPE;
-  if (M >= (1ll << 31) || N >= (1ll << 31) || K >= (1ll << 31)) return NVFP4_ERR_SHAPE;
-  if (!aligned(a_codes, 16) || !aligned(w_codes, 16) || !aligned(a_scales, 16) || !aligned(w_scales, 16) ||
-      !aligned(out_bf16, 16) || !aligned(g_a, 4) || !aligned(g_w, 4))
-    return NVFP4_ERR_ALIGN;
-  cudaStream_t s = static_cast<cudaStream_t>(stream);
+namespace nvfp4 {
+namespace {
+// Kernel choice for one block-scaled linear (arguments already validated).
+nvfp4_status linear_dispatch(const uint8_t* a_codes, const uint8_t* a_scales, const float* g_a,
+                             const uint8_t* w_codes, const uint8_t* w_scales, const float* g_w, int64_t M, int64_t N,
+                             int64_t K, void* out_bf16, int64_t ldo, cudaStream_t s, uint32_t idesc_fmt) {
   const int64_t tiles_m = (M + BM - 1) / BM;
   // Measured on GB300: sharing W tiles by cluster multicast did not beat
   // independent CTAs on these shapes (the cluster waits for its slowest CTA),
@@ -1141,14 +1147,17 @@ NVFP4_API nvfp4_status nvfp4_linear(const uint8_t* a_codes, const uint8_t* a_sca
   if (NVFP4_GEMM_PAIR && N % 256 == 0 && tiles_m >= 2) {
     const int64_t pair_units = ((tiles_m + 1) / 2) * (N / 256);
     if (use_w_resident(pair_units, K, resident_pairs<PairRes, false>()))
-      return launch_pair<PairRes>(a_codes, a_scales, g_a, w_codes, w_scales, g_w, M, N, K, out_bf16, ldo, s);
+      return launch_pair<PairRes>(a_codes, a_scales, g_a, w_codes, w_scales, g_w, M, N, K, out_bf16, ldo, s,
+                                  nullptr, idesc_fmt);
     if (2 * pair_units >= resident_pairs<Pair, false>())
-      return launch_pair<Pair>(a_codes, a_scales, g_a, w_codes, w_scales, g_w, M, N, K, out_bf16, ldo, s);
+      return launch_pair<Pair>(a_codes, a_scales, g_a, w_codes, w_scales, g_w, M, N, K, out_bf16, ldo, s, nullptr,
+                               idesc_fmt);
   }
   // Single CTAs: BN = 128 (measured faster than 256 at M <= 256 on GB300).
   const int bn = NVFP4_GEMM_BN ? NVFP4_GEMM_BN : 128;
 #define NVFP4_LAUNCH(BN_, ST_, CM_) \
-  return launch<Cfg<BN_, ST_, CM_>>(a_codes, a_scales, g_a, w_codes, w_scales, g_w, M, N, K, out_bf16, ldo, s)
+  return launch<Cfg<BN_, ST_, CM_>>(a_codes, a_scales, g_a, w_codes, w_scales, g_w, M, N, K, out_bf16, ldo, s, \
+                                    idesc_fmt)
   if (bn == 256) {
     if (cm >= 4) NVFP4_LAUNCH(256, 3, 4);
     if (cm == 2) NVFP4_LAUNCH(256, 3, 2);
@@ -1158,6 +1167,35 @@ NVFP4_API nvfp4_status nvfp4_linear(const uint8_t* a_codes, const uint8_t* a_sca
   if (cm == 2) NVFP4_LAUNCH(128, 5, 2);
   NVFP4_LAUNCH(128, 5, 1);
 #undef NVFP4_LAUNCH
+}
+
+}  // namespace
+}  // namespace nvfp4
+
+NVFP4_API nvfp4_status nvfp4_linear(const uint8_t* a_codes, const uint8_t* a_scales, const float* g_a,
+                                    const uint8_t* w_codes, const uint8_t* w_scales, const float* g_w, int64_t M,
+                                    int64_t N, int64_t K, void* out_bf16, int64_t ldo, void* stream) {
+  if (!a_codes || !a_scales || !g_a || !w_codes || !w_scales || !g_w || !out_bf16) return NVFP4_ERR_INVALID_ARG;
+  if (M <= 0 || N <= 0 || K <= 0 || K % BK || N % 16 || ldo < N || ldo % 8) return NVFP4_ERR_SHAPE;
+  if (M >= (1ll << 31) || N >= (1ll << 31) || K >= (1ll << 31)) return NVFP4_ERR_SHAPE;
+  if (!aligned(a_codes, 16) || !aligned(w_codes, 16) || !aligned(a_scales, 16) || !aligned(w_scales, 16) ||
+      !aligned(out_bf16, 16) || !aligned(g_a, 4) || !aligned(g_w, 4))
+    return NVFP4_ERR_ALIGN;
+  return linear_dispatch(a_codes, a_scales, g_a, w_codes, w_scales, g_w, M, N, K, out_bf16, ldo,
+                         static_cast<cudaStream_t>(stream), 0);
+}
+
+NVFP4_API nvfp4_status mxfp4_linear(const uint8_t* a_codes, const uint8_t* a_scales, const uint8_t* w_codes,
+                                    const uint8_t* w_scales, int64_t M, int64_t N, int64_t K, void* out_bf16,
+                                    int64_t ldo, void* stream) {
+  if (!a_codes || !a_scales || !w_codes || !w_scales || !out_bf16) return NVFP4_ERR_INVALID_ARG;
+  if (M <= 0 || N <= 0 || K <= 0 || K % BK || N % 16 || ldo < N || ldo % 8) return NVFP4_ERR_SHAPE;
+  if (M >= (1ll << 31) || N >= (1ll << 31) || K >= (1ll << 31)) return NVFP4_ERR_SHAPE;
+  if (!aligned(a_codes, 16) || !aligned(w_codes, 16) || !aligned(a_scales, 16) || !aligned(w_scales, 16) ||
+      !aligned(out_bf16, 16))
+    return NVFP4_ERR_ALIGN;
+  return linear_dispatch(a_codes, a_scales, nullptr, w_codes, w_scales, nullptr, M, N, K, out_bf16, ldo,
+                         static_cast<cudaStream_t>(stream), kScaleE8M0);
 }
 
 NVFP4_API nvfp4_status nvfp4_linear_swiglu_quantize(const uint8_t* a_codes, const uint8_t* a_scales, const float* g_a,

@@ -356,6 +356,98 @@ int dynamic_capacity(int stash_iters) {
   return cache[{d, stash_iters}];
 }
 
+// ---------------------------------------------------------------------------
+// MXFP4 (Appendix A): E2M1 elements, one E8M0 scale per 32 elements, no
+// global scale; optionally each 32-element block is first rotated by
+// H_32 / sqrt(32) (the block-wise rotation applied before MXFP4 quantization,
+// Sec. 4).  One thread quantizes one block per slot; no tensor-wide pass.
+// ---------------------------------------------------------------------------
+constexpr int kMxUnroll = 2;
+constexpr uint32_t kInvSqrt32Bits = 0x3E3504F3u;  // fp32(1 / sqrt(32)), round to nearest
+
+// In-register fast Walsh-Hadamard transform of 32 values: butterflies
+// (a + b, a - b) at strides 1, 2, 4, 8, 16, each rounded to fp32, then one
+// fp32 multiplication by 1/sqrt(32) (Sylvester order: the result is x H_32 / sqrt(32)).
+__device__ __forceinline__ void hadamard32(float x[32]) {
+#pragma unroll
+  for (int h = 1; h < 32; h <<= 1) {
+#pragma unroll
+    for (int i = 0; i < 32; ++i) {
+      if ((i & h) == 0) {
+        const float a = x[i], b = x[i + h];
+        x[i] = __fadd_rn(a, b);
+        x[i + h] = __fsub_rn(a, b);
+      }
+    }
+  }
+  const float inv = __uint_as_float(kInvSqrt32Bits);
+#pragma unroll
+  for (int i = 0; i < 32; ++i) x[i] = __fmul_rn(x[i], inv);
+}
+
+// Block index b (of rows * cols/32) -> its 32 bf16 elements as fp32, the row and block-in-row.
+template <bool kMMA, bool kRotate>
+__global__ void __launch_bounds__(kThreads) mx_quantize_kernel(const uint16_t* __restrict__ x, FastDiv nb_div,
+                                                               uint32_t total_blocks, int64_t ld, bool dense,
+                                                               uint32_t rows, uint4* __restrict__ codes,
+                                                               uint8_t* __restrict__ scales) {
+  griddep_wait_and_release();
+  const uint32_t nb = nb_div.d;           // 32-element blocks per row
+  const uint32_t kgroups = nb >> 1;       // 64-element scale groups per row (MMA layout)
+  const uint32_t lane = threadIdx.x & 31;
+  const uint32_t stride = gridDim.x * blockDim.x;
+  for (uint32_t b0 = blockIdx.x * blockDim.x + (threadIdx.x & ~31u); b0 < total_blocks; b0 += stride * kMxUnroll) {
+    uint4 v[kMxUnroll][4];
+    uint32_t row[kMxUnroll], j[kMxUnroll];
+#pragma unroll
+    for (int u = 0; u < kMxUnroll; ++u) {
+      const uint32_t b = b0 + u * stride + lane;
+      row[u] = nb_div.div(b);
+      j[u] = b - row[u] * nb;
+      const int64_t off = dense ? static_cast<int64_t>(b) * 32 : static_cast<int64_t>(row[u]) * ld + j[u] * 32;
+      const uint4* src = reinterpret_cast<const uint4*>(x + off);
+      const bool live = b < total_blocks;
+#pragma unroll
+      for (int q = 0; q < 4; ++q) v[u][q] = live ? __ldg(src + q) : make_uint4(0, 0, 0, 0);
+    }
+#pragma unroll
+    for (int u = 0; u < kMxUnroll; ++u) {
+      const uint32_t b = b0 + u * stride + lane;
+      const bool live = b < total_blocks;
+      float xf[32];
+#pragma unroll
+      for (int q = 0; q < 4; ++q) unpack_bf16x8(v[u][q], xf + 8 * q);
+      if (kRotate) hadamard32(xf);
+      float amax = 0.0f;
+#pragma unroll
+      for (int i = 0; i < 32; ++i) amax = fmaxf(amax, fabsf(xf[i]));
+      // e = floor(log2 amax) - 2, clamped to [-127, 127]: from the binary
+      // exponent field E (zero and subnormal amax have E = 0 and clamp), so the
+      // E8M0 code e + 127 is max(E - 2, 0); amax < 2^128 keeps e <= 125.
+      const uint32_t E = __float_as_uint(amax) >> 23;
+      const uint32_t code = E > 2u ? E - 2u : 0u;
+      // x / 2^e = x * 2^(127 - code): 2^(127 - code) is a normal fp32 (code <= 252).
+      const float inv_scale = __uint_as_float((254u - code) << 23);
+#pragma unroll
+      for (int i = 0; i < 32; ++i) xf[i] = __fmul_rn(xf[i], inv_scale);
+      const uint4 packed = make_uint4(e2m1x8(xf), e2m1x8(xf + 8), e2m1x8(xf + 16), e2m1x8(xf + 24));
+      if (live) codes[b] = packed;
+      if (kMMA) {
+        // The 16-element-block MMA layout with each E8M0 scale stored for both
+        // halves of its block: lanes 2i, 2i+1 hold the two blocks of one
+        // 64-element group (nb is even, so a group never straddles rows).
+        uint32_t w = (code | (code << 8)) << (16 * (lane & 1));
+        w |= __shfl_xor_sync(0xffffffffu, w, 1);
+        if (live && (lane & 1) == 0)
+          *reinterpret_cast<uint32_t*>(scales + mma_scale_offset(row[u], 2 * j[u], kgroups)) = w;
+      } else if (live) {
+        scales[static_cast<uint64_t>(row[u]) * nb + j[u]] = static_cast<uint8_t>(code);
+      }
+    }
+  }
+  if (kMMA) zero_scale_padding(rows, nb * 2, scales);
+}
+
 template <bool kToMMA>
 __global__ void relayout_kernel(const uint8_t* __restrict__ src, uint8_t* __restrict__ dst, uint32_t rows,
                                 uint32_t kblocks) {
@@ -533,6 +625,35 @@ NVFP4_API nvfp4_status nvfp4_scales_relayout(const uint8_t* src, uint8_t* dst, i
   if (launch_pdl(to == NVFP4_SCALES_MMA ? relayout_kernel<true> : relayout_kernel<false>, dim3(grid_for(n, 256)),
                  dim3(256), 0, s, src, dst, static_cast<uint32_t>(rows), kblocks) != cudaSuccess)
     return NVFP4_ERR_CUDA;
+  count_launches(1);
+  return launch_status();
+}
+
+NVFP4_API size_t mxfp4_scales_bytes(int64_t rows, int64_t cols, nvfp4_scale_layout layout) {
+  if (rows < 0 || cols < 0) return 0;
+  if (layout == NVFP4_SCALES_MMA) return nvfp4_scales_bytes(rows, cols, layout);
+  return static_cast<size_t>(rows * (cols / 32));
+}
+
+NVFP4_API nvfp4_status mxfp4_quantize(const void* x_bf16, int64_t rows, int64_t cols, int64_t ld, int rotate,
+                                      uint8_t* codes, uint8_t* scales, nvfp4_scale_layout layout, void* stream) {
+  if (layout != NVFP4_SCALES_ROWMAJOR && layout != NVFP4_SCALES_MMA) return NVFP4_ERR_INVALID_ARG;
+  if (rotate != 0 && rotate != 1) return NVFP4_ERR_INVALID_ARG;
+  nvfp4_status st = check_bf16_matrix(x_bf16, rows, cols, ld, layout == NVFP4_SCALES_MMA ? 64 : 32);
+  if (st != NVFP4_OK) return st;
+  if (rows == 0 || cols == 0) return NVFP4_OK;
+  if (!codes || !scales) return NVFP4_ERR_INVALID_ARG;
+  if (!aligned(codes, 16)) return NVFP4_ERR_ALIGN;
+  const uint32_t nb = static_cast<uint32_t>(cols / 32);
+  const uint32_t total_blocks = static_cast<uint32_t>(rows * nb);
+  const int grid = grid_for(total_blocks, kThreads * kMxUnroll);
+  const bool mma = layout == NVFP4_SCALES_MMA;
+  auto kernel = mma ? (rotate ? mx_quantize_kernel<true, true> : mx_quantize_kernel<true, false>)
+                    : (rotate ? mx_quantize_kernel<false, true> : mx_quantize_kernel<false, false>);
+  const cudaError_t e = launch_pdl(kernel, dim3(grid), dim3(kThreads), 0, static_cast<cudaStream_t>(stream),
+                                   static_cast<const uint16_t*>(x_bf16), FastDiv(nb), total_blocks, ld, ld == cols,
+                                   static_cast<uint32_t>(rows), reinterpret_cast<uint4*>(codes), scales);
+  if (e != cudaSuccess) return NVFP4_ERR_CUDA;
   count_launches(1);
   return launch_status();
 }

@@ -69,6 +69,9 @@ _get_status = _sig("nvfp4_get_device_status", [ctypes.POINTER(_i32), _p])
 _status_string = _sig("nvfp4_status_string", [ctypes.c_int], ctypes.c_char_p)
 _launch_count = _sig("nvfp4_launch_count", [], ctypes.c_uint64)
 _scales_bytes = _sig("nvfp4_scales_bytes", [_i64, _i64, ctypes.c_int], _sz)
+_mx_scales_bytes = _sig("mxfp4_scales_bytes", [_i64, _i64, ctypes.c_int], _sz)
+_mx_quantize = _sig("mxfp4_quantize", [_p, _i64, _i64, _i64, ctypes.c_int, _p, _p, ctypes.c_int, _p])
+_mx_linear = _sig("mxfp4_linear", [_p, _p, _p, _p, _i64, _i64, _i64, _p, _i64, _p])
 
 
 def _stream(stream):
@@ -136,6 +139,22 @@ def nvfp4_scales_relayout(src, dst, rows, cols, from_layout, to_layout, stream=N
 def nvfp4_linear(a_codes, a_scales, g_a, w_codes, w_scales, g_w, out, M, N, K, ldo=None, stream=None):
     _check("nvfp4_linear", _linear(_ptr(a_codes), _ptr(a_scales), _ptr(g_a), _ptr(w_codes), _ptr(w_scales),
                                    _ptr(g_w), M, N, K, _ptr(out), N if ldo is None else ldo, _stream(stream)))
+
+
+def mxfp4_scales_bytes(rows, cols, layout):
+    return int(_mx_scales_bytes(rows, cols, layout))
+
+
+def mxfp4_quantize(x, codes, scales, layout=SCALES_MMA, rotate=False, stream=None):
+    """MXFP4 codes and E8M0 block scales of a bf16 [rows, cols] tensor
+    (optionally after the 32-element block rotation)."""
+    _check("mxfp4_quantize", _mx_quantize(*_mat(x), int(bool(rotate)), _ptr(codes), _ptr(scales), layout,
+                                          _stream(stream)))
+
+
+def mxfp4_linear(a_codes, a_scales, w_codes, w_scales, out, M, N, K, ldo=None, stream=None):
+    _check("mxfp4_linear", _mx_linear(_ptr(a_codes), _ptr(a_scales), _ptr(w_codes), _ptr(w_scales), M, N, K,
+                                      _ptr(out), N if ldo is None else ldo, _stream(stream)))
 
 
 def nvfp4_linear_swiglu_quantize(a_codes, a_scales, g_a, w_codes, w_scales, g_w, M, I, K, g_out,
@@ -238,6 +257,7 @@ class KVCache:
 
 EXPORTED = ["nvfp4_scales_bytes", "nvfp4_tensor_scale", "nvfp4_quantize", "nvfp4_quantize_dynamic", "nvfp4_scales_relayout", "nvfp4_linear",
             "nvfp4_linear_swiglu_quantize", "nvfp4_interleave_gate_up",
+            "mxfp4_scales_bytes", "mxfp4_quantize", "mxfp4_linear",
             "kv_append_nvfp4", "kv_append_rope_nvfp4", "nvfp4_rope_table", "decode_attention_nvfp4_workspace_size", "decode_attention_nvfp4",
             "decode_attention_nvfp4_quantize",
             "decode_attention_nvfp4_static_scratch",

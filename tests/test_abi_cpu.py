@@ -69,6 +69,28 @@ def test_argument_validation_before_launch():
     assert L.nvfp4_quantize_dynamic(p, 4, 64, 64, st, p, None, p, 1, s) == 1  # no codes
 
 
+def test_mxfp4_validation_before_launch():
+    N = lib()
+    L = N._lib
+    p = ctypes.c_void_p(0x10000)
+    odd = ctypes.c_void_p(0x10008)       # 8-B but not 16-B aligned
+    s = ctypes.c_void_p(0)
+    assert N.mxfp4_scales_bytes(130, 256, N.SCALES_ROWMAJOR) == 130 * 8
+    assert N.mxfp4_scales_bytes(130, 256, N.SCALES_MMA) == N.nvfp4_scales_bytes(130, 256, N.SCALES_MMA)
+    assert L.mxfp4_quantize(p, 4, 48, 48, 0, p, p, 0, s) == 2         # cols % 32
+    assert L.mxfp4_quantize(p, 4, 96, 96, 0, p, p, 1, s) == 2         # MMA layout needs cols % 64
+    assert L.mxfp4_quantize(p, 4, 64, 64, 2, p, p, 1, s) == 1         # rotate must be 0 or 1
+    assert L.mxfp4_quantize(p, 4, 64, 64, 0, p, p, 5, s) == 1         # bad layout enum
+    assert L.mxfp4_quantize(odd, 4, 64, 64, 0, p, p, 1, s) == 3       # x alignment
+    assert L.mxfp4_quantize(p, 4, 64, 64, 0, odd, p, 1, s) == 3       # codes 16-B aligned
+    assert L.mxfp4_quantize(p, 4, 64, 64, 0, None, p, 1, s) == 1      # no codes
+    assert L.mxfp4_quantize(None, 0, 64, 64, 0, None, None, 1, s) == 0   # empty: nothing to do
+    assert L.mxfp4_linear(None, p, p, p, 128, 128, 256, p, 128, s) == 1
+    assert L.mxfp4_linear(p, p, p, p, 128, 128, 192, p, 128, s) == 2  # K % 256
+    assert L.mxfp4_linear(p, p, p, p, 128, 120, 256, p, 128, s) == 2  # N % 16
+    assert L.mxfp4_linear(p, odd, p, p, 128, 128, 256, p, 128, s) == 3
+
+
 def test_kv_and_attention_validation():
     N = lib()
     import torch  # noqa: F401  (struct only; no device memory)

@@ -1,0 +1,172 @@
+"""GPU parity of the MXFP4 format variant: the quantizer (with and without the
+32-element block rotation) bit-exact against the CPU oracle, and the MXFP4
+linear against the oracle's fp64 product of identical dequantized operands."""
+import numpy as np
+import pytest
+import torch
+
+from _util import assert_close, f32, lib, u8
+from oracle import mxfp4_oracle as X
+from oracle import nvfp4_oracle as O
+from paper_2606_15682_gb300 import synth
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def N():
+    assert torch.cuda.is_available(), "GPU tests need a CUDA device"
+    return lib()
+
+
+def gpu_mx_quantize(N, x, layout, rotate):
+    rows, cols = x.shape
+    codes = torch.full((rows, cols // 2), 0xEE, dtype=torch.uint8, device="cuda")
+    scales = torch.full((N.mxfp4_scales_bytes(rows, cols, layout),), 0xEE, dtype=torch.uint8, device="cuda")
+    N.mxfp4_quantize(x, codes, scales, layout=layout, rotate=rotate)
+    torch.cuda.synchronize()
+    assert N.nvfp4_get_device_status() == 0
+    return codes, scales
+
+
+def check_mx_quantize(N, x_bf16, layout, rotate, rows_sample=None, ld=None):
+    rows, cols = x_bf16.shape
+    if ld is None:
+        x = x_bf16.cuda()
+    else:
+        buf = torch.zeros(rows, ld, dtype=torch.bfloat16, device="cuda")
+        buf[:, :cols] = x_bf16.cuda()
+        x = buf[:, :cols]
+    codes, scales = gpu_mx_quantize(N, x, layout, rotate)
+    sel = np.arange(rows) if rows_sample is None else np.asarray(rows_sample)
+    assert sel.min() >= 0 and sel.max() < rows
+    rc, rs = X.quantize_mx(f32(x_bf16[torch.as_tensor(sel)]), rotate=rotate)
+    gc = u8(codes)[sel]
+    gs = u8(scales)
+    gs = gs.reshape(rows, cols // 32)[sel] if layout == 0 else X.mx_scales_from_mma(gs, rows, cols)[sel]
+    bad = np.argwhere(gc != rc)
+    assert bad.size == 0, f"{len(bad)} code bytes differ, first at {bad[:3].tolist()}"
+    assert np.array_equal(gs, rs)
+    if layout == 1 and rows % 128:
+        pad = np.setdiff1d(np.arange(O.mma_scale_bytes(rows, cols)), O._mma_offsets(rows, cols // 16).ravel())
+        assert not u8(scales)[pad].any(), "padding rows of the MMA scale layout must be zero"
+    return codes, scales
+
+
+@pytest.mark.parametrize("rotate", [False, True], ids=["plain", "rotated"])
+@pytest.mark.parametrize("layout", [0, 1], ids=["rowmajor", "mma"])
+@pytest.mark.parametrize("rows,cols", [(1, 64), (130, 256), (257, 1536), (64, 8960)])
+def test_mx_quantize_matches_oracle(N, rows, cols, layout, rotate):
+    x = synth.activation(rows, cols, 7000 + rows + cols, outlier_frac=0.01)
+    check_mx_quantize(N, x, layout, rotate)
+
+
+@pytest.mark.parametrize("rotate", [False, True], ids=["plain", "rotated"])
+def test_mx_quantize_padded_rows_and_rowmajor_32(N, rotate):
+    x = synth.activation(33, 96, 7101, outlier_frac=0.05)
+    check_mx_quantize(N, x, 0, rotate, ld=136)          # cols % 64 != 0: row-major only; padded leading dim
+    x = synth.activation(200, 512, 7102, outlier_frac=0.02)
+    check_mx_quantize(N, x, 1, rotate, ld=520)
+
+
+@pytest.mark.parametrize("rotate", [False, True], ids=["plain", "rotated"])
+def test_mx_quantize_edge_values(N, rotate):
+    """Zero blocks, signed zeros, bf16 subnormals, huge and tiny magnitudes,
+    exact E2M1 grid values and ties, saturation between 6 and 8 scales."""
+    g = torch.Generator().manual_seed(7200)
+    x = torch.randn(16, 256, generator=g)
+    x[0] = 0.0
+    x[1] = -0.0
+    x[2] = torch.randn(256, generator=g) * 1e-39            # bf16 subnormals
+    x[3] = torch.randn(256, generator=g) * 1e36            # large, and a rotated block sum stays finite
+    x[4, :32] = torch.tensor([6.0, 0.25, 0.75, 1.25, 1.75, 2.5, 3.5, 5.0] * 4)
+    x[5, :32] = torch.tensor([7.5, -7.9, 1.0, -0.0] * 8)
+    x[6] = torch.randn(256, generator=g) * 1e-38
+    x[6, ::32] = 1e-37                                     # amax near the bottom of E8M0's range
+    x[7, :32] = 2.0 ** -127
+    x[8, ::2] = 0.0
+    x = x.to(torch.bfloat16)
+    for layout in (0, 1):
+        check_mx_quantize(N, x, layout, rotate)
+
+
+def test_mx_quantize_full_size_sampled(N):
+    """The 32B prefill down projection's input (8192 x 27648), in the launch
+    configuration of the bench: sampled rows against the oracle."""
+    M, K = 8192, 27648
+    x = synth.activation(M, K, 7300, outlier_frac=0.01, device="cuda")
+    rows = np.unique(np.r_[0:16, 4096:4112, M - 16:M])
+    for rotate in (False, True):
+        codes, scales = gpu_mx_quantize(N, x, 1, rotate)
+        rc, rs = X.quantize_mx(f32(x[torch.as_tensor(rows, device="cuda")]), rotate=rotate)
+        assert np.array_equal(u8(codes[torch.as_tensor(rows, device="cuda")]), rc)
+        assert np.array_equal(X.mx_scales_from_mma(u8(scales), M, K)[rows], rs)
+
+
+def test_mx_quantize_empty_is_noop(N):
+    x = torch.empty(0, 64, dtype=torch.bfloat16, device="cuda")
+    N.mxfp4_quantize(x, None, None)
+    torch.cuda.synchronize()
+    assert N.nvfp4_get_device_status() == 0
+
+
+def run_mx_linear(N, a_codes, a_scales_rm, w_codes, w_scales_rm, M, Nn, K, ldo=None):
+    dev = "cuda"
+    ac = torch.from_numpy(a_codes).to(dev)
+    wc = torch.from_numpy(w_codes).to(dev)
+    asf = torch.from_numpy(X.mx_scales_to_mma(a_scales_rm)).to(dev)
+    wsf = torch.from_numpy(X.mx_scales_to_mma(w_scales_rm)).to(dev)
+    ldo = Nn if ldo is None else ldo
+    out = torch.full((M, ldo), float("nan"), dtype=torch.bfloat16, device=dev)
+    N.mxfp4_linear(ac, asf, wc, wsf, out, M, Nn, K, ldo=ldo)
+    torch.cuda.synchronize()
+    assert N.nvfp4_get_device_status() == 0
+    return out
+
+
+@pytest.mark.parametrize("M,Nn,K", [(128, 128, 256), (1, 16, 256), (130, 144, 512), (257, 384, 1024),
+                                    # N % 256 == 0: 256 x 256 CTA-pair tiles (enough of them)
+                                    (2048, 1280, 1024),
+                                    # more pair tiles than pairs with 6 k-blocks: the W-resident form
+                                    (2048, 2560, 1536)])
+def test_mx_linear_random_operands(N, M, Nn, K):
+    """Seeded random codes and E8M0 scales (isolates the GEMM from the quantizer)."""
+    gen = torch.Generator().manual_seed(7400 + M + Nn + K)
+    ac = torch.randint(0, 256, (M, K // 2), generator=gen, dtype=torch.int32).to(torch.uint8).numpy()
+    wc = torch.randint(0, 256, (Nn, K // 2), generator=gen, dtype=torch.int32).to(torch.uint8).numpy()
+    asf = torch.randint(118, 134, (M, K // 32), generator=gen, dtype=torch.int32).to(torch.uint8).numpy()
+    wsf = torch.randint(110, 126, (Nn, K // 32), generator=gen, dtype=torch.int32).to(torch.uint8).numpy()
+    out = run_mx_linear(N, ac, asf, wc, wsf, M, Nn, K)
+    assert_close(f32(out), X.linear_mx(ac, asf, wc, wsf), what=f"mxfp4 linear {M}x{Nn}x{K}")
+
+
+@pytest.mark.parametrize("rotate", [False, True], ids=["plain", "rotated"])
+def test_mx_linear_on_workload_operands(N, rotate):
+    """The 1.5B prefill qkv shape (2048 x 2048 x 1536) from bf16 activations and
+    weights quantized by the oracle (rotated along K on both sides when asked):
+    the GPU product matches the oracle's, and with the rotation both stay as
+    close to the unquantized product as the oracle's pipeline is."""
+    a, w = synth.linear_inputs("qwen1.5b_prefill_linears_m2048", "qkv")
+    ac, asf = X.quantize_mx(f32(a), rotate=rotate)
+    wc, wsf = X.quantize_mx(f32(w), rotate=rotate)
+    M, K = a.shape
+    Nn = w.shape[0]
+    out = run_mx_linear(N, ac, asf, wc, wsf, M, Nn, K)
+    ref = X.linear_mx(ac, asf, wc, wsf)
+    assert_close(f32(out), ref, what="mxfp4 qkv")
+    exact = f32(a).astype(np.float64) @ f32(w).astype(np.float64).T
+    e_orc = np.abs(ref - exact).max() / np.abs(exact).max()
+    e_gpu = np.abs(f32(out) - exact).max() / np.abs(exact).max()
+    assert e_gpu <= 1.05 * e_orc + 4e-3
+
+
+def test_mx_linear_padded_output(N):
+    gen = torch.Generator().manual_seed(7500)
+    M, Nn, K = 130, 144, 512
+    ac = torch.randint(0, 256, (M, K // 2), generator=gen, dtype=torch.int32).to(torch.uint8).numpy()
+    wc = torch.randint(0, 256, (Nn, K // 2), generator=gen, dtype=torch.int32).to(torch.uint8).numpy()
+    asf = torch.randint(120, 130, (M, K // 32), generator=gen, dtype=torch.int32).to(torch.uint8).numpy()
+    wsf = torch.randint(120, 130, (Nn, K // 32), generator=gen, dtype=torch.int32).to(torch.uint8).numpy()
+    out = run_mx_linear(N, ac, asf, wc, wsf, M, Nn, K, ldo=168)
+    assert_close(f32(out[:, :Nn]), X.linear_mx(ac, asf, wc, wsf), what="mxfp4 padded ldo")
+    assert torch.isnan(out[:, Nn:].float()).all(), "columns beyond N must be left untouched"
