@@ -367,6 +367,66 @@ def run_ours(args, rank, world):
         del lw, g
         torch.cuda.empty_cache()
 
+    # ---------------- MXFP4 W4A4 (the format variant): per linear, the activation
+    # rotated by H_32/sqrt(32) per 32-element block and MXFP4-quantized in one
+    # launch (no tensor-wide scale, so no amax pass), then the MXFP4 GEMM
+    # against W rotated and quantized once.
+    def build_mx_layers(wl):
+        Mw = synth.WORKLOADS[wl]["M"]
+        out_layers, out_flops = [], 0
+        for name, (Nn, K) in synth.WORKLOADS[wl]["linears"].items():
+            a, W = synth.linear_inputs(wl, name, device=dev)
+            wc = torch.empty(Nn, K // 2, dtype=torch.uint8, device=dev)
+            ws = torch.empty(N.mxfp4_scales_bytes(Nn, K, N.SCALES_MMA), dtype=torch.uint8, device=dev)
+            N.mxfp4_quantize(W, wc, ws, N.SCALES_MMA, rotate=True)
+            del W
+            out_layers.append(dict(name=name, N=Nn, K=K, a=a, wc=wc, ws=ws,
+                                   ac=torch.empty(Mw, K // 2, dtype=torch.uint8, device=dev),
+                                   asf=torch.empty(N.mxfp4_scales_bytes(Mw, K, N.SCALES_MMA), dtype=torch.uint8,
+                                                   device=dev),
+                                   out=torch.empty(Mw, Nn, dtype=torch.bfloat16, device=dev),
+                                   ev=[torch.cuda.Event(enable_timing=True) for _ in range(3)]))
+            out_flops += 2 * Mw * Nn * K
+        torch.cuda.synchronize()
+        return Mw, out_layers, out_flops
+
+    def mx_step(lw, Mw, record=False):
+        for L in lw:
+            if record:
+                L["ev"][0].record()
+            N.mxfp4_quantize(L["a"], L["ac"], L["asf"], N.SCALES_MMA, rotate=True)
+            if record:
+                L["ev"][1].record()
+            N.mxfp4_linear(L["ac"], L["asf"], L["wc"], L["ws"], L["out"], Mw, L["N"], L["K"])
+            if record:
+                L["ev"][2].record()
+
+    mx = {}
+    for wl in (GEMM_WL, "qwen32b_prefill_linears_m8192"):
+        Mw, lw, fw = build_mx_layers(wl)
+        g = graph_of(lambda lw=lw, Mw=Mw: mx_step(lw, Mw))
+        ms_w = statistics.mean(timed_loop(g.replay, other_steps, args.warmup))
+        q_ms, g_ms = {}, {}
+        with torch.cuda.stream(stream):
+            for _ in range(3):
+                flush_buf.zero_()
+                torch.cuda._sleep(2_000_000)
+                mx_step(lw, Mw, record=True)
+                stream.synchronize()
+                for L in lw:
+                    q_ms.setdefault(L["name"], []).append(L["ev"][0].elapsed_time(L["ev"][1]))
+                    g_ms.setdefault(L["name"], []).append(L["ev"][1].elapsed_time(L["ev"][2]))
+        q_bytes = {L["name"]: Mw * L["K"] * (2 + 0.5 + 1 / 16) for L in lw}
+        mx[wl] = {"step": "per linear: rotate (H_32 blocks) + MXFP4 quantize activation (one launch) + MXFP4 GEMM",
+                  "ms_per_step": ms_w, "tflops": fw / (ms_w * 1e-3) / 1e12,
+                  "gemm_us": {k: 1e3 * statistics.median(v) for k, v in g_ms.items()},
+                  "gemm_roofline": {L["name"]: roofline_of(2 * Mw * L["N"] * L["K"], gemm_bytes(Mw, L["N"], L["K"]),
+                                                           statistics.median(g_ms[L["name"]])) for L in lw},
+                  "quantize_us": {k: 1e3 * statistics.median(v) for k, v in q_ms.items()},
+                  "quantize_gbs": {k: q_bytes[k] / (statistics.median(v) * 1e-3) / 1e9 for k, v in q_ms.items()}}
+        del lw, g
+        torch.cuda.empty_cache()
+
     # ---------------- decode attention over the NVFP4 cache
     aw = synth.WORKLOADS[ATTN_WL]
     Bq, hq, hkv, T = aw["batch"], aw["num_q_heads"], aw["num_kv_heads"], aw["context"]
@@ -487,6 +547,7 @@ def run_ours(args, rank, world):
             "gpu_launches": attn_launches * args.steps,
         },
         "other_workloads": other,
+        "mxfp4_w4a4": mx,
         "clocks": sampler.summary(),
     }
     if rank == 0 and not args.no_cpu_baseline:

@@ -5,6 +5,8 @@
     python -m paper_2606_15682_gb300.cases quantize_dynamic --workload qwen32b_prefill_linears_m8192 --linear down
     python -m paper_2606_15682_gb300.cases attention --batch 64 --context 16384
     python -m paper_2606_15682_gb300.cases gemm_swiglu --workload qwen32b_prefill_linears_m8192
+    python -m paper_2606_15682_gb300.cases mx_gemm --workload qwen32b_prefill_linears_m8192 --linear down
+    python -m paper_2606_15682_gb300.cases mx_quantize --workload qwen32b_prefill_linears_m8192 --linear down --rotate
 
 Inputs are seeded synthetic tensors (paper_2606_15682_gb300.synth); for the
 attention case the cache is filled with seeded random codes and scales
@@ -49,7 +51,8 @@ def _time(fn, iters):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("kernel", choices=["gemm", "gemm_swiglu", "quantize", "quantize_dynamic", "tensor_scale",
-                                       "attention"])
+                                       "attention", "mx_gemm", "mx_quantize"])
+    ap.add_argument("--rotate", action="store_true", help="MXFP4: 32-element block rotation before quantizing")
     ap.add_argument("--workload", default="qwen1.5b_prefill_linears_m2048")
     ap.add_argument("--linear", default="gate_up")
     ap.add_argument("--batch", type=int, default=64)
@@ -88,6 +91,30 @@ def main():
         print(f"gemm_swiglu {a.workload} {M}x{2 * I}x{K}: fused {ms_f * 1e3:.1f} us "
               f"({2 * M * 2 * I * K / ms_f / 1e9:.1f} TFLOP/s); bf16 GEMM + quantize of h {ms_u * 1e3:.1f} us "
               f"(SwiGLU itself not included)")
+    elif a.kernel in ("mx_gemm", "mx_quantize"):
+        x, W = synth.linear_inputs(a.workload, a.linear, device=dev)
+        M, K = x.shape
+        Nn = W.shape[0]
+
+        def mx(t):
+            c = torch.empty(t.shape[0], t.shape[1] // 2, dtype=torch.uint8, device=dev)
+            sc = torch.empty(N.mxfp4_scales_bytes(t.shape[0], t.shape[1], N.SCALES_MMA), dtype=torch.uint8, device=dev)
+            return c, sc
+        ac, asf = mx(x)
+        if a.kernel == "mx_quantize":
+            ms = _time(lambda: N.mxfp4_quantize(x, ac, asf, N.SCALES_MMA, rotate=a.rotate), a.iters)
+            byt = M * K * (2 + 0.5 + 1 / 16)
+            print(f"mx_quantize{' (rotated)' if a.rotate else ''} {a.workload}/{a.linear} {M}x{K}: "
+                  f"{ms * 1e3:.1f} us, {byt / ms / 1e6:.0f} GB/s")
+        else:
+            wc, wsf = mx(W)
+            N.mxfp4_quantize(x, ac, asf, N.SCALES_MMA, rotate=a.rotate)
+            N.mxfp4_quantize(W, wc, wsf, N.SCALES_MMA, rotate=a.rotate)
+            del W
+            out = torch.empty(M, Nn, dtype=torch.bfloat16, device=dev)
+            ms = _time(lambda: N.mxfp4_linear(ac, asf, wc, wsf, out, M, Nn, K), a.iters)
+            print(f"mx_gemm {a.workload}/{a.linear} {M}x{Nn}x{K}: {ms * 1e3:.1f} us, "
+                  f"{2 * M * Nn * K / ms / 1e9:.1f} TFLOP/s")
     elif a.kernel in ("gemm", "quantize", "quantize_dynamic", "tensor_scale"):
         x, W = synth.linear_inputs(a.workload, a.linear, device=dev)
         M, K = x.shape
