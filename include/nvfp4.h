@@ -240,6 +240,27 @@ nvfp4_status mxfp4_linear(const uint8_t* a_codes, const uint8_t* a_scales, const
                           const uint8_t* w_scales, int64_t M, int64_t N, int64_t K, void* out_bf16,
                           int64_t ldo, void* stream);
 
+/*
+ * nvfp4_linear_swiglu_quantize for MXFP4 operands: the gate_up projection
+ * with h[m, i] = SiLU(G[m, i]) * U[m, i] (the fp32 accumulators; SiLU as in
+ * nvfp4_linear_swiglu_quantize) MXFP4-quantized in the epilogue by the recipe
+ * of mxfp4_quantize, as the down projection's A operand.  E8M0 scales are
+ * local to each 32-element block, so no output scale is needed.  rotate = 1
+ * rotates each 32-element block of h by H_32 / sqrt(32) first (the down
+ * weight's K dimension must be rotated the same way).
+ *   a_codes, a_scales : MXFP4 A operand, MMA-layout scales.
+ *   w_codes, w_scales : the [2I, K] MXFP4 gate/up weight, rows interleaved in
+ *                       blocks of 16 as for nvfp4_linear_swiglu_quantize.
+ *   out_codes         : [M, I/2] bytes, 16-B aligned.
+ *   out_scales        : mxfp4_scales_bytes(M, I, NVFP4_SCALES_MMA) bytes, 4-B
+ *                       aligned; padding rows are written as zeros.
+ * I % 128 == 0, K % 256 == 0, M, I, K > 0 (SHAPE); rotate not 0/1 -> INVALID_ARG.
+ */
+nvfp4_status mxfp4_linear_swiglu_quantize(const uint8_t* a_codes, const uint8_t* a_scales,
+                                          const uint8_t* w_codes, const uint8_t* w_scales, int64_t M,
+                                          int64_t I, int64_t K, int rotate, uint8_t* out_codes,
+                                          uint8_t* out_scales, void* stream);
+
 /* Element grid of the KV cache (the block scales are E4M3 per 16 either way). */
 typedef enum {
   /* E2M1, the NVFP4 element {0, 0.5, 1, 1.5, 2, 3, 4, 6} (the B200 deployment's

@@ -26,9 +26,10 @@ recipe; the readings used here are:
   butterflies (a + b, a - b) at strides 1, 2, 4, 8, 16, each result rounded to
   fp32, then one fp32 multiplication by fp32(1 / sqrt(32)).  ``rotate_blocks``
   is the fp64 definition (the matrix product) that pins it.
-* linear: D = A_hat W_hat^T in fp64 on the dequantized operands, as for NVFP4.
+* linear: D = A_hat W_hat^T in fp64 on the dequantized operands, as for NVFP4;
+  the fused gate_up form h = SiLU(G) * U (fp64), quantized from fp32 h.
 
-Parity status: every function here is pinned by ``tests/test_oracle_pins.py``
+Parity status: every function here is pinned by ``tests/test_oracle_pins_mx.py``
 (the E8M0 table, closed forms of the shared exponent, exact round trips,
 brute force over E2M1 grids, the Hadamard matrix's algebra); none is
 "parity unpinned".
@@ -37,7 +38,7 @@ from __future__ import annotations
 
 import numpy as np
 
-from oracle.nvfp4_oracle import e2m1_decode, e2m1_encode, scales_to_mma, scales_from_mma, unpack_codes
+from oracle.nvfp4_oracle import e2m1_decode, e2m1_encode, scales_to_mma, scales_from_mma, silu, unpack_codes
 
 MX_BLOCK = 32           # elements per E8M0 scale (Appendix A)
 E2M1_EMAX = 2           # exponent of E2M1's largest power of two (4 = 2**2)
@@ -164,3 +165,17 @@ def linear_mx_rows(a_codes, a_scales, w_codes, w_scales, rows):
     """The reference restricted to some output rows (full-size sampled checks)."""
     rows = np.asarray(rows)
     return dequantize_mx(a_codes[rows], a_scales[rows]) @ dequantize_mx(w_codes, w_scales).T
+
+
+def linear_swiglu_quantize_mx(a_codes, a_scales, wg_codes, wg_scales, wu_codes, wu_scales, rotate=False, rows=None):
+    """The down projection's input from MXFP4 operands: h = SiLU(A W_gate^T) *
+    (A W_up^T) in fp64, then MXFP4-quantized (``quantize_mx``, optionally after
+    the block rotation) from h rounded to fp32.  ``rows`` restricts to some
+    rows of A.  Returns (h fp64, codes, scales)."""
+    if rows is not None:
+        a_codes, a_scales = a_codes[np.asarray(rows)], a_scales[np.asarray(rows)]
+    G = linear_mx(a_codes, a_scales, wg_codes, wg_scales)
+    U = linear_mx(a_codes, a_scales, wu_codes, wu_scales)
+    h = silu(G) * U
+    codes, scales = quantize_mx(h.astype(np.float32), rotate=rotate)
+    return h, codes, scales

@@ -7,6 +7,7 @@
     python -m paper_2606_15682_gb300.cases gemm_swiglu --workload qwen32b_prefill_linears_m8192
     python -m paper_2606_15682_gb300.cases mx_gemm --workload qwen32b_prefill_linears_m8192 --linear down
     python -m paper_2606_15682_gb300.cases mx_quantize --workload qwen32b_prefill_linears_m8192 --linear down --rotate
+    python -m paper_2606_15682_gb300.cases mx_gemm_swiglu --workload qwen32b_prefill_linears_m8192 --rotate
 
 Inputs are seeded synthetic tensors (paper_2606_15682_gb300.synth); for the
 attention case the cache is filled with seeded random codes and scales
@@ -51,7 +52,7 @@ def _time(fn, iters):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("kernel", choices=["gemm", "gemm_swiglu", "quantize", "quantize_dynamic", "tensor_scale",
-                                       "attention", "mx_gemm", "mx_quantize"])
+                                       "attention", "mx_gemm", "mx_quantize", "mx_gemm_swiglu"])
     ap.add_argument("--rotate", action="store_true", help="MXFP4: 32-element block rotation before quantizing")
     ap.add_argument("--workload", default="qwen1.5b_prefill_linears_m2048")
     ap.add_argument("--linear", default="gate_up")
@@ -90,6 +91,38 @@ def main():
         ms_u = _time(unfused, a.iters)
         print(f"gemm_swiglu {a.workload} {M}x{2 * I}x{K}: fused {ms_f * 1e3:.1f} us "
               f"({2 * M * 2 * I * K / ms_f / 1e9:.1f} TFLOP/s); bf16 GEMM + quantize of h {ms_u * 1e3:.1f} us "
+              f"(SwiGLU itself not included)")
+    elif a.kernel == "mx_gemm_swiglu":
+        # MXFP4 gate_up with SwiGLU + MXFP4 quantization of h in the epilogue,
+        # against the MXFP4 GEMM with bf16 output followed by mxfp4_quantize of h.
+        x, W = synth.linear_inputs(a.workload, "gate_up", device=dev)
+        M, K = x.shape
+        I = W.shape[0] // 2
+        Wi = torch.empty_like(W)
+        N.nvfp4_interleave_gate_up(W[:I].contiguous(), W[I:].contiguous(), Wi)
+        del W
+
+        def mxq(t):
+            c = torch.empty(t.shape[0], t.shape[1] // 2, dtype=torch.uint8, device=dev)
+            sc = torch.empty(N.mxfp4_scales_bytes(t.shape[0], t.shape[1], N.SCALES_MMA), dtype=torch.uint8, device=dev)
+            N.mxfp4_quantize(t, c, sc, N.SCALES_MMA, rotate=a.rotate)
+            return c, sc
+        ac, asf = mxq(x)
+        wc, wsf = mxq(Wi)
+        del Wi
+        qc = torch.empty(M, I // 2, dtype=torch.uint8, device=dev)
+        qs = torch.empty(N.mxfp4_scales_bytes(M, I, N.SCALES_MMA), dtype=torch.uint8, device=dev)
+        ms_f = _time(lambda: N.mxfp4_linear_swiglu_quantize(ac, asf, wc, wsf, M, I, K, qc, qs, rotate=a.rotate),
+                     a.iters)
+        out = torch.empty(M, 2 * I, dtype=torch.bfloat16, device=dev)
+        h = out[:, :I].contiguous()
+
+        def unfused():
+            N.mxfp4_linear(ac, asf, wc, wsf, out, M, 2 * I, K)
+            N.mxfp4_quantize(h, qc, qs, N.SCALES_MMA, rotate=a.rotate)
+        ms_u = _time(unfused, a.iters)
+        print(f"mx_gemm_swiglu{' (rotated)' if a.rotate else ''} {a.workload} {M}x{2 * I}x{K}: fused {ms_f * 1e3:.1f} us "
+              f"({2 * M * 2 * I * K / ms_f / 1e9:.1f} TFLOP/s); bf16 GEMM + MXFP4 quantize of h {ms_u * 1e3:.1f} us "
               f"(SwiGLU itself not included)")
     elif a.kernel in ("mx_gemm", "mx_quantize"):
         x, W = synth.linear_inputs(a.workload, a.linear, device=dev)

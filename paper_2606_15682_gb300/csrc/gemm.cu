@@ -168,6 +168,9 @@ struct GemmArgs {
   uint8_t* q_codes;   // [M, N/4] bytes: N/2 SwiGLU outputs per row
   uint8_t* q_scales;  // MMA layout for [M, N/2]
   const float* g_out;
+  // Quantization of the fused output: 0 NVFP4 with the static scale g_out,
+  // 1 MXFP4, 2 MXFP4 after the H_32 block rotation.
+  uint32_t q_mode;
 };
 
 template <class C>
@@ -748,7 +751,7 @@ __global__ void __launch_bounds__(C::kThreads, 1)
     const int quarter = warp & 3;
     const int colbase = ((warp - kEpi0) >> 2) * 128;
     const float scale = args.ga ? __fmul_rn(__ldg(args.ga), __ldg(args.gb)) : 1.0f;
-    const float g_in = __ldg(args.g_out);
+    const float g_in = args.q_mode == 0 ? __ldg(args.g_out) : 1.0f;
     const bool g_ok = g_in > 0.0f && g_in <= FLT_MAX;
     if (!g_ok && blockIdx.x == 0 && threadIdx.x == 32 * kEpi0) set_status(args.status, NVFP4_ERR_INVALID_ARG);
     const float g = g_ok ? g_in : 1.0f, six_g = __fmul_rn(6.0f, g);
@@ -778,24 +781,56 @@ __global__ void __launch_bounds__(C::kThreads, 1)
       const uint32_t row = static_cast<uint32_t>(mb * BM + quarter * 32 + lane);
       const uint32_t oc0 = static_cast<uint32_t>(nb) * (BN / 2) + static_cast<uint32_t>(colbase / 2);
       uint32_t codes[8], sc = 0;
+      if (args.q_mode == 0) {
 #pragma unroll
-      for (int c = 0; c < 4; ++c) {
-        float h[16];
-        float amax = 0.0f;
+        for (int c = 0; c < 4; ++c) {
+          float h[16];
+          float amax = 0.0f;
 #pragma unroll
-        for (int i = 0; i < 16; ++i) {
-          // SiLU(x) = x sigmoid(x) = x/2 (1 + tanh(x/2)): one MUFU operation.
-          const float half_g = __uint_as_float(r[32 * c + i]) * (0.5f * scale);
-          const float up = __uint_as_float(r[32 * c + 16 + i]) * scale;
-          h[i] = fmaf(half_g, tanh_approx(half_g), half_g) * up;
-          amax = fmaxf(amax, fabsf(h[i]));
+          for (int i = 0; i < 16; ++i) {
+            // SiLU(x) = x sigmoid(x) = x/2 (1 + tanh(x/2)): one MUFU operation.
+            const float half_g = __uint_as_float(r[32 * c + i]) * (0.5f * scale);
+            const float up = __uint_as_float(r[32 * c + 16 + i]) * scale;
+            h[i] = fmaf(half_g, tanh_approx(half_g), half_g) * up;
+            amax = fmaxf(amax, fabsf(h[i]));
+          }
+          const BlockScale bs = block_scale(amax, g, six_g);
+#pragma unroll
+          for (int i = 0; i < 16; ++i) h[i] = __fmul_rn(h[i], bs.mult);
+          codes[2 * c] = g_ok ? e2m1x8(h) : 0u;
+          codes[2 * c + 1] = g_ok ? e2m1x8(h + 8) : 0u;
+          sc |= (g_ok ? bs.code : 0u) << (8 * c);
         }
-        const BlockScale bs = block_scale(amax, g, six_g);
+      } else {
+        // MXFP4: two TMEM loads give 32 consecutive outputs, one 32-element
+        // block (optionally rotated by H_32 / sqrt(32)) with one E8M0 scale,
+        // stored for both 16-element halves in the MMA scale word.
 #pragma unroll
-        for (int i = 0; i < 16; ++i) h[i] = __fmul_rn(h[i], bs.mult);
-        codes[2 * c] = g_ok ? e2m1x8(h) : 0u;
-        codes[2 * c + 1] = g_ok ? e2m1x8(h + 8) : 0u;
-        sc |= (g_ok ? bs.code : 0u) << (8 * c);
+        for (int j = 0; j < 2; ++j) {
+          float h[32];
+#pragma unroll
+          for (int cc = 0; cc < 2; ++cc) {
+#pragma unroll
+            for (int i = 0; i < 16; ++i) {
+              const float half_g = __uint_as_float(r[32 * (2 * j + cc) + i]) * (0.5f * scale);
+              const float up = __uint_as_float(r[32 * (2 * j + cc) + 16 + i]) * scale;
+              h[16 * cc + i] = fmaf(half_g, tanh_approx(half_g), half_g) * up;
+            }
+          }
+          if (args.q_mode == 2) hadamard32(h);
+          float amax = 0.0f;
+#pragma unroll
+          for (int i = 0; i < 32; ++i) amax = fmaxf(amax, fabsf(h[i]));
+          const uint32_t code = mx_scale_code(amax);
+          const float inv = mx_inv_scale(code);
+#pragma unroll
+          for (int i = 0; i < 32; ++i) h[i] = __fmul_rn(h[i], inv);
+          codes[4 * j] = e2m1x8(h);
+          codes[4 * j + 1] = e2m1x8(h + 8);
+          codes[4 * j + 2] = e2m1x8(h + 16);
+          codes[4 * j + 3] = e2m1x8(h + 24);
+          sc |= (code | (code << 8)) << (16 * j);
+        }
       }
       if (mb < args.tiles_m) {
         // Scales for every row of the 128-row tile (rows past M hold zeros: A's
@@ -1219,6 +1254,30 @@ NVFP4_API nvfp4_status nvfp4_linear_swiglu_quantize(const uint8_t* a_codes, cons
                                       static_cast<cudaStream_t>(stream), &extra);
   return launch_pair<PairCfg<NVFP4_GEMM_PAIR_STAGES>, true>(a_codes, a_scales, g_a, w_codes, w_scales, g_w, M, 2 * I,
                                                            K, nullptr, 0, static_cast<cudaStream_t>(stream), &extra);
+}
+
+NVFP4_API nvfp4_status mxfp4_linear_swiglu_quantize(const uint8_t* a_codes, const uint8_t* a_scales,
+                                                    const uint8_t* w_codes, const uint8_t* w_scales, int64_t M,
+                                                    int64_t I, int64_t K, int rotate, uint8_t* out_codes,
+                                                    uint8_t* out_scales, void* stream) {
+  if (!a_codes || !a_scales || !w_codes || !w_scales || !out_codes || !out_scales) return NVFP4_ERR_INVALID_ARG;
+  if (rotate != 0 && rotate != 1) return NVFP4_ERR_INVALID_ARG;
+  if (M <= 0 || I <= 0 || K <= 0 || K % BK || I % 128) return NVFP4_ERR_SHAPE;
+  if (M >= (1ll << 31) || 2 * I >= (1ll << 31) || K >= (1ll << 31)) return NVFP4_ERR_SHAPE;
+  if (!aligned(a_codes, 16) || !aligned(w_codes, 16) || !aligned(a_scales, 16) || !aligned(w_scales, 16) ||
+      !aligned(out_codes, 16) || !aligned(out_scales, 4))
+    return NVFP4_ERR_ALIGN;
+  GemmArgs extra = {};
+  extra.q_codes = out_codes;
+  extra.q_scales = out_scales;
+  extra.q_mode = rotate ? 2u : 1u;
+  const int64_t pair_units = ((M + 2 * BM - 1) / (2 * BM)) * (2 * I / 256);
+  if (use_w_resident(pair_units, K, resident_pairs<PairRes, true>()))
+    return launch_pair<PairRes, true>(a_codes, a_scales, nullptr, w_codes, w_scales, nullptr, M, 2 * I, K, nullptr,
+                                      0, static_cast<cudaStream_t>(stream), &extra, kScaleE8M0);
+  return launch_pair<PairCfg<NVFP4_GEMM_PAIR_STAGES>, true>(a_codes, a_scales, nullptr, w_codes, w_scales, nullptr, M,
+                                                           2 * I, K, nullptr, 0, static_cast<cudaStream_t>(stream),
+                                                           &extra, kScaleE8M0);
 }
 
 namespace nvfp4 {

@@ -104,6 +104,40 @@ __device__ __forceinline__ uint32_t quantize8_pair(const float x[8], float amax_
   return kE1M2 ? e1m2x8(v) : e2m1x8(v);
 }
 
+// ---- MXFP4 (Appendix A: E8M0 scale per 32 elements, no global scale) ----
+constexpr uint32_t kInvSqrt32Bits = 0x3E3504F3u;  // fp32(1 / sqrt(32)), round to nearest
+
+// In-register fast Walsh-Hadamard transform of 32 values: butterflies
+// (a + b, a - b) at strides 1, 2, 4, 8, 16, each rounded to fp32, then one
+// fp32 multiplication by 1/sqrt(32) (Sylvester order: the result is x H_32 / sqrt(32)).
+__device__ __forceinline__ void hadamard32(float x[32]) {
+#pragma unroll
+  for (int h = 1; h < 32; h <<= 1) {
+#pragma unroll
+    for (int i = 0; i < 32; ++i) {
+      if ((i & h) == 0) {
+        const float a = x[i], b = x[i + h];
+        x[i] = __fadd_rn(a, b);
+        x[i + h] = __fsub_rn(a, b);
+      }
+    }
+  }
+  const float inv = __uint_as_float(kInvSqrt32Bits);
+#pragma unroll
+  for (int i = 0; i < 32; ++i) x[i] = __fmul_rn(x[i], inv);
+}
+
+// E8M0 code of a 32-element block with this amax: e = floor(log2 amax) - 2,
+// clamped to [-127, 127], read off the binary exponent field E (zero and
+// subnormal amax have E = 0 and clamp), so the code e + 127 is max(E - 2, 0);
+// a finite amax < 2^128 keeps e <= 125.
+__device__ __forceinline__ uint32_t mx_scale_code(float amax) {
+  const uint32_t E = __float_as_uint(amax) >> 23;
+  return E > 2u ? E - 2u : 0u;
+}
+// 1 / 2^e = 2^(127 - code), a normal fp32 for every code the quantizer makes (<= 252).
+__device__ __forceinline__ float mx_inv_scale(uint32_t code) { return __uint_as_float((254u - code) << 23); }
+
 // Byte offset of block scale (row r, k-block kb) in the tensor-core storage
 // order: 128-row tiles, groups of 4 k-blocks, 512-byte atoms k-group fastest,
 // inside an atom (r%32)*16 + ((r%128)/32)*4 + kb%4.

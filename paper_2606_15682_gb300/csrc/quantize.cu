@@ -363,28 +363,6 @@ int dynamic_capacity(int stash_iters) {
 // Sec. 4).  One thread quantizes one block per slot; no tensor-wide pass.
 // ---------------------------------------------------------------------------
 constexpr int kMxUnroll = 2;
-constexpr uint32_t kInvSqrt32Bits = 0x3E3504F3u;  // fp32(1 / sqrt(32)), round to nearest
-
-// In-register fast Walsh-Hadamard transform of 32 values: butterflies
-// (a + b, a - b) at strides 1, 2, 4, 8, 16, each rounded to fp32, then one
-// fp32 multiplication by 1/sqrt(32) (Sylvester order: the result is x H_32 / sqrt(32)).
-__device__ __forceinline__ void hadamard32(float x[32]) {
-#pragma unroll
-  for (int h = 1; h < 32; h <<= 1) {
-#pragma unroll
-    for (int i = 0; i < 32; ++i) {
-      if ((i & h) == 0) {
-        const float a = x[i], b = x[i + h];
-        x[i] = __fadd_rn(a, b);
-        x[i + h] = __fsub_rn(a, b);
-      }
-    }
-  }
-  const float inv = __uint_as_float(kInvSqrt32Bits);
-#pragma unroll
-  for (int i = 0; i < 32; ++i) x[i] = __fmul_rn(x[i], inv);
-}
-
 // Block index b (of rows * cols/32) -> its 32 bf16 elements as fp32, the row and block-in-row.
 template <bool kMMA, bool kRotate>
 __global__ void __launch_bounds__(kThreads) mx_quantize_kernel(const uint16_t* __restrict__ x, FastDiv nb_div,
@@ -421,13 +399,8 @@ __global__ void __launch_bounds__(kThreads) mx_quantize_kernel(const uint16_t* _
       float amax = 0.0f;
 #pragma unroll
       for (int i = 0; i < 32; ++i) amax = fmaxf(amax, fabsf(xf[i]));
-      // e = floor(log2 amax) - 2, clamped to [-127, 127]: from the binary
-      // exponent field E (zero and subnormal amax have E = 0 and clamp), so the
-      // E8M0 code e + 127 is max(E - 2, 0); amax < 2^128 keeps e <= 125.
-      const uint32_t E = __float_as_uint(amax) >> 23;
-      const uint32_t code = E > 2u ? E - 2u : 0u;
-      // x / 2^e = x * 2^(127 - code): 2^(127 - code) is a normal fp32 (code <= 252).
-      const float inv_scale = __uint_as_float((254u - code) << 23);
+      const uint32_t code = mx_scale_code(amax);
+      const float inv_scale = mx_inv_scale(code);
 #pragma unroll
       for (int i = 0; i < 32; ++i) xf[i] = __fmul_rn(xf[i], inv_scale);
       const uint4 packed = make_uint4(e2m1x8(xf), e2m1x8(xf + 8), e2m1x8(xf + 16), e2m1x8(xf + 24));

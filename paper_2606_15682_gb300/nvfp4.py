@@ -72,6 +72,7 @@ _scales_bytes = _sig("nvfp4_scales_bytes", [_i64, _i64, ctypes.c_int], _sz)
 _mx_scales_bytes = _sig("mxfp4_scales_bytes", [_i64, _i64, ctypes.c_int], _sz)
 _mx_quantize = _sig("mxfp4_quantize", [_p, _i64, _i64, _i64, ctypes.c_int, _p, _p, ctypes.c_int, _p])
 _mx_linear = _sig("mxfp4_linear", [_p, _p, _p, _p, _i64, _i64, _i64, _p, _i64, _p])
+_mx_linear_swiglu = _sig("mxfp4_linear_swiglu_quantize", [_p, _p, _p, _p, _i64, _i64, _i64, ctypes.c_int, _p, _p, _p])
 
 
 def _stream(stream):
@@ -155,6 +156,13 @@ def mxfp4_quantize(x, codes, scales, layout=SCALES_MMA, rotate=False, stream=Non
 def mxfp4_linear(a_codes, a_scales, w_codes, w_scales, out, M, N, K, ldo=None, stream=None):
     _check("mxfp4_linear", _mx_linear(_ptr(a_codes), _ptr(a_scales), _ptr(w_codes), _ptr(w_scales), M, N, K,
                                       _ptr(out), N if ldo is None else ldo, _stream(stream)))
+
+
+def mxfp4_linear_swiglu_quantize(a_codes, a_scales, w_codes, w_scales, M, I, K, out_codes, out_scales,
+                                  rotate=False, stream=None):
+    _check("mxfp4_linear_swiglu_quantize",
+           _mx_linear_swiglu(_ptr(a_codes), _ptr(a_scales), _ptr(w_codes), _ptr(w_scales), M, I, K,
+                             int(bool(rotate)), _ptr(out_codes), _ptr(out_scales), _stream(stream)))
 
 
 def nvfp4_linear_swiglu_quantize(a_codes, a_scales, g_a, w_codes, w_scales, g_w, M, I, K, g_out,
@@ -257,7 +265,7 @@ class KVCache:
 
 EXPORTED = ["nvfp4_scales_bytes", "nvfp4_tensor_scale", "nvfp4_quantize", "nvfp4_quantize_dynamic", "nvfp4_scales_relayout", "nvfp4_linear",
             "nvfp4_linear_swiglu_quantize", "nvfp4_interleave_gate_up",
-            "mxfp4_scales_bytes", "mxfp4_quantize", "mxfp4_linear",
+            "mxfp4_scales_bytes", "mxfp4_quantize", "mxfp4_linear", "mxfp4_linear_swiglu_quantize",
             "kv_append_nvfp4", "kv_append_rope_nvfp4", "nvfp4_rope_table", "decode_attention_nvfp4_workspace_size", "decode_attention_nvfp4",
             "decode_attention_nvfp4_quantize",
             "decode_attention_nvfp4_static_scratch",

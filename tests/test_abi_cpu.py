@@ -89,6 +89,11 @@ def test_mxfp4_validation_before_launch():
     assert L.mxfp4_linear(p, p, p, p, 128, 128, 192, p, 128, s) == 2  # K % 256
     assert L.mxfp4_linear(p, p, p, p, 128, 120, 256, p, 128, s) == 2  # N % 16
     assert L.mxfp4_linear(p, odd, p, p, 128, 128, 256, p, 128, s) == 3
+    assert L.mxfp4_linear_swiglu_quantize(p, p, p, p, 256, 192, 512, 0, p, p, s) == 2    # I % 128
+    assert L.mxfp4_linear_swiglu_quantize(p, p, p, p, 256, 256, 384, 0, p, p, s) == 2    # K % 256
+    assert L.mxfp4_linear_swiglu_quantize(p, p, p, p, 256, 256, 512, 3, p, p, s) == 1    # rotate 0/1
+    assert L.mxfp4_linear_swiglu_quantize(p, p, p, p, 256, 256, 512, 0, None, p, s) == 1
+    assert L.mxfp4_linear_swiglu_quantize(p, p, p, p, 256, 256, 512, 0, odd, p, s) == 3
 
 
 def test_kv_and_attention_validation():

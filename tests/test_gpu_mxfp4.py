@@ -170,3 +170,71 @@ def test_mx_linear_padded_output(N):
     out = run_mx_linear(N, ac, asf, wc, wsf, M, Nn, K, ldo=168)
     assert_close(f32(out[:, :Nn]), X.linear_mx(ac, asf, wc, wsf), what="mxfp4 padded ldo")
     assert torch.isnan(out[:, Nn:].float()).all(), "columns beyond N must be left untouched"
+
+
+def mx_random_operand(rows, K, gen, lo, hi):
+    codes = torch.randint(0, 256, (rows, K // 2), generator=gen, dtype=torch.int32).to(torch.uint8).numpy()
+    scales = torch.randint(lo, hi, (rows, K // 32), generator=gen, dtype=torch.int32).to(torch.uint8).numpy()
+    return codes, scales
+
+
+def mx_swiglu_case(N, M, I, K, seed, rotate, rows=None):
+    gen = torch.Generator().manual_seed(seed)
+    a_c, a_s = mx_random_operand(M, K, gen, 121, 129)
+    wg_c, wg_s = mx_random_operand(I, K, gen, 116, 122)
+    wu_c, wu_s = mx_random_operand(I, K, gen, 116, 122)
+    rows = np.arange(M) if rows is None else np.asarray(rows)
+    h, rc, rs = X.linear_swiglu_quantize_mx(a_c, a_s, wg_c, wg_s, wu_c, wu_s, rotate=rotate, rows=rows)
+    w_c = O.interleave_gate_up(wg_c, wu_c)
+    w_s = O.interleave_gate_up(wg_s, wu_s)
+    dev = "cuda"
+    out_c = torch.full((M, I // 2), 0xEE, dtype=torch.uint8, device=dev)
+    out_s = torch.full((N.mxfp4_scales_bytes(M, I, 1),), 0xEE, dtype=torch.uint8, device=dev)
+    N.mxfp4_linear_swiglu_quantize(torch.from_numpy(a_c).to(dev), torch.from_numpy(X.mx_scales_to_mma(a_s)).to(dev),
+                                   torch.from_numpy(w_c).to(dev), torch.from_numpy(X.mx_scales_to_mma(w_s)).to(dev),
+                                   M, I, K, out_c, out_s, rotate=rotate)
+    torch.cuda.synchronize()
+    assert N.nvfp4_get_device_status() == 0
+    return h, rc, rs, rows, u8(out_c), u8(out_s)
+
+
+def check_mx_swiglu(h, rc, rs, rows, out_c, out_s, M, I, rotate):
+    """Scales within one E8M0 step of the oracle's, almost all equal; almost all
+    codes equal; every element within the format's error bound of the fp64 h
+    (rotated by the exact H_32 / sqrt(32) when asked); padding scales zero."""
+    gs = X.mx_scales_from_mma(out_s, M, I)[rows]
+    assert np.abs(gs.astype(int) - rs.astype(int)).max() <= 1
+    assert (gs == rs).mean() > 0.99
+    assert (out_c[rows] == rc).mean() > 0.99
+    target = X.rotate_blocks(h) if rotate else h
+    deq = X.dequantize_mx(out_c[rows], gs)
+    scale = np.repeat(X.e8m0_decode(gs), 32, axis=1)
+    assert np.all(np.abs(deq - target) <= 2.0 * scale + 1e-4 * np.abs(target))
+    pad = np.setdiff1d(np.arange(O.mma_scale_bytes(M, I)), O._mma_offsets(M, I // 16).ravel())
+    assert not out_s[pad].any(), "padding rows of the output scales must be zero"
+
+
+@pytest.mark.parametrize("rotate", [False, True], ids=["plain", "rotated"])
+@pytest.mark.parametrize("M,I,K", [(256, 128, 256), (129, 384, 512), (640, 512, 768)])
+def test_mx_linear_swiglu_quantize(N, M, I, K, rotate):
+    h, rc, rs, rows, out_c, out_s = mx_swiglu_case(N, M, I, K, seed=M + I + K + rotate, rotate=rotate)
+    check_mx_swiglu(h, rc, rs, rows, out_c, out_s, M, I, rotate)
+
+
+@pytest.mark.parametrize("rotate", [False, True], ids=["plain", "rotated"])
+def test_mx_linear_swiglu_quantize_prefill_shape_then_down(N, rotate):
+    """The 1.5B-prefill MLP shape (M=2048, I=8960, K=1536; the W-resident form)
+    on sampled rows, then fed to the MXFP4 down projection as its A operand."""
+    M, I, K, Hd = 2048, 8960, 1536, 1536
+    rows = np.sort(np.r_[np.random.default_rng(3).choice(M - 1, 40, replace=False), M - 1])
+    h, rc, rs, rows, out_c, out_s = mx_swiglu_case(N, M, I, K, seed=123 + rotate, rotate=rotate, rows=rows)
+    check_mx_swiglu(h, rc, rs, rows, out_c, out_s, M, I, rotate)
+    gen = torch.Generator().manual_seed(8)
+    wd_c, wd_s = mx_random_operand(Hd, I, gen, 116, 122)
+    out = torch.empty(M, Hd, dtype=torch.bfloat16, device="cuda")
+    N.mxfp4_linear(torch.from_numpy(out_c).cuda(), torch.from_numpy(out_s).cuda(), torch.from_numpy(wd_c).cuda(),
+                   torch.from_numpy(X.mx_scales_to_mma(wd_s)).cuda(), out, M, Hd, I)
+    torch.cuda.synchronize()
+    assert N.nvfp4_get_device_status() == 0
+    ref = X.linear_mx_rows(out_c, X.mx_scales_from_mma(out_s, M, I), wd_c, wd_s, rows)
+    assert_close(f32(out[torch.as_tensor(rows, device="cuda")]), ref, what="mx down(swiglu)")

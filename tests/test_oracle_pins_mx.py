@@ -217,3 +217,27 @@ def test_mx_scales_mma_layout_duplicates_each_block_scale():
     bad[O._mma_offsets(130, 16)[0, 1]] ^= 1
     with pytest.raises(ValueError):
         X.mx_scales_from_mma(bad, 130, 256)
+
+
+def test_swiglu_quantize_mx_composes_library_silu_and_the_quantizer():
+    # SiLU against scipy's logistic function; the fused form is SiLU(G) * U of
+    # the fp64 products, quantized from fp32 (brute-force products here).
+    import scipy.special
+    x = np.linspace(-30, 30, 1001)
+    assert np.allclose(O.silu(x), x * scipy.special.expit(x), rtol=1e-14, atol=1e-300)
+    rng = np.random.default_rng(10)
+    a = _f32(rng.standard_normal((6, 64)))
+    wg = _f32(rng.standard_normal((64, 64)) * 0.1)
+    wu = _f32(rng.standard_normal((64, 64)) * 0.1)
+    (ac, asf), (gc, gsf), (uc, usf) = X.quantize_mx(a), X.quantize_mx(wg), X.quantize_mx(wu)
+    ah, gh, uh = X.dequantize_mx(ac, asf), X.dequantize_mx(gc, gsf), X.dequantize_mx(uc, usf)
+    G = np.array([[sum(ah[i, k] * gh[j, k] for k in range(64)) for j in range(64)] for i in range(6)])
+    U = np.array([[sum(ah[i, k] * uh[j, k] for k in range(64)) for j in range(64)] for i in range(6)])
+    h_ref = G * scipy.special.expit(G) * U
+    for rotate in (False, True):
+        h, c, s = X.linear_swiglu_quantize_mx(ac, asf, gc, gsf, uc, usf, rotate=rotate)
+        assert np.allclose(h, h_ref, rtol=1e-12, atol=1e-15)
+        rc, rs = X.quantize_mx(h_ref.astype(np.float32), rotate=rotate)
+        assert np.array_equal(c, rc) and np.array_equal(s, rs)
+        hr, cr, sr = X.linear_swiglu_quantize_mx(ac, asf, gc, gsf, uc, usf, rotate=rotate, rows=[5, 1])
+        assert np.array_equal(cr, c[[5, 1]]) and np.array_equal(sr, s[[5, 1]])
