@@ -238,3 +238,48 @@ def test_mx_linear_swiglu_quantize_prefill_shape_then_down(N, rotate):
     assert N.nvfp4_get_device_status() == 0
     ref = X.linear_mx_rows(out_c, X.mx_scales_from_mma(out_s, M, I), wd_c, wd_s, rows)
     assert_close(f32(out[torch.as_tensor(rows, device="cuda")]), ref, what="mx down(swiglu)")
+
+
+@pytest.mark.parametrize("rotate", [False, True], ids=["plain", "rotated"])
+def test_mx_mlp_chain_tracks_the_exact_mlp(N, rotate):
+    """x -> mxfp4_quantize -> fused gate_up (SwiGLU + MXFP4 h) -> mxfp4_linear
+    against W_down, with every operand rotated along its K when asked: the GPU
+    chain is as close to the exact fp64 MLP as the oracle's chain is (the
+    rotation preserves each product only if both operands are rotated)."""
+    M, H, I = 256, 1536, 1024
+    dev = "cuda"
+    x = synth.activation(M, H, 7600, outlier_frac=0.01)
+    wg, wu = synth.weight(I, H, 7601), synth.weight(I, H, 7602)
+    wd = synth.weight(H, I, 7603)
+    exact_h = O.silu(f32(x).astype(np.float64) @ f32(wg).astype(np.float64).T) * (
+        f32(x).astype(np.float64) @ f32(wu).astype(np.float64).T)
+    exact = exact_h @ f32(wd).astype(np.float64).T
+
+    def q(t):
+        c = torch.empty(t.shape[0], t.shape[1] // 2, dtype=torch.uint8, device=dev)
+        s = torch.empty(N.mxfp4_scales_bytes(t.shape[0], t.shape[1], 1), dtype=torch.uint8, device=dev)
+        N.mxfp4_quantize(t.to(dev).contiguous(), c, s, 1, rotate=rotate)
+        return c, s
+    wi = torch.empty(2 * I, H, dtype=torch.bfloat16, device=dev)
+    N.nvfp4_interleave_gate_up(wg.to(dev), wu.to(dev), wi)
+    (xc, xs), (wc, ws), (dc, ds) = q(x), q(wi), q(wd)
+    hc = torch.empty(M, I // 2, dtype=torch.uint8, device=dev)
+    hs = torch.empty(N.mxfp4_scales_bytes(M, I, 1), dtype=torch.uint8, device=dev)
+    N.mxfp4_linear_swiglu_quantize(xc, xs, wc, ws, M, I, H, hc, hs, rotate=rotate)
+    y = torch.empty(M, H, dtype=torch.bfloat16, device=dev)
+    N.mxfp4_linear(hc, hs, dc, ds, y, M, H, I)
+    torch.cuda.synchronize()
+    assert N.nvfp4_get_device_status() == 0
+
+    oc, os_ = X.quantize_mx(f32(x), rotate=rotate)
+    gc, gs = X.quantize_mx(f32(wg), rotate=rotate)
+    uc, us = X.quantize_mx(f32(wu), rotate=rotate)
+    odc, ods = X.quantize_mx(f32(wd), rotate=rotate)
+    _, ohc, ohs = X.linear_swiglu_quantize_mx(oc, os_, gc, gs, uc, us, rotate=rotate)
+    y_orc = X.linear_mx(ohc, ohs, odc, ods)
+    scale = np.abs(exact).max()
+    e_orc = np.abs(y_orc - exact).max() / scale
+    e_gpu = np.abs(f32(y).astype(np.float64) - exact).max() / scale
+    print(f"MXFP4 MLP ({'rotated' if rotate else 'plain'}): GPU {e_gpu:.3e}, oracle {e_orc:.3e}")
+    assert e_orc < 0.5
+    assert e_gpu <= 1.25 * e_orc + 5e-3
