@@ -112,8 +112,10 @@ nvfp4_status nvfp4_quantize(const void* x_bf16, int64_t rows, int64_t cols, int6
  * with it (exactly as nvfp4_quantize does); codes, scales and g are
  * bit-identical to the two calls in sequence.
  *   state_dev : NVFP4_DYNAMIC_STATE_BYTES of device memory, 16-B aligned,
- *               zero-filled once before its first use and left alone by the
- *               caller afterwards.  Calls that may run concurrently (other
+ *               zero-filled once before its first use (the fill must be
+ *               ordered before the call: same stream, or synchronized with
+ *               it; a call that reads a stale state can report TIMEOUT) and
+ *               left alone by the caller afterwards.  Calls that may run concurrently (other
  *               streams) need separate states; calls in one stream may share.
  *   g_dev     : device float, written (never read first).
  *   x, codes, scales, layout : as nvfp4_quantize.
