@@ -283,3 +283,36 @@ def test_mx_mlp_chain_tracks_the_exact_mlp(N, rotate):
     print(f"MXFP4 MLP ({'rotated' if rotate else 'plain'}): GPU {e_gpu:.3e}, oracle {e_orc:.3e}")
     assert e_orc < 0.5
     assert e_gpu <= 1.25 * e_orc + 5e-3
+
+
+WL = [w for w in synth.WORKLOADS if "linears" in synth.WORKLOADS[w]]
+
+
+@pytest.mark.parametrize("workload", WL)
+def test_mx_workload_linears(N, workload):
+    """Every linear of every workload at full size in the MXFP4 W4A4 launch
+    configuration the bench times (activation and weight rotated and
+    quantized on the GPU, then mxfp4_linear), on seeded samples of output
+    rows and columns; the sampled operands' codes and scales are bit-exact."""
+    dev = "cuda"
+    for name, (Nn, K) in synth.WORKLOADS[workload]["linears"].items():
+        a, W = synth.linear_inputs(workload, name, device=dev)
+        M = a.shape[0]
+        ac, asf = gpu_mx_quantize(N, a, 1, True)
+        wc, wsf = gpu_mx_quantize(N, W, 1, True)
+        out = torch.empty(M, Nn, dtype=torch.bfloat16, device=dev)
+        N.mxfp4_linear(ac, asf, wc, wsf, out, M, Nn, K)
+        torch.cuda.synchronize()
+        assert N.nvfp4_get_device_status() == 0
+        rng = np.random.default_rng(2)
+        rows = np.arange(M) if M * K <= 2048 * 8960 else np.sort(np.r_[rng.choice(M - 1, 64, replace=False), M - 1])
+        cols = np.arange(Nn) if Nn * K <= 17920 * 1536 else np.sort(np.r_[rng.choice(Nn - 1, 192, replace=False), Nn - 1])
+        assert rows.max() < M and cols.max() < Nn
+        tr, tc = torch.as_tensor(rows, device=dev), torch.as_tensor(cols, device=dev)
+        ra_c, ra_s = X.quantize_mx(f32(a[tr]), rotate=True)
+        rw_c, rw_s = X.quantize_mx(f32(W[tc]), rotate=True)
+        assert np.array_equal(u8(ac[tr]), ra_c) and np.array_equal(X.mx_scales_from_mma(u8(asf), M, K)[rows], ra_s)
+        assert np.array_equal(u8(wc[tc]), rw_c) and np.array_equal(X.mx_scales_from_mma(u8(wsf), Nn, K)[cols], rw_s)
+        ref = X.linear_mx(ra_c, ra_s, rw_c, rw_s)
+        assert_close(f32(out[tr][:, tc]), ref, what=f"mxfp4 {workload}/{name}")
+        del a, W, ac, asf, wc, wsf, out
