@@ -56,6 +56,7 @@ void count_launches(uint64_t n) { g_launches.fetch_add(n, std::memory_order_rela
 using namespace nvfp4;
 
 NVFP4_API nvfp4_status nvfp4_get_device_status(int32_t* status_host, void* stream) {
+  NVFP4_TRACE("nvfp4_get_device_status");
   if (!status_host) return NVFP4_ERR_INVALID_ARG;
   int* p = status_word_dev();
   if (!p) return NVFP4_ERR_CUDA;

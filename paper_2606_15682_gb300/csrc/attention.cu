@@ -652,6 +652,7 @@ nvfp4_status attention_params(const nvfp4_kv_cache* cache, const void* q_bf16, i
 NVFP4_API nvfp4_status decode_attention_nvfp4(const nvfp4_kv_cache* cache, const void* q_bf16, int32_t num_q_heads,
                                               float softmax_scale, void* out_bf16, void* workspace,
                                               size_t workspace_bytes, void* stream) {
+  NVFP4_TRACE("decode_attention_nvfp4");
   if (!out_bf16 || !workspace) return NVFP4_ERR_INVALID_ARG;
   nvfp4_status st = attention_validate(cache, q_bf16, num_q_heads, softmax_scale);
   if (st != NVFP4_OK) return st;
@@ -676,6 +677,7 @@ NVFP4_API nvfp4_status decode_attention_nvfp4_quantize(const nvfp4_kv_cache* cac
                                                        int32_t num_q_heads, float softmax_scale, const float* g_out,
                                                        uint8_t* out_codes, uint8_t* out_scales, void* workspace,
                                                        size_t workspace_bytes, void* stream) {
+  NVFP4_TRACE("decode_attention_nvfp4_quantize");
   if (!g_out || !out_codes || !out_scales || !workspace) return NVFP4_ERR_INVALID_ARG;
   nvfp4_status st = attention_validate(cache, q_bf16, num_q_heads, softmax_scale);
   if (st != NVFP4_OK) return st;
@@ -737,6 +739,7 @@ float* attn_static_scratch_dev() {
 NVFP4_API nvfp4_status decode_attention_nvfp4_static_scratch(const nvfp4_kv_cache* cache, const void* q_bf16,
                                                              int32_t num_q_heads, float softmax_scale,
                                                              void* out_bf16, void* stream) {
+  NVFP4_TRACE("decode_attention_nvfp4_static_scratch");
   if (!out_bf16) return NVFP4_ERR_INVALID_ARG;
   nvfp4_status st = attention_validate(cache, q_bf16, num_q_heads, softmax_scale);
   if (st != NVFP4_OK) return st;

@@ -6,6 +6,7 @@
 #pragma once
 
 #include <cuda_runtime.h>
+#include <nvtx3/nvToolsExt.h>
 #include <stdint.h>
 
 #include <utility>
@@ -28,6 +29,18 @@ int* status_word_dev();
 void count_launches(uint64_t n);
 int sm_count();
 inline bool aligned(const void* p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+// An NVTX range named after the C-ABI call, open for the call's host-side
+// duration (argument checks and launches).  A profiler that records NVTX
+// (ncu --nvtx, nsys) attributes each launch to the call that made it;
+// without one attached the push and pop are calls to no-op stubs.
+struct TraceRange {
+  explicit TraceRange(const char* name) { nvtxRangePushA(name); }
+  ~TraceRange() { nvtxRangePop(); }
+  TraceRange(const TraceRange&) = delete;
+  TraceRange& operator=(const TraceRange&) = delete;
+};
+#define NVFP4_TRACE(name) ::nvfp4::TraceRange nvfp4_trace_range_(name)
 inline nvfp4_status launch_status() {
   cudaError_t e = cudaGetLastError();
   return e == cudaSuccess ? NVFP4_OK : NVFP4_ERR_CUDA;

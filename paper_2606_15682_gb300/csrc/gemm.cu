@@ -1210,6 +1210,7 @@ nvfp4_status linear_dispatch(const uint8_t* a_codes, const uint8_t* a_scales, co
 NVFP4_API nvfp4_status nvfp4_linear(const uint8_t* a_codes, const uint8_t* a_scales, const float* g_a,
                                     const uint8_t* w_codes, const uint8_t* w_scales, const float* g_w, int64_t M,
                                     int64_t N, int64_t K, void* out_bf16, int64_t ldo, void* stream) {
+  NVFP4_TRACE("nvfp4_linear");
   if (!a_codes || !a_scales || !g_a || !w_codes || !w_scales || !g_w || !out_bf16) return NVFP4_ERR_INVALID_ARG;
   if (M <= 0 || N <= 0 || K <= 0 || K % BK || N % 16 || ldo < N || ldo % 8) return NVFP4_ERR_SHAPE;
   if (M >= (1ll << 31) || N >= (1ll << 31) || K >= (1ll << 31)) return NVFP4_ERR_SHAPE;
@@ -1223,6 +1224,7 @@ NVFP4_API nvfp4_status nvfp4_linear(const uint8_t* a_codes, const uint8_t* a_sca
 NVFP4_API nvfp4_status mxfp4_linear(const uint8_t* a_codes, const uint8_t* a_scales, const uint8_t* w_codes,
                                     const uint8_t* w_scales, int64_t M, int64_t N, int64_t K, void* out_bf16,
                                     int64_t ldo, void* stream) {
+  NVFP4_TRACE("mxfp4_linear");
   if (!a_codes || !a_scales || !w_codes || !w_scales || !out_bf16) return NVFP4_ERR_INVALID_ARG;
   if (M <= 0 || N <= 0 || K <= 0 || K % BK || N % 16 || ldo < N || ldo % 8) return NVFP4_ERR_SHAPE;
   if (M >= (1ll << 31) || N >= (1ll << 31) || K >= (1ll << 31)) return NVFP4_ERR_SHAPE;
@@ -1237,6 +1239,7 @@ NVFP4_API nvfp4_status nvfp4_linear_swiglu_quantize(const uint8_t* a_codes, cons
                                                     const uint8_t* w_codes, const uint8_t* w_scales, const float* g_w,
                                                     int64_t M, int64_t I, int64_t K, const float* g_out,
                                                     uint8_t* out_codes, uint8_t* out_scales, void* stream) {
+  NVFP4_TRACE("nvfp4_linear_swiglu_quantize");
   if (!a_codes || !a_scales || !g_a || !w_codes || !w_scales || !g_w || !g_out || !out_codes || !out_scales)
     return NVFP4_ERR_INVALID_ARG;
   if (M <= 0 || I <= 0 || K <= 0 || K % BK || I % 128) return NVFP4_ERR_SHAPE;
@@ -1260,6 +1263,7 @@ NVFP4_API nvfp4_status mxfp4_linear_swiglu_quantize(const uint8_t* a_codes, cons
                                                     const uint8_t* w_codes, const uint8_t* w_scales, int64_t M,
                                                     int64_t I, int64_t K, int rotate, uint8_t* out_codes,
                                                     uint8_t* out_scales, void* stream) {
+  NVFP4_TRACE("mxfp4_linear_swiglu_quantize");
   if (!a_codes || !a_scales || !w_codes || !w_scales || !out_codes || !out_scales) return NVFP4_ERR_INVALID_ARG;
   if (rotate != 0 && rotate != 1) return NVFP4_ERR_INVALID_ARG;
   if (M <= 0 || I <= 0 || K <= 0 || K % BK || I % 128) return NVFP4_ERR_SHAPE;
@@ -1300,6 +1304,7 @@ __global__ void interleave_gate_up_kernel(const uint4* __restrict__ gate, const 
 
 NVFP4_API nvfp4_status nvfp4_interleave_gate_up(const void* w_gate, const void* w_up, int64_t I, int64_t row_bytes,
                                                 void* w_out, void* stream) {
+  NVFP4_TRACE("nvfp4_interleave_gate_up");
   if (!w_gate || !w_up || !w_out) return NVFP4_ERR_INVALID_ARG;
   if (I <= 0 || I % 16 || row_bytes <= 0 || row_bytes % 16) return NVFP4_ERR_SHAPE;
   if (!aligned(w_gate, 16) || !aligned(w_up, 16) || !aligned(w_out, 16)) return NVFP4_ERR_ALIGN;

@@ -151,6 +151,7 @@ using namespace nvfp4;
 NVFP4_API nvfp4_status kv_append_nvfp4(const nvfp4_kv_cache* cache, const void* k_bf16, const void* v_bf16,
                                        const int32_t* seq_idx, const int32_t* pos, int64_t n_new,
                                        const float* k_shift, void* stream) {
+  NVFP4_TRACE("kv_append_nvfp4");
   return append(cache, k_bf16, v_bf16, seq_idx, pos, n_new, k_shift, nullptr, stream);
 }
 
@@ -158,12 +159,14 @@ NVFP4_API nvfp4_status kv_append_rope_nvfp4(const nvfp4_kv_cache* cache, const v
                                             const int32_t* seq_idx, const int32_t* pos, int64_t n_new,
                                             const float* rope_table, int64_t rope_positions, const float* k_shift,
                                             void* stream) {
+  NVFP4_TRACE("kv_append_rope_nvfp4");
   if (!cache || !rope_table) return NVFP4_ERR_INVALID_ARG;
   if (rope_positions < cache->capacity) return NVFP4_ERR_SHAPE;
   return append(cache, k_pre_bf16, v_bf16, seq_idx, pos, n_new, k_shift, rope_table, stream);
 }
 
 NVFP4_API nvfp4_status nvfp4_rope_table(float* table, int64_t n_pos, int32_t head_dim, float theta, void* stream) {
+  NVFP4_TRACE("nvfp4_rope_table");
   if (n_pos < 0 || head_dim <= 0 || head_dim % 2 || n_pos * (head_dim / 2) >= (1ll << 40)) return NVFP4_ERR_SHAPE;
   if (!(theta > 1.0f && theta <= FLT_MAX)) return NVFP4_ERR_INVALID_ARG;
   if (n_pos == 0) return NVFP4_OK;

@@ -475,6 +475,7 @@ NVFP4_API size_t nvfp4_scales_bytes(int64_t rows, int64_t cols, nvfp4_scale_layo
 
 NVFP4_API nvfp4_status nvfp4_tensor_scale(const void* x_bf16, int64_t rows, int64_t cols, int64_t ld,
                                           float* g_dev, void* stream) {
+  NVFP4_TRACE("nvfp4_tensor_scale");
   if (!g_dev) return NVFP4_ERR_INVALID_ARG;
   nvfp4_status st = check_bf16_matrix(x_bf16, rows, cols, ld, 8);
   if (st != NVFP4_OK) return st;
@@ -497,6 +498,7 @@ NVFP4_API nvfp4_status nvfp4_tensor_scale(const void* x_bf16, int64_t rows, int6
 NVFP4_API nvfp4_status nvfp4_quantize(const void* x_bf16, int64_t rows, int64_t cols, int64_t ld,
                                       const float* g_dev, uint8_t* codes, uint8_t* scales,
                                       nvfp4_scale_layout layout, void* stream) {
+  NVFP4_TRACE("nvfp4_quantize");
   if (layout != NVFP4_SCALES_ROWMAJOR && layout != NVFP4_SCALES_MMA) return NVFP4_ERR_INVALID_ARG;
   nvfp4_status st = check_bf16_matrix(x_bf16, rows, cols, ld, layout == NVFP4_SCALES_MMA ? 64 : 16);
   if (st != NVFP4_OK) return st;
@@ -520,6 +522,7 @@ NVFP4_API nvfp4_status nvfp4_quantize(const void* x_bf16, int64_t rows, int64_t 
 NVFP4_API nvfp4_status nvfp4_quantize_dynamic(const void* x_bf16, int64_t rows, int64_t cols, int64_t ld,
                                               void* state_dev, float* g_dev, uint8_t* codes, uint8_t* scales,
                                               nvfp4_scale_layout layout, void* stream) {
+  NVFP4_TRACE("nvfp4_quantize_dynamic");
   if (layout != NVFP4_SCALES_ROWMAJOR && layout != NVFP4_SCALES_MMA) return NVFP4_ERR_INVALID_ARG;
   nvfp4_status st = check_bf16_matrix(x_bf16, rows, cols, ld, layout == NVFP4_SCALES_MMA ? 64 : 16);
   if (st != NVFP4_OK) return st;
@@ -581,6 +584,7 @@ NVFP4_API nvfp4_status nvfp4_quantize_dynamic(const void* x_bf16, int64_t rows, 
 
 NVFP4_API nvfp4_status nvfp4_scales_relayout(const uint8_t* src, uint8_t* dst, int64_t rows, int64_t cols,
                                              nvfp4_scale_layout from, nvfp4_scale_layout to, void* stream) {
+  NVFP4_TRACE("nvfp4_scales_relayout");
   if (!src || !dst) return NVFP4_ERR_INVALID_ARG;
   if ((from != NVFP4_SCALES_ROWMAJOR && from != NVFP4_SCALES_MMA) ||
       (to != NVFP4_SCALES_ROWMAJOR && to != NVFP4_SCALES_MMA))
@@ -610,6 +614,7 @@ NVFP4_API size_t mxfp4_scales_bytes(int64_t rows, int64_t cols, nvfp4_scale_layo
 
 NVFP4_API nvfp4_status mxfp4_quantize(const void* x_bf16, int64_t rows, int64_t cols, int64_t ld, int rotate,
                                       uint8_t* codes, uint8_t* scales, nvfp4_scale_layout layout, void* stream) {
+  NVFP4_TRACE("mxfp4_quantize");
   if (layout != NVFP4_SCALES_ROWMAJOR && layout != NVFP4_SCALES_MMA) return NVFP4_ERR_INVALID_ARG;
   if (rotate != 0 && rotate != 1) return NVFP4_ERR_INVALID_ARG;
   nvfp4_status st = check_bf16_matrix(x_bf16, rows, cols, ld, layout == NVFP4_SCALES_MMA ? 64 : 32);
