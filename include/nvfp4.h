@@ -429,6 +429,20 @@ nvfp4_status decode_attention_nvfp4_static_scratch(const nvfp4_kv_cache* cache, 
  * *status_host (an nvfp4_status value) and clear it. */
 nvfp4_status nvfp4_get_device_status(int32_t* status_host, void* stream);
 
+/*
+ * Test-only fault injection for the failure-detection tests: arms one fault
+ * for the next call of the kind it names, then disarms itself.
+ *   NVFP4_FAULT_ATTN_SKIP_STAGE: in the next decode-attention launch, CTA 0's
+ *     producer leaves its first ring stage neither armed nor loaded, so the
+ *     consumers' bounded wait on it runs out after ~2 s: the call reports
+ *     NVFP4_ERR_TIMEOUT through nvfp4_get_device_status, its output is
+ *     undefined, and the device stays usable.
+ *   NVFP4_FAULT_NONE disarms.  Other values -> INVALID_ARG.
+ */
+#define NVFP4_FAULT_NONE 0
+#define NVFP4_FAULT_ATTN_SKIP_STAGE 1
+nvfp4_status nvfp4_debug_inject_fault(int what);
+
 /* Static, human-readable name of a status. */
 const char* nvfp4_status_string(nvfp4_status s);
 

@@ -51,6 +51,13 @@ int sm_count() {
 
 void count_launches(uint64_t n) { g_launches.fetch_add(n, std::memory_order_relaxed); }
 
+std::atomic<int> g_fault{NVFP4_FAULT_NONE};
+
+bool take_fault(int what) {
+  int armed = what;
+  return what != NVFP4_FAULT_NONE && g_fault.compare_exchange_strong(armed, NVFP4_FAULT_NONE);
+}
+
 }  // namespace nvfp4
 
 using namespace nvfp4;
@@ -84,3 +91,10 @@ NVFP4_API const char* nvfp4_status_string(nvfp4_status s) {
 }
 
 NVFP4_API uint64_t nvfp4_launch_count(void) { return g_launches.load(std::memory_order_relaxed); }
+
+NVFP4_API nvfp4_status nvfp4_debug_inject_fault(int what) {
+  NVFP4_TRACE("nvfp4_debug_inject_fault");
+  if (what != NVFP4_FAULT_NONE && what != NVFP4_FAULT_ATTN_SKIP_STAGE) return NVFP4_ERR_INVALID_ARG;
+  g_fault.store(what);
+  return NVFP4_OK;
+}

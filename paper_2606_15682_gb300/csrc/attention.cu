@@ -173,6 +173,7 @@ struct Params {
   int* status;
   int hkv, capacity, hq, group, n_splits, n_items;
   float logit_mult;  // softmax_scale * g_K * log2(e)
+  int fault_skip_stage;  // test-only: CTA 0's producer leaves its first stage unissued
 };
 
 // kE1M2: the cache holds E1M2 elements (decoded to n, the scale carries 1/2).
@@ -211,6 +212,7 @@ __global__ void __launch_bounds__(kThreads, NVFP4_ATTN_MIN_CTAS) attn_partial_ke
       uint32_t issued_parity[kStages];
       bool issued[kStages];
       for (int s = 0; s < kStages; ++s) issued[s] = false;
+      bool skip_stage = p.fault_skip_stage && blockIdx.x == 0;
       for (int item = blockIdx.x; item < p.n_items && !abort_flag; item += gridDim.x) {
         const Item it = decode_item(item, p.n_splits, p.hkv, p.seq_lens, p.capacity);
         const size_t row0 = (static_cast<size_t>(it.b) * p.hkv + it.kvh) * p.capacity;
@@ -221,6 +223,13 @@ __global__ void __launch_bounds__(kThreads, NVFP4_ATTN_MIN_CTAS) attn_partial_ke
             set_status(p.status, NVFP4_ERR_TIMEOUT);
             abort_flag = 1;
             break;
+          }
+          if (skip_stage) {
+            // Injected fault: the stage is neither armed nor loaded, so the
+            // consumers' bounded wait on it runs out (NVFP4_ERR_TIMEOUT).
+            skip_stage = false;
+            if (++stage == kStages) { stage = 0; phase ^= 1u; }
+            continue;
           }
           uint8_t* st = ring + stage * kStageBytes;
           mbar_arrive_expect_tx(&full[stage], 2u * (n * 64 + n_even * 8));
@@ -638,6 +647,7 @@ nvfp4_status attention_params(const nvfp4_kv_cache* cache, const void* q_bf16, i
   prm->n_splits = splits_for(cache->capacity);
   prm->n_items = static_cast<int>(n_items);
   prm->logit_mult = softmax_scale * cache->k_gscale * kLog2e;
+  prm->fault_skip_stage = take_fault(NVFP4_FAULT_ATTN_SKIP_STAGE) ? 1 : 0;
   // Every record the combine kernel reads is written by the partial kernel of
   // the same call, so nothing left from an earlier call needs clearing.
   prm->o_ws = partials;

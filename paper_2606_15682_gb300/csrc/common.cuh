@@ -27,6 +27,8 @@ namespace nvfp4 {
 // once per device with cudaGetSymbolAddress; never allocates.
 int* status_word_dev();
 void count_launches(uint64_t n);
+// True once after nvfp4_debug_inject_fault(what) armed `what` (then disarmed).
+bool take_fault(int what);
 int sm_count();
 inline bool aligned(const void* p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
 

@@ -70,6 +70,13 @@ _status_string = _sig("nvfp4_status_string", [ctypes.c_int], ctypes.c_char_p)
 _launch_count = _sig("nvfp4_launch_count", [], ctypes.c_uint64)
 _scales_bytes = _sig("nvfp4_scales_bytes", [_i64, _i64, ctypes.c_int], _sz)
 _mx_scales_bytes = _sig("mxfp4_scales_bytes", [_i64, _i64, ctypes.c_int], _sz)
+_inject_fault = _sig("nvfp4_debug_inject_fault", [ctypes.c_int])
+FAULT_NONE, FAULT_ATTN_SKIP_STAGE = 0, 1
+
+
+def nvfp4_debug_inject_fault(what):
+    """Test-only: arm one injected fault for the next call of its kind (see include/nvfp4.h)."""
+    _check("nvfp4_debug_inject_fault", _inject_fault(what))
 _mx_quantize = _sig("mxfp4_quantize", [_p, _i64, _i64, _i64, ctypes.c_int, _p, _p, ctypes.c_int, _p])
 _mx_linear = _sig("mxfp4_linear", [_p, _p, _p, _p, _i64, _i64, _i64, _p, _i64, _p])
 _mx_linear_swiglu = _sig("mxfp4_linear_swiglu_quantize", [_p, _p, _p, _p, _i64, _i64, _i64, ctypes.c_int, _p, _p, _p])
@@ -269,4 +276,4 @@ EXPORTED = ["nvfp4_scales_bytes", "nvfp4_tensor_scale", "nvfp4_quantize", "nvfp4
             "kv_append_nvfp4", "kv_append_rope_nvfp4", "nvfp4_rope_table", "decode_attention_nvfp4_workspace_size", "decode_attention_nvfp4",
             "decode_attention_nvfp4_quantize",
             "decode_attention_nvfp4_static_scratch",
-            "nvfp4_get_device_status", "nvfp4_status_string", "nvfp4_launch_count"]
+            "nvfp4_get_device_status", "nvfp4_status_string", "nvfp4_launch_count", "nvfp4_debug_inject_fault"]

@@ -96,6 +96,13 @@ def test_mxfp4_validation_before_launch():
     assert L.mxfp4_linear_swiglu_quantize(p, p, p, p, 256, 256, 512, 0, odd, p, s) == 3
 
 
+def test_fault_injection_knob_validation():
+    N = lib()
+    assert N._lib.nvfp4_debug_inject_fault(5) == 1
+    assert N._lib.nvfp4_debug_inject_fault(N.FAULT_ATTN_SKIP_STAGE) == 0
+    assert N._lib.nvfp4_debug_inject_fault(N.FAULT_NONE) == 0
+
+
 def test_kv_and_attention_validation():
     N = lib()
     import torch  # noqa: F401  (struct only; no device memory)

@@ -438,3 +438,43 @@ def test_qfit_calibration_matches_oracle_grid(N):
     assert np.unravel_index(err.argmin(), err.shape) == np.unravel_index(r_err.argmin(), r_err.shape)
     assert np.allclose(s_k.cpu().numpy(), r_sk, rtol=1e-6) and np.allclose(m.cpu().numpy(), r_m, rtol=1e-5, atol=1e-6)
     assert r_err.min() < r_err[0, 0]            # the calibration improves on no transform
+
+
+def test_injected_missing_stage_times_out_and_device_stays_usable(N):
+    """Failure detection without a GPU fault: the test-only fault knob makes
+    CTA 0's producer leave its first ring stage unissued (a barrier that
+    nothing completes).  The consumers' bounded wait runs out after ~2 s, the
+    call reports NVFP4_ERR_TIMEOUT, and the next call on the same cache is
+    exact again."""
+    import time
+    B, hq, hkv, lens = 2, 10, 2, [300, 257]
+    cap = 304
+    rec = synth.KVRecipe(hkv, seed=41)
+    T = sum(lens)
+    k, v = rec.kv(T, seed=42)
+    seq = np.concatenate([np.full(l, b) for b, l in enumerate(lens)]).astype(np.int64)
+    pos = np.concatenate([np.arange(l) for l in lens]).astype(np.int64)
+    gk, gv = O.tensor_scale(f32(k)), O.tensor_scale(f32(v))
+    cache = N.KVCache(B, hkv, cap, gk, gv)
+    fill(N, cache, k, v, seq, pos)
+    cache.seq_lens.copy_(torch.tensor(lens, dtype=torch.int32))
+    q = rec.queries(B, hq, seed=43)
+    scale = 1.0 / math.sqrt(128)
+    torch.cuda.synchronize()
+    assert N.nvfp4_get_device_status() == 0
+    N.nvfp4_debug_inject_fault(N.FAULT_ATTN_SKIP_STAGE)
+    try:
+        t0 = time.time()
+        run_attention(N, cache, q, scale)
+        waited = time.time() - t0
+    finally:
+        N.nvfp4_debug_inject_fault(N.FAULT_NONE)
+    assert N.nvfp4_get_device_status() == 6
+    assert waited > 1.0, "the injected stage must be waited for (bounded) before the kernel gives up"
+    out = run_attention(N, cache, q, scale)
+    assert N.nvfp4_get_device_status() == 0
+    rkc, rks, rvc, rvs = oracle_cache(B, hkv, cap)
+    O.kv_append(rkc, rks, rvc, rvs, f32(k), f32(v), seq, pos, np.float32(gk), np.float32(gv))
+    ref = O.decode_attention(f32(q), rkc, rks, rvc, rvs, lens, gk, gv, scale)
+    for b in range(B):
+        assert_close(f32(out)[b], ref[b], what=f"after the injected timeout, seq {b}")
