@@ -55,7 +55,9 @@ typedef enum {
   NVFP4_ERR_UNSUPPORTED = 4, /* no sm_103a device, or device lacks a feature  */
   NVFP4_ERR_CUDA = 5,        /* a CUDA runtime/driver call or launch failed   */
   NVFP4_ERR_TIMEOUT = 6,     /* a bounded on-device wait gave up              */
-  NVFP4_ERR_CAPACITY = 7     /* KV append position beyond the cache capacity  */
+  NVFP4_ERR_CAPACITY = 7,    /* KV append position beyond the cache capacity  */
+  NVFP4_ERR_BOUNDS = 8       /* bounds-checked build only: a computed store   */
+                             /* index left its buffer; the store was skipped  */
 } nvfp4_status;
 
 typedef enum {

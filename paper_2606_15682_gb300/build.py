@@ -3,6 +3,12 @@
 Each CUDA translation unit is compiled in parallel, then linked into one
 shared library under ``paper_2606_15682_gb300/_build``.  Re-running only
 recompiles translation units whose sources or headers changed.
+
+``build(debug=True)`` (or ``NVFP4_DEBUG=1`` in the environment) builds the
+bounds-checked variant into ``_build_debug``: every computed store index of the
+non-TMA kernels is checked against the extent the kernel derives from its
+shape arguments, and a violation sets NVFP4_ERR_BOUNDS instead of writing.
+The binding loads that variant when ``NVFP4_DEBUG=1``.
 """
 from __future__ import annotations
 
@@ -18,6 +24,7 @@ ROOT = os.path.dirname(PKG)
 CSRC = os.path.join(PKG, "csrc")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(BUILD, "libnvfp4.so")
+BUILD_DEBUG = os.path.join(PKG, "_build_debug")
 SOURCES = ["api.cu", "quantize.cu", "kv_append.cu", "attention.cu", "gemm.cu"]
 HEADERS = ["common.cuh", "nvfp4_quant.cuh", os.path.join("..", "..", "include", "nvfp4.h")]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
@@ -31,23 +38,23 @@ def _nvcc():
     return cand
 
 
-def _digest(src):
+def _digest(src, flags):
     h = hashlib.sha256()
     for p in [src] + [os.path.join(CSRC, x) for x in HEADERS]:
         with open(p, "rb") as f:
             h.update(f.read())
-    h.update(" ".join(ARCH + FLAGS).encode())
+    h.update(" ".join(ARCH + flags).encode())
     return h.hexdigest()[:16]
 
 
-def _compile(nvcc, name, verbose):
+def _compile(nvcc, name, verbose, build_dir, flags):
     src = os.path.join(CSRC, name)
-    obj = os.path.join(BUILD, name.replace(".cu", ".o"))
+    obj = os.path.join(build_dir, name.replace(".cu", ".o"))
     stamp = obj + ".sha"
-    dig = _digest(src)
+    dig = _digest(src, flags)
     if os.path.exists(obj) and os.path.exists(stamp) and open(stamp).read() == dig:
         return obj, ""
-    cmd = [nvcc, *ARCH, *FLAGS, "-c", src, "-o", obj]
+    cmd = [nvcc, *ARCH, *flags, "-c", src, "-o", obj]
     r = subprocess.run(cmd, capture_output=True, text=True)
     if r.returncode != 0:
         raise RuntimeError(f"nvcc failed for {name}:\n{r.stdout}\n{r.stderr}")
@@ -56,11 +63,22 @@ def _compile(nvcc, name, verbose):
     return obj, (r.stderr if verbose else "")
 
 
-def build(verbose: bool = False) -> str:
-    os.makedirs(BUILD, exist_ok=True)
+def lib_path(debug: bool | None = None) -> str:
+    if debug is None:
+        debug = os.environ.get("NVFP4_DEBUG") == "1"
+    return os.path.join(BUILD_DEBUG if debug else BUILD, "libnvfp4.so")
+
+
+def build(verbose: bool = False, debug: bool | None = None) -> str:
+    if debug is None:
+        debug = os.environ.get("NVFP4_DEBUG") == "1"
+    build_dir = BUILD_DEBUG if debug else BUILD
+    flags = FLAGS + (["-DNVFP4_DEBUG"] if debug else [])
+    LIB = lib_path(debug)
+    os.makedirs(build_dir, exist_ok=True)
     nvcc = _nvcc()
     with cf.ThreadPoolExecutor(max_workers=len(SOURCES)) as ex:
-        results = list(ex.map(lambda s: _compile(nvcc, s, verbose), SOURCES))
+        results = list(ex.map(lambda s: _compile(nvcc, s, verbose, build_dir, flags), SOURCES))
     objs = [o for o, _ in results]
     for _, log in results:
         if log:
@@ -78,4 +96,4 @@ def build(verbose: bool = False) -> str:
 
 
 if __name__ == "__main__":
-    print(build(verbose="-v" in sys.argv))
+    print(build(verbose="-v" in sys.argv, debug=True if "--debug" in sys.argv else None))

@@ -86,6 +86,7 @@ NVFP4_API const char* nvfp4_status_string(nvfp4_status s) {
     case NVFP4_ERR_CUDA: return "CUDA error";
     case NVFP4_ERR_TIMEOUT: return "bounded device wait timed out";
     case NVFP4_ERR_CAPACITY: return "KV cache capacity exceeded";
+    case NVFP4_ERR_BOUNDS: return "store index out of bounds (bounds-checked build)";
   }
   return "unknown status";
 }

@@ -539,16 +539,22 @@ __global__ void __launch_bounds__(kD) attn_combine_kernel(const float* __restric
       : "=r"(pair)
       : "f"(other), "f"(mine));
   const uint32_t row = blockIdx.y, head = blockIdx.x, c = threadIdx.x;
-  if ((c & 1) == 0)
-    out.codes[static_cast<size_t>(row) * (gridDim.x * (kD / 2)) + head * (kD / 2) + c / 2] =
-        g_ok ? static_cast<uint8_t>(pair & 0xFFu) : 0;
+  const uint32_t padded = (static_cast<uint32_t>(out.rows) + 127u) & ~127u;
+  const uint64_t code_bytes = static_cast<uint64_t>(out.rows) * gridDim.x * (kD / 2);
+  const uint64_t scale_bytes = static_cast<uint64_t>(padded) * out.kgroups * 4;
+  const uint64_t code_off = static_cast<uint64_t>(row) * (gridDim.x * (kD / 2)) + head * (kD / 2) + c / 2;
+  if ((c & 1) == 0 && in_bounds(out.status, code_off < code_bytes))
+    out.codes[code_off] = g_ok ? static_cast<uint8_t>(pair & 0xFFu) : 0;
   const uint32_t kb = head * (kD / 16) + c / 16;
-  if ((c & 15) == 0) out.scales[mma_scale_offset(row, kb, out.kgroups)] = g_ok ? static_cast<uint8_t>(bs.code) : 0;
+  const uint64_t sc_off = mma_scale_offset(row, kb, out.kgroups);
+  if ((c & 15) == 0 && in_bounds(out.status, sc_off < scale_bytes))
+    out.scales[sc_off] = g_ok ? static_cast<uint8_t>(bs.code) : 0;
   // Rows from batch up to the next multiple of 128 hold zero scales.
   if (row == 0 && c < kD / 16) {
-    const uint32_t padded = (static_cast<uint32_t>(out.rows) + 127u) & ~127u;
-    for (uint32_t pr = out.rows; pr < padded; ++pr)
-      out.scales[mma_scale_offset(pr, head * (kD / 16) + c, out.kgroups)] = 0;
+    for (uint32_t pr = out.rows; pr < padded; ++pr) {
+      const uint64_t off = mma_scale_offset(pr, head * (kD / 16) + c, out.kgroups);
+      if (in_bounds(out.status, off < scale_bytes)) out.scales[off] = 0;
+    }
   }
 }
 

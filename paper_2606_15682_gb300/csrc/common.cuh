@@ -84,6 +84,20 @@ __device__ __forceinline__ void set_status(int* status, int code) {
   if (status) atomicCAS(status, 0, code);
 }
 
+// Bounds-checked build (-DNVFP4_DEBUG): a computed store index checked
+// against the extent the kernel derives from its shape arguments.  A failed
+// check sets NVFP4_ERR_BOUNDS and the caller skips the store (no trap).  In
+// the release build the check is the constant true and the condition is
+// never evaluated for its effect.
+#ifdef NVFP4_DEBUG
+__device__ __forceinline__ bool in_bounds(int* status, bool ok) {
+  if (!ok) set_status(status, NVFP4_ERR_BOUNDS);
+  return ok;
+}
+#else
+__device__ __forceinline__ bool in_bounds(int*, bool) { return true; }
+#endif
+
 __device__ __forceinline__ uint64_t globaltimer_ns() {
   uint64_t t;
   asm volatile("mov.u64 %0, %globaltimer;" : "=l"(t));

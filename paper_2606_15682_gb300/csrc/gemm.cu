@@ -835,9 +835,14 @@ __global__ void __launch_bounds__(C::kThreads, 1)
       if (mb < args.tiles_m) {
         // Scales for every row of the 128-row tile (rows past M hold zeros: A's
         // missing rows load as zeros), codes for rows < M.
-        *reinterpret_cast<uint32_t*>(args.q_scales + mma_scale_offset(row, oc0 / 16, q_kgroups)) = sc;
-        if (row < static_cast<uint32_t>(args.M)) {
-          uint4* dst = reinterpret_cast<uint4*>(args.q_codes + static_cast<uint64_t>(row) * (q_cols / 2) + oc0 / 2);
+        const uint64_t sc_off = mma_scale_offset(row, oc0 / 16, q_kgroups);
+        const uint64_t sc_bytes = static_cast<uint64_t>((args.M + 127) & ~127) * (q_cols / 16);
+        if (in_bounds(args.status, sc_off % 4 == 0 && sc_off + 4 <= sc_bytes))
+          *reinterpret_cast<uint32_t*>(args.q_scales + sc_off) = sc;
+        const uint64_t code_off = static_cast<uint64_t>(row) * (q_cols / 2) + oc0 / 2;
+        if (row < static_cast<uint32_t>(args.M) &&
+            in_bounds(args.status, code_off + 32 <= static_cast<uint64_t>(args.M) * (q_cols / 2))) {
+          uint4* dst = reinterpret_cast<uint4*>(args.q_codes + code_off);
           dst[0] = make_uint4(codes[0], codes[1], codes[2], codes[3]);
           dst[1] = make_uint4(codes[4], codes[5], codes[6], codes[7]);
         }

@@ -86,6 +86,7 @@ __global__ void __launch_bounds__(kThreads) kv_append_kernel(
       continue;
     }
     const uint64_t row = (static_cast<uint64_t>(b) * hkv.d + h) * capacity + static_cast<uint32_t>(p);
+    if (!in_bounds(status, row < static_cast<uint64_t>(batch) * hkv.d * capacity && j < 16u)) continue;
     uint8_t* codes = is_v ? vc : kc;
     uint8_t* scales = is_v ? vs : ks;
     reinterpret_cast<uint32_t*>(codes + row * 64)[j] = packed;

@@ -119,8 +119,11 @@ __device__ __forceinline__ uint32_t amax_bits_of(const BlockSlots& sl) {
 template <bool kMMA>
 __device__ __forceinline__ void quantize_loaded(const BlockSlots& sl, uint32_t total_blocks, uint32_t kblocks,
                                                 uint32_t bidx0, uint32_t stride, uint32_t lane, float g, float six_g,
-                                                bool g_ok, uint2* __restrict__ codes, uint8_t* __restrict__ scales) {
+                                                bool g_ok, uint2* __restrict__ codes, uint8_t* __restrict__ scales, int* status) {
   const uint32_t kgroups = kblocks >> 2;
+  // Scale bytes the kernel may write: padded rows in the MMA layout.
+  const uint64_t scale_bytes =
+      kMMA ? static_cast<uint64_t>((total_blocks / kblocks + 127u) & ~127u) * kblocks : total_blocks;
 #pragma unroll
   for (int u = 0; u < kUnroll; ++u) {
     const uint32_t b = bidx0 + u * stride + lane;
@@ -143,22 +146,26 @@ __device__ __forceinline__ void quantize_loaded(const BlockSlots& sl, uint32_t t
       uint32_t w = sc << (8 * (lane & 3));
       w |= __shfl_xor_sync(0xffffffffu, w, 1);
       w |= __shfl_xor_sync(0xffffffffu, w, 2);
-      if (live && (lane & 3) == 0)
-        *reinterpret_cast<uint32_t*>(scales + mma_scale_offset(sl.row[u], sl.kb[u], kgroups)) = w;
+      const uint64_t off = mma_scale_offset(sl.row[u], sl.kb[u], kgroups);
+      if (live && (lane & 3) == 0 && in_bounds(status, off % 4 == 0 && off + 4 <= scale_bytes))
+        *reinterpret_cast<uint32_t*>(scales + off) = w;
     } else if (live) {
-      scales[static_cast<uint64_t>(sl.row[u]) * kblocks + sl.kb[u]] = static_cast<uint8_t>(sc);
+      const uint64_t off = static_cast<uint64_t>(sl.row[u]) * kblocks + sl.kb[u];
+      if (in_bounds(status, off < scale_bytes)) scales[off] = static_cast<uint8_t>(sc);
     }
   }
 }
 
 // Zero the MMA-layout scales of the padding rows up to the next multiple of 128.
-__device__ __forceinline__ void zero_scale_padding(uint32_t rows, uint32_t kblocks, uint8_t* __restrict__ scales) {
+__device__ __forceinline__ void zero_scale_padding(uint32_t rows, uint32_t kblocks, uint8_t* __restrict__ scales,
+                                                   int* status) {
   const uint32_t kgroups = kblocks >> 2;
   const uint32_t padded = (rows + 127u) & ~127u;
   const uint32_t pad = (padded - rows) * kblocks;
   for (uint32_t i = blockIdx.x * blockDim.x + threadIdx.x; i < pad; i += gridDim.x * blockDim.x) {
     const uint32_t r = rows + i / kblocks, k = i % kblocks;
-    scales[mma_scale_offset(r, k, kgroups)] = 0;
+    const uint64_t off = mma_scale_offset(r, k, kgroups);
+    if (in_bounds(status, off < static_cast<uint64_t>(padded) * kblocks)) scales[off] = 0;
   }
 }
 
@@ -170,7 +177,7 @@ template <bool kMMA>
 __device__ __forceinline__ void quantize_blocks(const uint16_t* __restrict__ x, FastDiv kblocks_div,
                                                 uint32_t total_blocks, int64_t ld, bool dense, uint32_t rows,
                                                 float g, bool g_ok, uint2* __restrict__ codes,
-                                                uint8_t* __restrict__ scales) {
+                                                uint8_t* __restrict__ scales, int* status) {
   const float six_g = __fmul_rn(6.0f, g);
   const uint32_t lane = threadIdx.x & 31;
   const uint32_t stride = gridDim.x * blockDim.x;
@@ -178,9 +185,10 @@ __device__ __forceinline__ void quantize_blocks(const uint16_t* __restrict__ x, 
   for (uint32_t bidx0 = blockIdx.x * blockDim.x + (threadIdx.x & ~31u); bidx0 < total_blocks; bidx0 += stride * kUnroll) {
     BlockSlots sl;
     load_blocks(x, kblocks_div, total_blocks, ld, dense, bidx0, stride, lane, sl);
-    quantize_loaded<kMMA>(sl, total_blocks, kblocks_div.d, bidx0, stride, lane, g, six_g, g_ok, codes, scales);
+    quantize_loaded<kMMA>(sl, total_blocks, kblocks_div.d, bidx0, stride, lane, g, six_g, g_ok, codes, scales,
+                          status);
   }
-  if (kMMA) zero_scale_padding(rows, kblocks_div.d, scales);
+  if (kMMA) zero_scale_padding(rows, kblocks_div.d, scales, status);
 }
 
 template <bool kMMA>
@@ -193,7 +201,8 @@ __global__ void __launch_bounds__(kThreads) quantize_kernel(const uint16_t* __re
   const float g_in = *g_ptr;
   const bool g_ok = g_in > 0.0f && g_in <= FLT_MAX;
   if (!g_ok && blockIdx.x == 0 && threadIdx.x == 0) set_status(status, NVFP4_ERR_INVALID_ARG);
-  quantize_blocks<kMMA>(x, kblocks_div, total_blocks, ld, dense, rows, g_ok ? g_in : 1.0f, g_ok, codes, scales);
+  quantize_blocks<kMMA>(x, kblocks_div, total_blocks, ld, dense, rows, g_ok ? g_in : 1.0f, g_ok, codes, scales,
+                        status);
 }
 
 __device__ __forceinline__ unsigned long long ld_acquire_u64(const unsigned long long* p) {
@@ -300,7 +309,8 @@ __global__ void __launch_bounds__(kThreads) quantize_dynamic_kernel(
   const float six_g = __fmul_rn(6.0f, g);
   if (blockIdx.x == 0 && threadIdx.x == 0) *g_out = g;
   if (bidx_last < total_blocks)
-    quantize_loaded<kMMA>(sl, total_blocks, kblocks_div.d, bidx_last, stride, lane, g, six_g, true, codes, scales);
+    quantize_loaded<kMMA>(sl, total_blocks, kblocks_div.d, bidx_last, stride, lane, g, six_g, true, codes, scales,
+                          status);
   it = 0;
   for (uint32_t bidx0 = bidx_first; bidx0 < bidx_last; bidx0 += stride * kUnroll, ++it) {
     BlockSlots t;
@@ -317,9 +327,9 @@ __global__ void __launch_bounds__(kThreads) quantize_dynamic_kernel(
     } else {
       load_blocks(x, kblocks_div, total_blocks, ld, dense, bidx0, stride, lane, t);
     }
-    quantize_loaded<kMMA>(t, total_blocks, kblocks_div.d, bidx0, stride, lane, g, six_g, true, codes, scales);
+    quantize_loaded<kMMA>(t, total_blocks, kblocks_div.d, bidx0, stride, lane, g, six_g, true, codes, scales, status);
   }
-  if (kMMA) zero_scale_padding(rows, kblocks_div.d, scales);
+  if (kMMA) zero_scale_padding(rows, kblocks_div.d, scales, status);
 }
 
 // Blocks of quantize_dynamic_kernel that fit on the device at once (a
@@ -368,7 +378,7 @@ template <bool kMMA, bool kRotate>
 __global__ void __launch_bounds__(kThreads) mx_quantize_kernel(const uint16_t* __restrict__ x, FastDiv nb_div,
                                                                uint32_t total_blocks, int64_t ld, bool dense,
                                                                uint32_t rows, uint4* __restrict__ codes,
-                                                               uint8_t* __restrict__ scales) {
+                                                               uint8_t* __restrict__ scales, int* status) {
   griddep_wait_and_release();
   const uint32_t nb = nb_div.d;           // 32-element blocks per row
   const uint32_t kgroups = nb >> 1;       // 64-element scale groups per row (MMA layout)
@@ -411,14 +421,17 @@ __global__ void __launch_bounds__(kThreads) mx_quantize_kernel(const uint16_t* _
         // 64-element group (nb is even, so a group never straddles rows).
         uint32_t w = (code | (code << 8)) << (16 * (lane & 1));
         w |= __shfl_xor_sync(0xffffffffu, w, 1);
-        if (live && (lane & 1) == 0)
-          *reinterpret_cast<uint32_t*>(scales + mma_scale_offset(row[u], 2 * j[u], kgroups)) = w;
+        const uint64_t off = mma_scale_offset(row[u], 2 * j[u], kgroups);
+        if (live && (lane & 1) == 0 &&
+            in_bounds(status, off % 4 == 0 && off + 4 <= static_cast<uint64_t>((rows + 127u) & ~127u) * 2 * nb))
+          *reinterpret_cast<uint32_t*>(scales + off) = w;
       } else if (live) {
-        scales[static_cast<uint64_t>(row[u]) * nb + j[u]] = static_cast<uint8_t>(code);
+        const uint64_t off = static_cast<uint64_t>(row[u]) * nb + j[u];
+        if (in_bounds(status, off < total_blocks)) scales[off] = static_cast<uint8_t>(code);
       }
     }
   }
-  if (kMMA) zero_scale_padding(rows, nb * 2, scales);
+  if (kMMA) zero_scale_padding(rows, nb * 2, scales, status);
 }
 
 template <bool kToMMA>
@@ -630,7 +643,8 @@ NVFP4_API nvfp4_status mxfp4_quantize(const void* x_bf16, int64_t rows, int64_t 
                     : (rotate ? mx_quantize_kernel<false, true> : mx_quantize_kernel<false, false>);
   const cudaError_t e = launch_pdl(kernel, dim3(grid), dim3(kThreads), 0, static_cast<cudaStream_t>(stream),
                                    static_cast<const uint16_t*>(x_bf16), FastDiv(nb), total_blocks, ld, ld == cols,
-                                   static_cast<uint32_t>(rows), reinterpret_cast<uint4*>(codes), scales);
+                                   static_cast<uint32_t>(rows), reinterpret_cast<uint4*>(codes), scales,
+                                   status_word_dev());
   if (e != cudaSuccess) return NVFP4_ERR_CUDA;
   count_launches(1);
   return launch_status();

@@ -27,6 +27,7 @@ def test_status_strings_and_sizes():
     N = lib()
     assert N.nvfp4_status_string(0) == "ok"
     assert "capacity" in N.nvfp4_status_string(7)
+    assert "bounds" in N.nvfp4_status_string(8)
     assert N.nvfp4_scales_bytes(130, 256, N.SCALES_ROWMAJOR) == 130 * 16
     assert N.nvfp4_scales_bytes(130, 256, N.SCALES_MMA) == 256 * 16
     assert N.decode_attention_nvfp4_workspace_size(64, 40, 16384) > 0
