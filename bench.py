@@ -46,11 +46,11 @@ CSRC = os.path.join(ROOT, "paper_2606_15682_gb300", "csrc")
 # same kernel and shape (commands in profiles/).  Each entry holds only while the kernel sources
 # hash to the value they had at capture time; otherwise the line reports traffic = null.
 NCU_TRAFFIC = {
-    "gemm": {"bytes": 17294336 + 11984128, "sources": ("gemm.cu", "common.cuh"), "sha": "c82c2ce095dbf4e2",
+    "gemm": {"bytes": 17296384 + 11984640, "sources": ("gemm.cu", "common.cuh"), "sha": "6a81315cc83b08bd",
              "shape": (2048, 17920, 1536),
              "profile": "profiles/gemm_qwen1.5b_prefill_gate_up_m2048_n17920_k1536.md"},
-    "attention": {"bytes": 1208721920 + 21919232, "sources": ("attention.cu", "common.cuh"),
-                  "sha": "0ce677bc4a92a5a4", "shape": (64, 16384),
+    "attention": {"bytes": 1208783616 + 22233856, "sources": ("attention.cu", "common.cuh"),
+                  "sha": "b4d25eaf23259ae3", "shape": (64, 16384),
                   "profile": "profiles/attention_qwen14b_decode_b64_t16384.md (attn_partial_kernel)"},
 }
 
