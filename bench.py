@@ -423,7 +423,10 @@ def run_ours(args, rank, world):
                   "gemm_roofline": {L["name"]: roofline_of(2 * Mw * L["N"] * L["K"], gemm_bytes(Mw, L["N"], L["K"]),
                                                            statistics.median(g_ms[L["name"]])) for L in lw},
                   "quantize_us": {k: 1e3 * statistics.median(v) for k, v in q_ms.items()},
-                  "quantize_gbs": {k: q_bytes[k] / (statistics.median(v) * 1e-3) / 1e9 for k, v in q_ms.items()}}
+                  "quantize_gbs": {k: q_bytes[k] / (statistics.median(v) * 1e-3) / 1e9 for k, v in q_ms.items()},
+                  "quantize_roofline": {k: {"bound": "hbm", "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                                            "frac": q_bytes[k] / (statistics.median(v) * 1e-3) / 1e9 / peaks["hbm_gbs"]}
+                                        for k, v in q_ms.items()}}
         del lw, g
         torch.cuda.empty_cache()
 
