@@ -372,9 +372,10 @@ int dynamic_capacity(int stash_iters) {
 // H_32 / sqrt(32) (the block-wise rotation applied before MXFP4 quantization,
 // Sec. 4).  One thread quantizes one block per slot; no tensor-wide pass.
 // ---------------------------------------------------------------------------
-constexpr int kMxUnroll = 2;
 // Block index b (of rows * cols/32) -> its 32 bf16 elements as fp32, the row and block-in-row.
-template <bool kMMA, bool kRotate>
+// U blocks per thread per pass: 1 when one pass covers the tensor (more CTAs
+// to hide the load latency of small tensors), 2 for large ones.
+template <bool kMMA, bool kRotate, int U>
 __global__ void __launch_bounds__(kThreads) mx_quantize_kernel(const uint16_t* __restrict__ x, FastDiv nb_div,
                                                                uint32_t total_blocks, int64_t ld, bool dense,
                                                                uint32_t rows, uint4* __restrict__ codes,
@@ -384,11 +385,11 @@ __global__ void __launch_bounds__(kThreads) mx_quantize_kernel(const uint16_t* _
   const uint32_t kgroups = nb >> 1;       // 64-element scale groups per row (MMA layout)
   const uint32_t lane = threadIdx.x & 31;
   const uint32_t stride = gridDim.x * blockDim.x;
-  for (uint32_t b0 = blockIdx.x * blockDim.x + (threadIdx.x & ~31u); b0 < total_blocks; b0 += stride * kMxUnroll) {
-    uint4 v[kMxUnroll][4];
-    uint32_t row[kMxUnroll], j[kMxUnroll];
+  for (uint32_t b0 = blockIdx.x * blockDim.x + (threadIdx.x & ~31u); b0 < total_blocks; b0 += stride * U) {
+    uint4 v[U][4];
+    uint32_t row[U], j[U];
 #pragma unroll
-    for (int u = 0; u < kMxUnroll; ++u) {
+    for (int u = 0; u < U; ++u) {
       const uint32_t b = b0 + u * stride + lane;
       row[u] = nb_div.div(b);
       j[u] = b - row[u] * nb;
@@ -399,7 +400,7 @@ __global__ void __launch_bounds__(kThreads) mx_quantize_kernel(const uint16_t* _
       for (int q = 0; q < 4; ++q) v[u][q] = live ? __ldg(src + q) : make_uint4(0, 0, 0, 0);
     }
 #pragma unroll
-    for (int u = 0; u < kMxUnroll; ++u) {
+    for (int u = 0; u < U; ++u) {
       const uint32_t b = b0 + u * stride + lane;
       const bool live = b < total_blocks;
       float xf[32];
@@ -637,10 +638,13 @@ NVFP4_API nvfp4_status mxfp4_quantize(const void* x_bf16, int64_t rows, int64_t 
   if (!aligned(codes, 16)) return NVFP4_ERR_ALIGN;
   const uint32_t nb = static_cast<uint32_t>(cols / 32);
   const uint32_t total_blocks = static_cast<uint32_t>(rows * nb);
-  const int grid = grid_for(total_blocks, kThreads * kMxUnroll);
   const bool mma = layout == NVFP4_SCALES_MMA;
-  auto kernel = mma ? (rotate ? mx_quantize_kernel<true, true> : mx_quantize_kernel<true, false>)
-                    : (rotate ? mx_quantize_kernel<false, true> : mx_quantize_kernel<false, false>);
+  const bool one_pass = total_blocks <= static_cast<uint64_t>(sm_count()) * 8 * kThreads;
+  const int grid = grid_for(total_blocks, kThreads * (one_pass ? 1 : 2));
+  auto kernel = one_pass ? (mma ? (rotate ? mx_quantize_kernel<true, true, 1> : mx_quantize_kernel<true, false, 1>)
+                                : (rotate ? mx_quantize_kernel<false, true, 1> : mx_quantize_kernel<false, false, 1>))
+                         : (mma ? (rotate ? mx_quantize_kernel<true, true, 2> : mx_quantize_kernel<true, false, 2>)
+                                : (rotate ? mx_quantize_kernel<false, true, 2> : mx_quantize_kernel<false, false, 2>));
   const cudaError_t e = launch_pdl(kernel, dim3(grid), dim3(kThreads), 0, static_cast<cudaStream_t>(stream),
                                    static_cast<const uint16_t*>(x_bf16), FastDiv(nb), total_blocks, ld, ld == cols,
                                    static_cast<uint32_t>(rows), reinterpret_cast<uint4*>(codes), scales,
