@@ -23,6 +23,20 @@ def test_library_exports_every_declared_symbol():
     assert sorted(N.EXPORTED) == header_functions()
 
 
+def test_bounds_checked_build_compiles_and_exports_every_call():
+    """The NVFP4_DEBUG variant (store indices checked, NVFP4_ERR_BOUNDS instead
+    of a write) builds and exports the same C ABI."""
+    import os
+    from paper_2606_15682_gb300 import build as B
+    path = B.build(debug=True)
+    assert os.path.basename(os.path.dirname(path)) == "_build_debug"
+    so = ctypes.CDLL(path)
+    for name in header_functions():
+        assert hasattr(so, name), name
+    so.nvfp4_status_string.restype = ctypes.c_char_p
+    assert b"bounds" in so.nvfp4_status_string(8)
+
+
 def test_status_strings_and_sizes():
     N = lib()
     assert N.nvfp4_status_string(0) == "ok"
