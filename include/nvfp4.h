@@ -420,6 +420,10 @@ nvfp4_status decode_attention_nvfp4_quantize(const nvfp4_kv_cache* cache, const 
  *   - The first call on a device looks up the device address of the array
  *     (a one-time host-side query); make that first call before capturing
  *     stream work into a CUDA graph.
+ *   - The looked-up address is kept per device ordinal until the process
+ *     exits.  Resetting the device (cudaDeviceReset) after the first call is
+ *     not supported: the kept address, like that of the device status word,
+ *     would then point into a freed context.
  * Errors: as decode_attention_nvfp4.
  */
 #define NVFP4_ATTN_STATIC_SCRATCH_BYTES (24u << 20)

@@ -4,16 +4,12 @@
 //
 //   out[m, n] = bf16( g_a g_w sum_k a[m,k] w[n,k] )      (all linears, Appendix D.1)
 //
-// Persistent, warp-specialized CTAs (one per SM), tile 128 x BN x 256, launched
-// in clusters of CM CTAs that work on CM consecutive 128-row tiles of the
-// same BN-column tile:
-//   warp 0      TMA producer: its own A tile (codes via a 2-D tensor map with
-//               the 128-byte swizzle) and A block scales (1-D bulk copy), plus
-//               1/CM of the shared W tile and W scales, multicast to every CTA
-//               of the cluster -- W bytes leave L2 once per cluster.
+// Persistent, warp-specialized CTAs (one per SM), tile 128 x BN x 256:
+//   warp 0      TMA producer: the A and W tiles (codes via 2-D tensor maps
+//               with the 128-byte swizzle) and their block scales (1-D bulk
+//               copies).
 //   warp 1      allocates 512 TMEM columns; one lane issues 4 MMAs of K = 64
-//               per stage; its commit releases the stage in every CTA of the
-//               cluster.
+//               per stage; its commit releases the stage.
 //   warp 2      one lane copies each stage's block scales smem -> TMEM
 //               (tcgen05.cp) as soon as the stage lands, so the copies run
 //               ahead of, and in a different issue stream from, the MMAs.
@@ -51,11 +47,10 @@ constexpr uint32_t kEpiBufBytes = kEpiRows * kEpiCols * 2;  // 4 KiB per epilogu
 // BN = 128: double-buffered TMEM accumulator, 4 epilogue warps.  BN = 256:
 // one accumulator (TMEM also holds the scale slots) and 8 epilogue warps that
 // drain it into registers and release it before storing.
-template <int BN_, int STAGES_, int CM_>
+template <int BN_, int STAGES_>
 struct Cfg {
   static constexpr int BN = BN_;
   static constexpr int kStages = STAGES_;
-  static constexpr int CM = CM_;  // cluster size along M
   static constexpr int kAccBufs = BN == 128 ? 2 : 1;
   static constexpr int kEpiWarps = BN / 32;  // 128 accumulator columns each
   static constexpr int kThreads = 96 + 32 * kEpiWarps;  // producer, MMA, scale copier, epilogue
@@ -64,8 +59,6 @@ struct Cfg {
   static constexpr uint32_t kSfaBytes = 128 * (BK / 16);  // four 512-byte scale atoms
   static constexpr uint32_t kSfbBytes = kSfaBytes * (BN / 128);
   static constexpr uint32_t kStageBytes = kTileBytesA + kTileBytesB + kSfaBytes + kSfbBytes;
-  static constexpr int kBRowsPerCta = BN / CM;           // W rows each CTA loads and multicasts
-  static constexpr uint32_t kSfbSlice = kSfbBytes / CM;  // W scale bytes each CTA loads
   static constexpr uint32_t kSfbColsPerMma = 4 * (BN / 128);
   static constexpr uint32_t kSfCols = 16 + 4 * kSfbColsPerMma;  // TMEM columns of one stage's scales
   static constexpr uint32_t kSfTmemCol = kAccBufs * BN;
@@ -77,8 +70,6 @@ struct Cfg {
                                      (static_cast<uint32_t>(BM >> 4) << 24);
   static_assert(kSfTmemCol + kStages * kSfCols <= kTmemCols, "TMEM budget");
   static_assert(kSmemBytes <= 227 * 1024, "shared memory budget");
-  static_assert(kBRowsPerCta % 8 == 0 && kSfbSlice % 16 == 0, "multicast slice granularity");
-  static_assert(kSfbSlice <= kSfaBytes || kSfbSlice % kSfaBytes == 0, "scale slices stay inside 128-row tiles");
 };
 
 // Shared-memory matrix descriptor of a K-major operand tile stored with the
@@ -179,7 +170,6 @@ __global__ void __launch_bounds__(C::kThreads, 1)
                       const __grid_constant__ CUtensorMap tmap_out, const GemmArgs args) {
   constexpr int BN = C::BN;
   constexpr int kStages = C::kStages;
-  constexpr int CM = C::CM;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* sA = smem;
@@ -200,17 +190,15 @@ __global__ void __launch_bounds__(C::kThreads, 1)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int kblocks = args.K / BK;
   const int kgroups = args.K / 64;
-  const uint32_t rank = CM > 1 ? cluster_ctarank() : 0;
-  const uint16_t cluster_mask = static_cast<uint16_t>((1u << CM) - 1);
-  // Work unit: CM consecutive 128-row tiles x one BN-column tile, one per cluster.
-  const int msup = (args.tiles_m + CM - 1) / CM;
+  // Work unit: one 128-row tile x one BN-column tile.
+  const int msup = args.tiles_m;
   const int total_units = msup * args.tiles_n;
-  const int cluster_id = blockIdx.x / CM, n_clusters = gridDim.x / CM;
+  const int cta_id = blockIdx.x, n_ctas = gridDim.x;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
       mbar_init(&full[s], 1);
-      mbar_init(&empty[s], CM);  // one MMA commit from every CTA reading the stage
+      mbar_init(&empty[s], 1);  // the MMA commit that retires the stage
       mbar_init(&sfready[s], 1);
     }
     for (int a = 0; a < 2; ++a) {
@@ -230,8 +218,7 @@ __global__ void __launch_bounds__(C::kThreads, 1)
     tmem_relinquish();
   }
   tc_fence_before();
-  if (CM > 1) cluster_sync_all();  // peers' barriers exist before any multicast lands
-  else __syncthreads();
+  __syncthreads();
   tc_fence_after();
   griddep_wait_and_release();
   const uint32_t tmem = *tmem_slot;
@@ -248,10 +235,10 @@ __global__ void __launch_bounds__(C::kThreads, 1)
     uint32_t issued_parity[kStages];
     bool issued[kStages];
     for (int s = 0; s < kStages; ++s) issued[s] = false;
-    for (int u = cluster_id; u < total_units && !abort_flag; u += n_clusters) {
+    for (int u = cta_id; u < total_units && !abort_flag; u += n_ctas) {
       int ms, nb;
       unit_coords(u, msup, args.tiles_n, &ms, &nb);
-      const int mb = min(ms * CM + static_cast<int>(rank), args.tiles_m - 1);  // spare CTAs redo the last tile
+      const int mb = ms;
       const uint8_t* sfa_tile = args.sfa + (static_cast<size_t>(mb) * kgroups) * 512;
       const uint8_t* sfb_tiles = args.sfb + (static_cast<size_t>(nb) * (BN / 128) * kgroups) * 512;
       for (int kb = 0; kb < kblocks; ++kb) {
@@ -260,21 +247,13 @@ __global__ void __launch_bounds__(C::kThreads, 1)
         tma_load_2d(sA + stage * C::kTileBytesA, &tmap_a, &full[stage], kb * (BK / 2), mb * BM);
         bulk_load(sSFA + stage * C::kSfaBytes, sfa_tile + static_cast<size_t>(kb) * C::kSfaBytes, C::kSfaBytes,
                   &full[stage]);
-        // This CTA's share of the stage's W scales: bytes [rank*slice, +slice) of
-        // the stage buffer, which holds BN/128 row tiles of 2 KiB each.
+        // The stage's W scales: BN/128 row tiles of 2 KiB each.
 #pragma unroll
-        for (uint32_t off = rank * C::kSfbSlice; off < (rank + 1) * C::kSfbSlice; off += C::kSfaBytes) {
-          const uint32_t len = C::kSfbSlice < C::kSfaBytes ? C::kSfbSlice : C::kSfaBytes;
-          const uint32_t j = off / C::kSfaBytes, within = off % C::kSfaBytes;
-          const uint8_t* src =
-              sfb_tiles + (static_cast<size_t>(j) * kgroups) * 512 + static_cast<size_t>(kb) * C::kSfaBytes + within;
-          if (CM > 1) bulk_load_mc(sSFB + stage * C::kSfbBytes + off, src, len, &full[stage], cluster_mask);
-          else bulk_load(sSFB + stage * C::kSfbBytes + off, src, len, &full[stage]);
-        }
-        uint8_t* b_dst = sB + stage * C::kTileBytesB + rank * C::kBRowsPerCta * (BK / 2);
-        const int b_row = nb * BN + static_cast<int>(rank) * C::kBRowsPerCta;
-        if (CM > 1) tma_load_2d_mc(b_dst, &tmap_b, &full[stage], kb * (BK / 2), b_row, cluster_mask);
-        else tma_load_2d(b_dst, &tmap_b, &full[stage], kb * (BK / 2), b_row);
+        for (int j = 0; j < BN / 128; ++j)
+          bulk_load(sSFB + stage * C::kSfbBytes + j * C::kSfaBytes,
+                    sfb_tiles + (static_cast<size_t>(j) * kgroups) * 512 + static_cast<size_t>(kb) * C::kSfaBytes,
+                    C::kSfaBytes, &full[stage]);
+        tma_load_2d(sB + stage * C::kTileBytesB, &tmap_b, &full[stage], kb * (BK / 2), nb * BN);
         issued[stage] = true;
         issued_parity[stage] = phase;
         if (++stage == kStages) { stage = 0; phase ^= 1u; }
@@ -291,7 +270,7 @@ __global__ void __launch_bounds__(C::kThreads, 1)
     uint32_t phase = 0;
     int local = 0;
     const uint32_t sA0 = smem_u32(sA), sB0 = smem_u32(sB), sSFA0 = smem_u32(sSFA), sSFB0 = smem_u32(sSFB);
-    for (int u = cluster_id; u < total_units && !abort_flag; u += n_clusters, ++local) {
+    for (int u = cta_id; u < total_units && !abort_flag; u += n_ctas, ++local) {
       const int acc = local % C::kAccBufs;
       const uint32_t acc_phase = (local / C::kAccBufs) & 1;
       if (!mbar_wait_bounded(&tempty[acc], acc_phase ^ 1u, &abort_flag)) { fail(); break; }
@@ -309,8 +288,7 @@ __global__ void __launch_bounds__(C::kThreads, 1)
                   desc_sw128(sB0 + stage * C::kTileBytesB + kk * 32), C::kIdesc | args.idesc_fmt, sfa_col + kk * 4,
                   sfb_col + kk * C::kSfbColsPerMma, (kb | kk) != 0);
         }
-        if (CM > 1) tc_commit_mc(&empty[stage], cluster_mask);
-        else tc_commit(&empty[stage]);
+        tc_commit(&empty[stage]);
         if (++stage == kStages) { stage = 0; phase ^= 1u; }
       }
       if (!ok) break;
@@ -326,7 +304,7 @@ __global__ void __launch_bounds__(C::kThreads, 1)
     int stage = 0;
     uint32_t phase = 0;
     const uint32_t sSFA0 = smem_u32(sSFA), sSFB0 = smem_u32(sSFB);
-    for (int u = cluster_id; u < total_units && !abort_flag; u += n_clusters) {
+    for (int u = cta_id; u < total_units && !abort_flag; u += n_ctas) {
       bool ok = true;
       for (int kb = 0; kb < kblocks; ++kb) {
         if (!mbar_wait_bounded(&full[stage], phase, &abort_flag)) { fail(); ok = false; break; }
@@ -356,10 +334,10 @@ __global__ void __launch_bounds__(C::kThreads, 1)
     const uint32_t buf = smem_u32(buf_ptr);
     const float scale = args.ga ? __fmul_rn(__ldg(args.ga), __ldg(args.gb)) : 1.0f;
     int local = 0;
-    for (int u = cluster_id; u < total_units; u += n_clusters, ++local) {
+    for (int u = cta_id; u < total_units; u += n_ctas, ++local) {
       int ms, nb;
       unit_coords(u, msup, args.tiles_n, &ms, &nb);
-      const int mb = ms * CM + static_cast<int>(rank);  // spare CTAs (mb >= tiles_m) store nothing
+      const int mb = ms;
       const int acc = local % C::kAccBufs;
       const uint32_t acc_phase = (local / C::kAccBufs) & 1;
       // Lane 0 waits and broadcasts, so the warp stays converged for the
@@ -409,8 +387,7 @@ __global__ void __launch_bounds__(C::kThreads, 1)
   }
 
   tc_fence_before();
-  if (CM > 1) cluster_sync_all();  // no peer may still multicast into, or arrive on, this CTA
-  else __syncthreads();
+  __syncthreads();
   tc_fence_after();
   if (warp == 1) tmem_dealloc(tmem, kTmemCols);
 }
@@ -969,7 +946,7 @@ bool make_out_map(CUtensorMap* map, void* base, int64_t M, int64_t N, int64_t ld
 // Per-device, per-configuration launch set-up: the shared-memory opt-in and
 // the number of clusters resident on the GPU at once (persistent grid).
 template <class C>
-int resident_clusters() {
+int resident_ctas() {
   static std::mutex mu;
   static std::map<int, int> cache;
   int d = 0;
@@ -980,26 +957,7 @@ int resident_clusters() {
   if (cudaFuncSetAttribute(nvfp4_gemm_kernel<C>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                            static_cast<int>(C::kSmemBytes)) != cudaSuccess)
     return 0;
-  int n = sm_count() / C::CM;
-  if (C::CM > 1) {
-    cudaLaunchConfig_t cfg = {};
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeClusterDimension;
-    attr[0].val.clusterDim.x = C::CM;
-    attr[0].val.clusterDim.y = 1;
-    attr[0].val.clusterDim.z = 1;
-    cfg.gridDim = dim3(C::CM * n, 1, 1);
-    cfg.blockDim = dim3(C::kThreads, 1, 1);
-    cfg.dynamicSmemBytes = C::kSmemBytes;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    int clusters = 0;
-    if (cudaOccupancyMaxActiveClusters(&clusters, nvfp4_gemm_kernel<C>, &cfg) != cudaSuccess || clusters <= 0) {
-      cudaGetLastError();
-      return 0;
-    }
-    n = clusters;
-  }
+  const int n = sm_count();  // one CTA per SM (launch bounds and shared memory allow no more)
   cache[d] = n;
   return n;
 }
@@ -1009,14 +967,14 @@ nvfp4_status launch(const uint8_t* a_codes, const uint8_t* a_scales, const float
                     const uint8_t* w_scales, const float* g_w, int64_t M, int64_t N, int64_t K, void* out_bf16,
                     int64_t ldo, cudaStream_t stream, uint32_t idesc_fmt) {
   const int64_t tiles_m = (M + BM - 1) / BM, tiles_n = (N + C::BN - 1) / C::BN;
-  const int64_t units = ((tiles_m + C::CM - 1) / C::CM) * tiles_n;
+  const int64_t units = tiles_m * tiles_n;
   if (units >= (1ll << 31)) return NVFP4_ERR_SHAPE;
   CUtensorMap ma, mb, mo;
-  if (!make_code_map(&ma, a_codes, M, K, BM) || !make_code_map(&mb, w_codes, N, K, C::kBRowsPerCta) ||
+  if (!make_code_map(&ma, a_codes, M, K, BM) || !make_code_map(&mb, w_codes, N, K, C::BN) ||
       !make_out_map(&mo, out_bf16, M, N, ldo))
     return NVFP4_ERR_CUDA;
-  const int clusters_max = resident_clusters<C>();
-  if (clusters_max <= 0) return NVFP4_ERR_CUDA;
+  const int ctas_max = resident_ctas<C>();
+  if (ctas_max <= 0) return NVFP4_ERR_CUDA;
   GemmArgs args = {};
   args.idesc_fmt = idesc_fmt;
   args.sfa = a_scales;
@@ -1029,22 +987,10 @@ nvfp4_status launch(const uint8_t* a_codes, const uint8_t* a_scales, const float
   args.tiles_m = static_cast<int>(tiles_m);
   args.tiles_n = static_cast<int>(tiles_n);
   args.status = status_word_dev();
-  const int clusters = static_cast<int>(units < clusters_max ? units : clusters_max);
-  cudaLaunchConfig_t cfg = {};
-  cudaLaunchAttribute attr[2];
-  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[1].val.programmaticStreamSerializationAllowed = 1;
-  attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = C::CM;
-  attr[0].val.clusterDim.y = 1;
-  attr[0].val.clusterDim.z = 1;
-  cfg.gridDim = dim3(clusters * C::CM, 1, 1);
-  cfg.blockDim = dim3(C::kThreads, 1, 1);
-  cfg.dynamicSmemBytes = C::kSmemBytes;
-  cfg.stream = stream;
-  cfg.attrs = attr;
-  cfg.numAttrs = 2;
-  if (cudaLaunchKernelEx(&cfg, nvfp4_gemm_kernel<C>, ma, mb, mo, args) != cudaSuccess) return NVFP4_ERR_CUDA;
+  const int ctas = static_cast<int>(units < ctas_max ? units : ctas_max);
+  if (launch_pdl(nvfp4_gemm_kernel<C>, dim3(ctas), dim3(C::kThreads), C::kSmemBytes, stream, ma, mb, mo, args) !=
+      cudaSuccess)
+    return NVFP4_ERR_CUDA;
   count_launches(1);
   return launch_status();
 }
@@ -1139,9 +1085,6 @@ nvfp4_status launch_pair(const uint8_t* a_codes, const uint8_t* a_scales, const 
 #ifndef NVFP4_GEMM_BN
 #define NVFP4_GEMM_BN 0  // 0: choose per shape
 #endif
-#ifndef NVFP4_GEMM_CM
-#define NVFP4_GEMM_CM 0  // 0: choose per shape
-#endif
 #ifndef NVFP4_GEMM_PAIR
 #define NVFP4_GEMM_PAIR 1  // 0: never use the CTA-pair kernel
 #endif
@@ -1175,10 +1118,6 @@ nvfp4_status linear_dispatch(const uint8_t* a_codes, const uint8_t* a_scales, co
                              const uint8_t* w_codes, const uint8_t* w_scales, const float* g_w, int64_t M, int64_t N,
                              int64_t K, void* out_bf16, int64_t ldo, cudaStream_t s, uint32_t idesc_fmt) {
   const int64_t tiles_m = (M + BM - 1) / BM;
-  // Measured on GB300: sharing W tiles by cluster multicast did not beat
-  // independent CTAs on these shapes (the cluster waits for its slowest CTA),
-  // so clusters are off by default; the multicast path stays selectable.
-  const int cm = NVFP4_GEMM_CM ? NVFP4_GEMM_CM : 1;
   // The CTA pair, unless its 256 x 256 tiles would leave most pairs idle
   // (decode-sized M): then 128 x 128 tiles on single CTAs spread the W stream
   // over more SMs (measured faster at M = 256 with N = 5120 or 7168, slower
@@ -1195,18 +1134,9 @@ nvfp4_status linear_dispatch(const uint8_t* a_codes, const uint8_t* a_scales, co
   }
   // Single CTAs: BN = 128 (measured faster than 256 at M <= 256 on GB300).
   const int bn = NVFP4_GEMM_BN ? NVFP4_GEMM_BN : 128;
-#define NVFP4_LAUNCH(BN_, ST_, CM_) \
-  return launch<Cfg<BN_, ST_, CM_>>(a_codes, a_scales, g_a, w_codes, w_scales, g_w, M, N, K, out_bf16, ldo, s, \
-                                    idesc_fmt)
-  if (bn == 256) {
-    if (cm >= 4) NVFP4_LAUNCH(256, 3, 4);
-    if (cm == 2) NVFP4_LAUNCH(256, 3, 2);
-    NVFP4_LAUNCH(256, 3, 1);
-  }
-  if (cm >= 4) NVFP4_LAUNCH(128, 5, 4);
-  if (cm == 2) NVFP4_LAUNCH(128, 5, 2);
-  NVFP4_LAUNCH(128, 5, 1);
-#undef NVFP4_LAUNCH
+  if (bn == 256)
+    return launch<Cfg<256, 3>>(a_codes, a_scales, g_a, w_codes, w_scales, g_w, M, N, K, out_bf16, ldo, s, idesc_fmt);
+  return launch<Cfg<128, 5>>(a_codes, a_scales, g_a, w_codes, w_scales, g_w, M, N, K, out_bf16, ldo, s, idesc_fmt);
 }
 
 }  // namespace

@@ -160,3 +160,9 @@ def test_kv_and_attention_validation():
     assert L.decode_attention_nvfp4_quantize(ctypes.byref(cache()), p, 4, f, p, p, p, p, ws - 16, s) == 2   # workspace
     assert L.decode_attention_nvfp4_quantize(ctypes.byref(cache()), p, 4, f, p, odd, p, p, ws, s) == 3      # codes align
     assert L.decode_attention_nvfp4_quantize(ctypes.byref(cache(kv_format=5)), p, 4, f, p, p, p, p, ws, s) == 1
+    # static-scratch attention: a problem whose partials exceed the fixed
+    # scratch is refused on the host, before any CUDA call
+    big = cache(batch=64, num_kv_heads=1, capacity=131072)
+    assert N.decode_attention_nvfp4_workspace_size(64, 8, 131072) > N.ATTN_STATIC_SCRATCH_BYTES
+    assert L.decode_attention_nvfp4_static_scratch(ctypes.byref(big), p, 8, f, p, s) == 2
+    assert L.decode_attention_nvfp4_static_scratch(ctypes.byref(cache()), p, 4, f, None, s) == 1
