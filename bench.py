@@ -1,11 +1,13 @@
 """Benchmark of the NVFP4 W4A4KV4 hot path on GB300.
 
 One step = one pass of the path over one batch of synthetic inputs of the
-Qwen-1.5B-shaped prefill layer (M = 2048 tokens): for each linear (qkv, o,
-gate_up, down) the FP32 tensor scale of its bf16 activation, NVFP4
-quantization of the activation, and the block-scaled FP4 GEMM to bf16.
-Weights are quantized once, before timing.  The headline value is the GEMM
-FLOPs of the step divided by its device time (TFLOP/s).
+Qwen-32B-shaped prefill layer (M = 8192 tokens, the largest single-GPU
+workload): for each linear (qkv, o, gate_up, down) the FP32 tensor scale of
+its bf16 activation and NVFP4 quantization of the activation (one launch),
+then the block-scaled FP4 GEMM to bf16.  Weights are quantized once, before
+timing.  The headline value is the GEMM FLOPs of the step divided by its
+device time (TFLOP/s); the roofline entry is the step's dominant kernel, the
+gate_up GEMM (8192 x 55296 x 5120), against the dense FP4 tensor peak.
 
 The decode-attention half of the metric is measured in the same run on the
 Qwen-14B-shaped decode workload (batch 64, 40/8 heads, 16384-token NVFP4
@@ -34,11 +36,11 @@ import time
 ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
-GEMM_WL = "qwen1.5b_prefill_linears_m2048"
+GEMM_WL = "qwen32b_prefill_linears_m8192"
 ATTN_WL = "qwen14b_decode_attention_b64_t16384"
 # Reported beside the headline (same step form, graph-replayed, L2 flushed): the single linear, the
-# decode-batch linears with their K/V append, and the 32B prefill layer chain.
-OTHER_LINEAR_WLS = ("w4a4_linear_m16_k1536_n1536", "qwen14b_decode_linears_m256", "qwen32b_prefill_linears_m8192")
+# 1.5B prefill linears, and the decode-batch linears with their K/V append.
+OTHER_LINEAR_WLS = ("w4a4_linear_m16_k1536_n1536", "qwen1.5b_prefill_linears_m2048", "qwen14b_decode_linears_m256")
 METRIC = "NVFP4 GEMM TFLOP/s & FP4-KV decode-attn HBM GB/s vs GB300 roofline"
 FP4_OVER_BF16 = 13.5 / 2.25  # nominal dense FP4 / BF16 tensor ratio of GB300
 CSRC = os.path.join(ROOT, "paper_2606_15682_gb300", "csrc")
@@ -46,9 +48,9 @@ CSRC = os.path.join(ROOT, "paper_2606_15682_gb300", "csrc")
 # same kernel and shape (commands in profiles/).  Each entry holds only while the kernel sources
 # hash to the value they had at capture time; otherwise the line reports traffic = null.
 NCU_TRAFFIC = {
-    "gemm": {"bytes": 17296384 + 11984640, "sources": ("gemm.cu", "common.cuh"), "sha": "6a81315cc83b08bd",
-             "shape": (2048, 17920, 1536),
-             "profile": "profiles/gemm_qwen1.5b_prefill_gate_up_m2048_n17920_k1536.md"},
+    "gemm": {"bytes": None, "sources": ("gemm.cu", "common.cuh"), "sha": None,
+             "shape": (8192, 55296, 5120),
+             "profile": "profiles/gemm_qwen32b_prefill_gate_up_m8192_n55296_k5120.md"},
     "attention": {"bytes": 1208783616 + 22233856, "sources": ("attention.cu", "common.cuh"),
                   "sha": "b4d25eaf23259ae3", "shape": (64, 16384),
                   "profile": "profiles/attention_qwen14b_decode_b64_t16384.md (attn_partial_kernel)"},
@@ -61,6 +63,8 @@ def ncu_traffic(kind, shape):
     for f in e["sources"]:
         with open(os.path.join(CSRC, f), "rb") as fh:
             h.update(fh.read())
+    if e["bytes"] is None:
+        return None
     return e["bytes"] if h.hexdigest()[:16] == e["sha"] and tuple(shape) == e["shape"] else None
 
 
@@ -402,7 +406,7 @@ def run_ours(args, rank, world):
                 L["ev"][2].record()
 
     mx = {}
-    for wl in (GEMM_WL, "qwen32b_prefill_linears_m8192"):
+    for wl in ("qwen1.5b_prefill_linears_m2048", GEMM_WL):
         Mw, lw, fw = build_mx_layers(wl)
         g = graph_of(lambda lw=lw, Mw=Mw: mx_step(lw, Mw))
         ms_w = statistics.mean(timed_loop(g.replay, other_steps, args.warmup))
@@ -549,6 +553,8 @@ def run_ours(args, rank, world):
                          "kernel": "attn_partial_kernel + attn_combine_kernel (one decode_attention_nvfp4 call)"},
             "gpu_launches": attn_launches * args.steps,
         },
+        "attention_gbs": world * attn_gbs,
+        "attention_frac": attn_gbs / peaks["hbm_gbs"],
         "other_workloads": other,
         "mxfp4_w4a4": mx,
         "clocks": sampler.summary(),
@@ -560,83 +566,100 @@ def run_ours(args, rank, world):
 
 # ------------------------------------------------------- oracle arm ---
 
-def oracle_sample(rows=64, cols=None):
-    """One bounded oracle step: the workload's 4 linears on `rows` activation rows
-    (tensor scale of the whole activation + quantize the rows, dequantized fp64
-    GEMM) against the first `cols` output columns of each weight (all when
-    None), the weights pre-quantized with their whole-tensor scales."""
-    import numpy as np
+class OracleSample:
+    """Bounded oracle steps on the bench workload.
 
-    from oracle import nvfp4_oracle as O
-    from paper_2606_15682_gb300 import synth
-    w = synth.WORKLOADS[GEMM_WL]
-    prep = []
-    for name, (Nn, K) in w["linears"].items():
-        a, W = synth.linear_inputs(GEMM_WL, name)
-        Wf = W.float().numpy()
-        gw = O.tensor_scale(Wf)
-        n = Nn if cols is None else min(cols, Nn)
-        wc, ws = O.quantize(Wf[:n], gw)
-        prep.append((a.float().numpy(), wc, ws, gw, n, K))
+    One step: for each of the workload's 4 linears, the tensor scale of the
+    whole activation, quantization of its first `rows` rows, and the fp64
+    dequantized GEMM against the first `cols` output columns of the weight
+    (all when fewer).  The weights' first `cols_max` rows are quantized once,
+    with their whole-tensor scales, when the sample is built."""
 
-    def step():
+    def __init__(self, cols_max):
+        from oracle import nvfp4_oracle as O
+        from paper_2606_15682_gb300 import synth
+        self.O = O
+        self.prep = []
+        for name, (Nn, K) in synth.WORKLOADS[GEMM_WL]["linears"].items():
+            a, W = synth.linear_inputs(GEMM_WL, name)
+            Wf = W.float().numpy()
+            del W
+            gw = O.tensor_scale(Wf)
+            n = min(cols_max, Nn)
+            wc, ws = O.quantize(Wf[:n], gw)
+            del Wf
+            self.prep.append((a.float().numpy(), wc, ws, gw, n, K))
+
+    def step(self, rows=64, cols=None):
+        O = self.O
         fl = 0
-        for a, wc, ws, gw, n, K in prep:
+        for a, wc, ws, gw, n, K in self.prep:
+            n = n if cols is None else min(cols, n)
             ga = O.tensor_scale(a)
             ac, as_ = O.quantize(a[:rows], ga)
-            O.linear(ac, as_, ga, wc, ws, gw)
+            O.linear(ac, as_, ga, wc[:n], ws[:n], gw)
             fl += 2 * rows * n * K
         return fl
-    return step
+
+    def sample_text(self, rows, cols):
+        return (f"{rows} activation rows x the first {cols} output columns (all when fewer) of each of the 4 "
+                f"linears of {GEMM_WL} per step (tensor scale of the whole activation + quantize the rows + "
+                f"fp64 dequantized GEMM)")
+
+
+def calibrated_cols(sample, budget_s, cols_max):
+    """Output columns per linear that make one 64-row step take about budget_s."""
+    t0 = time.perf_counter()
+    sample.step(rows=64, cols=64)
+    t = time.perf_counter() - t0
+    return int(max(16, min(cols_max, 64 * budget_s / max(t, 1e-6))))
+
+
+CPU_COLS_MAX = 2048
 
 
 def cpu_baseline(seconds=15.0):
-    step = oracle_sample()
+    """The oracle timed on the host cores for about `seconds` (rank 0, N = 1)."""
+    sample = OracleSample(CPU_COLS_MAX)
+    cols = calibrated_cols(sample, 2.0, CPU_COLS_MAX)
     t0 = time.perf_counter()
     fl = 0
     n = 0
     while True:
-        fl += step()
+        fl += sample.step(rows=64, cols=cols)
         n += 1
         if time.perf_counter() - t0 > seconds:
             break
     dt = time.perf_counter() - t0
     return {"value": fl / dt / 1e12, "unit": "TFLOP/s", "cores": os.cpu_count(), "kind": "oracle",
-            "sample": f"{n} oracle steps of 64 activation rows x all 4 linears of {GEMM_WL} "
-                      f"(quantize + fp64 dequantized GEMM), {dt:.1f} s"}
+            "sample": f"{n} steps of {sample.sample_text(64, cols)}, {dt:.1f} s"}
 
 
 def run_reference(args):
-    """The oracle as it stands, on the host cores.  Each step is a bounded sample
-    of the workload: 64 activation rows against the first `cols` output columns
-    of each of the 4 linears.  `cols` is chosen from one calibration step so
-    that the whole run (warm-up and timed steps) takes about 90 s of host
-    time, whatever --steps and --warmup ask for."""
+    """The oracle as it stands, on the host cores.  Each step is a bounded
+    sample of the workload: 64 activation rows against the first `cols`
+    output columns of each of the 4 linears.  `cols` is chosen from one
+    calibration step so that warm-up and timed steps together take about
+    90 s of host time, whatever --steps and --warmup ask for."""
     n_steps = args.steps + max(args.warmup, 1)
-    probe = oracle_sample(rows=64, cols=64)
-    t0 = time.perf_counter()
-    probe()
-    t_probe = time.perf_counter() - t0
-    cols = int(max(16, min(1 << 20, 64 * (90.0 / n_steps) / max(t_probe, 1e-6))))
-    step = oracle_sample(rows=64, cols=cols)
+    sample = OracleSample(CPU_COLS_MAX)
+    cols = calibrated_cols(sample, 90.0 / n_steps, CPU_COLS_MAX)
     for _ in range(max(args.warmup, 1)):
-        step()
+        sample.step(rows=64, cols=cols)
     times = []
     fl = 0
     for _ in range(args.steps):
         t0 = time.perf_counter()
-        fl = step()
+        fl = sample.step(rows=64, cols=cols)
         times.append(time.perf_counter() - t0)
     ms = statistics.mean(times) * 1e3
     value = fl / (ms * 1e-3) / 1e12
-    sample = (f"64 activation rows x the first {cols} output columns (all when fewer) of each of the 4 linears "
-              f"of {GEMM_WL} per step (tensor scale + quantize + fp64 dequantized GEMM)")
     return {"impl": "reference", "metric": METRIC, "value": value, "unit": "TFLOP/s", "n_gpus": 1,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64 (dequantized)", "data": "synthetic",
             "config": {"workload": GEMM_WL, "sample_rows": 64, "sample_cols": cols},
             "cpu_baseline": {"value": value, "unit": "TFLOP/s", "cores": os.cpu_count(), "kind": "oracle",
-                             "sample": sample},
+                             "sample": sample.sample_text(64, cols)},
             "e2e": {"value": value, "unit": "TFLOP/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
 
 
@@ -652,6 +675,10 @@ def main():
     args.warmup = max(args.warmup, 3)
     rank = int(os.environ.get("RANK", 0))
     world = int(os.environ.get("WORLD_SIZE", 1))
+    if args.gpus != world:
+        # N GPUs means N ranks, one per GPU, started by torch.distributed.run.
+        sys.exit(f"bench.py: --gpus {args.gpus} but WORLD_SIZE={world}; launch N > 1 with "
+                 f"python -m torch.distributed.run --nproc-per-node {args.gpus} bench.py --gpus {args.gpus}")
     if args.impl == "reference":
         if rank == 0:
             print(json.dumps(run_reference(args)))

@@ -131,7 +131,10 @@ __device__ __forceinline__ void st_shared_v4(uint32_t addr, uint32_t a, uint32_t
 // Work-unit order: units walk the N tiles within groups of kGroupM row
 // super-tiles, so the CTAs running at the same time share a few A and W
 // tiles that stay in L2 instead of streaming all of A for every column.
-constexpr int kGroupM = 8;
+#ifndef NVFP4_GEMM_GROUP_M
+#define NVFP4_GEMM_GROUP_M 8
+#endif
+constexpr int kGroupM = NVFP4_GEMM_GROUP_M;
 __device__ __forceinline__ void unit_coords(int u, int msup, int tiles_n, int* ms, int* nb) {
   const int per_group = kGroupM * tiles_n;
   const int group = u / per_group, r = u - group * per_group;
