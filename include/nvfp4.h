@@ -443,10 +443,19 @@ nvfp4_status nvfp4_get_device_status(int32_t* status_host, void* stream);
  *     consumers' bounded wait on it runs out after ~2 s: the call reports
  *     NVFP4_ERR_TIMEOUT through nvfp4_get_device_status, its output is
  *     undefined, and the device stays usable.
+ *   NVFP4_FAULT_GEMM_SKIP_STAGE: in the next launch of a CTA-pair GEMM kernel
+ *     (the 256 x 256 tiles that nvfp4_linear / mxfp4_linear use when N % 256
+ *     == 0 and the tiles fill the GPU, and the fused SwiGLU calls), both CTAs
+ *     of pair 0 leave their first ring stage neither armed nor loaded; the MMA
+ *     issuer's and the scale copiers' bounded waits run out after ~2 s, every
+ *     role of the pair stops, the MMAs issued so far drain and TMEM is freed.
+ *     The call reports NVFP4_ERR_TIMEOUT, its output is undefined, and the
+ *     device stays usable.
  *   NVFP4_FAULT_NONE disarms.  Other values -> INVALID_ARG.
  */
 #define NVFP4_FAULT_NONE 0
 #define NVFP4_FAULT_ATTN_SKIP_STAGE 1
+#define NVFP4_FAULT_GEMM_SKIP_STAGE 2
 nvfp4_status nvfp4_debug_inject_fault(int what);
 
 /* Static, human-readable name of a status. */

@@ -95,7 +95,8 @@ NVFP4_API uint64_t nvfp4_launch_count(void) { return g_launches.load(std::memory
 
 NVFP4_API nvfp4_status nvfp4_debug_inject_fault(int what) {
   NVFP4_TRACE("nvfp4_debug_inject_fault");
-  if (what != NVFP4_FAULT_NONE && what != NVFP4_FAULT_ATTN_SKIP_STAGE) return NVFP4_ERR_INVALID_ARG;
+  if (what != NVFP4_FAULT_NONE && what != NVFP4_FAULT_ATTN_SKIP_STAGE && what != NVFP4_FAULT_GEMM_SKIP_STAGE)
+    return NVFP4_ERR_INVALID_ARG;
   g_fault.store(what);
   return NVFP4_OK;
 }

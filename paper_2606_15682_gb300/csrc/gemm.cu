@@ -165,6 +165,9 @@ struct GemmArgs {
   // Quantization of the fused output: 0 NVFP4 with the static scale g_out,
   // 1 MXFP4, 2 MXFP4 after the H_32 block rotation.
   uint32_t q_mode;
+  // Test-only (nvfp4_debug_inject_fault): both CTAs of pair 0 leave their
+  // first stage unissued (CTA-pair kernel).
+  int fault_skip_stage;
 };
 
 template <class C>
@@ -591,6 +594,7 @@ __global__ void __launch_bounds__(C::kThreads, 1)
     bool issued[kStages];
     for (int s = 0; s < kStages; ++s) issued[s] = false;
     int prev_nb = -1;
+    int g = 0;  // k-blocks this pair has passed so far
     for (int u = u_first; u < u_end && !abort_flag; u += u_step) {
       int ms, nb;
       coords(u, &ms, &nb);
@@ -605,8 +609,15 @@ __global__ void __launch_bounds__(C::kThreads, 1)
       // k-block) group of four 512-byte atoms is 8 rows of that view.
       const int sfa_row = mb * kgroups * 2;
       const int sfb_row = nb * 2 * kgroups * 2;
-      for (int kb = 0; kb < kblocks; ++kb) {
+      for (int kb = 0; kb < kblocks; ++kb, ++g) {
         if (!mbar_wait_bounded(&empty[stage], phase ^ 1u, &abort_flag)) { fail(); break; }
+        if (args.fault_skip_stage && pair_id == 0 && g == 0) {
+          // Test-only injected fault: both CTAs of pair 0 leave their first
+          // stage neither armed nor loaded, so no copy is ever in flight for
+          // it and the consumers' bounded waits on it run out.
+          if (++stage == kStages) { stage = 0; phase ^= 1u; }
+          continue;
+        }
         uint8_t* a_dst = sA + stage * C::kTileBytesA;
         uint8_t* b_dst = sB + (C::kRes ? kb : stage) * C::kTileBytesB;
         uint8_t* sfa_dst = sSFA + stage * C::kSfaBytes;
@@ -1064,6 +1075,7 @@ nvfp4_status launch_pair(const uint8_t* a_codes, const uint8_t* a_scales, const 
   args.tiles_m = static_cast<int>(tiles_m);
   args.tiles_n = static_cast<int>(tiles_n);
   args.status = status_word_dev();
+  args.fault_skip_stage = take_fault(NVFP4_FAULT_GEMM_SKIP_STAGE) ? 1 : 0;
   const int pairs = static_cast<int>(units < pairs_max ? units : pairs_max);
   cudaLaunchConfig_t cfg = {};
   cudaLaunchAttribute attr[2];

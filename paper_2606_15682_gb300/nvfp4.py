@@ -72,7 +72,7 @@ _launch_count = _sig("nvfp4_launch_count", [], ctypes.c_uint64)
 _scales_bytes = _sig("nvfp4_scales_bytes", [_i64, _i64, ctypes.c_int], _sz)
 _mx_scales_bytes = _sig("mxfp4_scales_bytes", [_i64, _i64, ctypes.c_int], _sz)
 _inject_fault = _sig("nvfp4_debug_inject_fault", [ctypes.c_int])
-FAULT_NONE, FAULT_ATTN_SKIP_STAGE = 0, 1
+FAULT_NONE, FAULT_ATTN_SKIP_STAGE, FAULT_GEMM_SKIP_STAGE = 0, 1, 2
 
 
 def nvfp4_debug_inject_fault(what):

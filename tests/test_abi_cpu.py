@@ -114,6 +114,7 @@ def test_mxfp4_validation_before_launch():
 def test_fault_injection_knob_validation():
     N = lib()
     assert N._lib.nvfp4_debug_inject_fault(5) == 1
+    assert N._lib.nvfp4_debug_inject_fault(N.FAULT_GEMM_SKIP_STAGE) == 0
     assert N._lib.nvfp4_debug_inject_fault(N.FAULT_ATTN_SKIP_STAGE) == 0
     assert N._lib.nvfp4_debug_inject_fault(N.FAULT_NONE) == 0
 

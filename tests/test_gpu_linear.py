@@ -55,7 +55,10 @@ def run_linear(N, a_codes, a_scales_rm, g_a, w_codes, w_scales_rm, g_w, M, Nn, K
                                     # more 256 x 256 tiles than pairs: a second round of tiles (K = 1024), and
                                     # the W-resident form (K = 1280, 1536): runs of two units per pair, an M
                                     # tail, runs that cross a W tile
-                                    (512, 10240, 1024), (300, 15360, 1536), (640, 7680, 1280)])
+                                    (512, 10240, 1024), (300, 15360, 1536), (640, 7680, 1280),
+                                    # N % 256 != 0 with K >= 2048 (single CTAs), and a pair shape with K = 4096
+                                    # and a one-row M tail
+                                    (640, 10112, 2048), (512, 10576, 2048), (257, 15360, 4096)])
 def test_random_codes(N, M, Nn, K):
     gen = torch.Generator().manual_seed(M * 1000 + Nn * 10 + K)
     a_c, a_s = random_operand(M, K, gen)
@@ -143,6 +146,41 @@ def test_workload_linears(N, workload):
         got = f32(out[torch.as_tensor(rows, device="cuda")][:, torch.as_tensor(cols, device="cuda")])
         report.append((name,) + assert_close(got, ref, what=f"{workload}/{name}"))
     print(workload, report)
+
+
+def test_injected_missing_stage_times_out_and_next_call_is_exact(N):
+    """Failure detection of the GEMM without a GPU fault: the test-only fault
+    knob makes both CTAs of the first CTA pair leave their first ring stage
+    unissued.  The MMA issuer's and scale copiers' bounded waits run out after
+    ~2 s, the pair drains its MMAs, frees TMEM and exits, the call reports
+    NVFP4_ERR_TIMEOUT, and the next call is exact again."""
+    import time
+    M, Nn, K = 640, 10240, 2048  # a CTA-pair shape with more tiles than resident pairs
+    gen = torch.Generator().manual_seed(31)
+    a_c, a_s = random_operand(M, K, gen)
+    w_c, w_s = random_operand(Nn, K, gen)
+    dev = "cuda"
+    args = (torch.from_numpy(a_c).to(dev), torch.from_numpy(O.scales_to_mma(a_s)).to(dev),
+            torch.ones(1, device=dev), torch.from_numpy(w_c).to(dev),
+            torch.from_numpy(O.scales_to_mma(w_s)).to(dev), torch.ones(1, device=dev))
+    out = torch.full((M, Nn), float("nan"), dtype=torch.bfloat16, device=dev)
+    torch.cuda.synchronize()
+    assert N.nvfp4_get_device_status() == 0
+    N.nvfp4_debug_inject_fault(N.FAULT_GEMM_SKIP_STAGE)
+    try:
+        t0 = time.time()
+        N.nvfp4_linear(*args, out, M, Nn, K)
+        torch.cuda.synchronize()
+        waited = time.time() - t0
+    finally:
+        N.nvfp4_debug_inject_fault(N.FAULT_NONE)
+    assert N.nvfp4_get_device_status() == 6
+    assert 1.0 < waited < 20.0, f"bounded wait expected (~2-4 s), took {waited:.1f} s"
+    out.fill_(float("nan"))
+    N.nvfp4_linear(*args, out, M, Nn, K)
+    torch.cuda.synchronize()
+    assert N.nvfp4_get_device_status() == 0
+    assert_close(f32(out), O.linear(a_c, a_s, 1.0, w_c, w_s, 1.0), what="after the injected timeout")
 
 
 # ------------------------------------ gate_up with SwiGLU + quantize fused ---
