@@ -9,6 +9,12 @@ bounds-checked variant into ``_build_debug``: every computed store index of the
 non-TMA kernels is checked against the extent the kernel derives from its
 shape arguments, and a violation sets NVFP4_ERR_BOUNDS instead of writing.
 The binding loads that variant when ``NVFP4_DEBUG=1``.
+
+``build(timeline=True)`` (or ``NVFP4_TIMELINE=1``) builds a profiling variant
+into ``_build_timeline``: the one-launch dynamic quantizer records per-block
+globaltimer stamps (entry, loads done, barrier arrival, release, stores
+issued), read back with ``nvfp4_timeline_quantize_dynamic`` (that build only).
+The binding loads it when ``NVFP4_TIMELINE=1``.
 """
 from __future__ import annotations
 
@@ -25,6 +31,7 @@ CSRC = os.path.join(PKG, "csrc")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(BUILD, "libnvfp4.so")
 BUILD_DEBUG = os.path.join(PKG, "_build_debug")
+BUILD_TIMELINE = os.path.join(PKG, "_build_timeline")
 SOURCES = ["api.cu", "quantize.cu", "kv_append.cu", "attention.cu", "gemm.cu"]
 HEADERS = ["common.cuh", "nvfp4_quant.cuh", os.path.join("..", "..", "include", "nvfp4.h")]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
@@ -63,18 +70,26 @@ def _compile(nvcc, name, verbose, build_dir, flags):
     return obj, (r.stderr if verbose else "")
 
 
-def lib_path(debug: bool | None = None) -> str:
+def _variant(debug, timeline):
     if debug is None:
         debug = os.environ.get("NVFP4_DEBUG") == "1"
-    return os.path.join(BUILD_DEBUG if debug else BUILD, "libnvfp4.so")
+    if timeline is None:
+        timeline = os.environ.get("NVFP4_TIMELINE") == "1"
+    if debug and timeline:
+        raise ValueError("the bounds-checked and the timeline builds are separate variants")
+    return debug, timeline
 
 
-def build(verbose: bool = False, debug: bool | None = None) -> str:
-    if debug is None:
-        debug = os.environ.get("NVFP4_DEBUG") == "1"
-    build_dir = BUILD_DEBUG if debug else BUILD
-    flags = FLAGS + (["-DNVFP4_DEBUG"] if debug else [])
-    LIB = lib_path(debug)
+def lib_path(debug: bool | None = None, timeline: bool | None = None) -> str:
+    debug, timeline = _variant(debug, timeline)
+    return os.path.join(BUILD_DEBUG if debug else (BUILD_TIMELINE if timeline else BUILD), "libnvfp4.so")
+
+
+def build(verbose: bool = False, debug: bool | None = None, timeline: bool | None = None) -> str:
+    debug, timeline = _variant(debug, timeline)
+    build_dir = BUILD_DEBUG if debug else (BUILD_TIMELINE if timeline else BUILD)
+    flags = FLAGS + (["-DNVFP4_DEBUG"] if debug else []) + (["-DNVFP4_TIMELINE"] if timeline else [])
+    LIB = lib_path(debug, timeline)
     os.makedirs(build_dir, exist_ok=True)
     nvcc = _nvcc()
     with cf.ThreadPoolExecutor(max_workers=len(SOURCES)) as ex:

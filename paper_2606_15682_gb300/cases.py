@@ -8,11 +8,15 @@
     python -m paper_2606_15682_gb300.cases mx_gemm --workload qwen32b_prefill_linears_m8192 --linear down
     python -m paper_2606_15682_gb300.cases mx_quantize --workload qwen32b_prefill_linears_m8192 --linear down --rotate
     python -m paper_2606_15682_gb300.cases mx_gemm_swiglu --workload qwen32b_prefill_linears_m8192 --rotate
+    NVFP4_TIMELINE=1 python -m paper_2606_15682_gb300.cases quantize_timeline --workload qwen1.5b_prefill_linears_m2048 --linear qkv
 
 Inputs are seeded synthetic tensors (paper_2606_15682_gb300.synth); for the
 attention case the cache is filled with seeded random codes and scales
 directly, which is enough to time the kernel.  Prints the mean CUDA-event time
-of the measured call.
+of the measured call.  quantize_timeline (timeline build, NVFP4_TIMELINE=1)
+prints, for one launch of the one-launch dynamic quantizer after an L2 flush,
+when its blocks started, finished their loads, arrived at the grid barrier,
+were released and issued their stores.
 """
 from __future__ import annotations
 
@@ -49,10 +53,48 @@ def _time(fn, iters):
     return ev[0].elapsed_time(ev[1]) / iters
 
 
+def _quantize_timeline(a, dev):
+    import ctypes
+    if not hasattr(N._lib, "nvfp4_timeline_quantize_dynamic"):
+        raise SystemExit("quantize_timeline needs the timeline build: run with NVFP4_TIMELINE=1")
+    read = N._lib.nvfp4_timeline_quantize_dynamic
+    read.argtypes = [ctypes.c_void_p]
+    read.restype = ctypes.c_int
+    x, _ = synth.linear_inputs(a.workload, a.linear, device=dev)
+    M, K = x.shape
+    state = torch.zeros(N.DYNAMIC_STATE_BYTES, dtype=torch.uint8, device=dev)
+    g = torch.empty(1, dtype=torch.float32, device=dev)
+    c = torch.empty(M, K // 2, dtype=torch.uint8, device=dev)
+    s = torch.empty(N.nvfp4_scales_bytes(M, K, N.SCALES_MMA), dtype=torch.uint8, device=dev)
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    torch.cuda.synchronize()  # the zeroed barrier state is ordered before the first call
+    for _ in range(3):
+        N.nvfp4_quantize_dynamic(x, state, g, c, s, N.SCALES_MMA)
+    host = (ctypes.c_ulonglong * (2048 * 5))()
+    read(host)  # clears the stamps of the warm-up calls
+    flush.zero_()
+    torch.cuda._sleep(1_000_000)
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
+    ev[0].record()
+    N.nvfp4_quantize_dynamic(x, state, g, c, s, N.SCALES_MMA)
+    ev[1].record()
+    if read(host) != 0:
+        raise SystemExit("reading the timeline failed")
+    assert N.nvfp4_get_device_status() == 0
+    rows = [host[5 * b:5 * b + 5] for b in range(2048) if host[5 * b] != 0]
+    t0 = min(r[0] for r in rows)
+    print(f"{a.workload}/{a.linear}: x {M}x{K} bf16 ({M * K * 2 / 1e6:.1f} MB), {len(rows)} blocks, "
+          f"event {ev[0].elapsed_time(ev[1]) * 1e3:.2f} us, in-kernel span "
+          f"{(max(r[4] for r in rows) - t0) / 1e3:.2f} us")
+    for e, name in enumerate(["entry", "loads done", "arrived", "released", "stores issued"]):
+        v = sorted(r[e] - t0 for r in rows)
+        print(f"  {name:13s} min {v[0] / 1e3:6.2f}  median {v[len(v) // 2] / 1e3:6.2f}  max {v[-1] / 1e3:6.2f} us")
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("kernel", choices=["gemm", "gemm_swiglu", "quantize", "quantize_dynamic", "tensor_scale",
-                                       "attention", "mx_gemm", "mx_quantize", "mx_gemm_swiglu"])
+                                       "attention", "mx_gemm", "mx_quantize", "mx_gemm_swiglu", "quantize_timeline"])
     ap.add_argument("--rotate", action="store_true", help="MXFP4: 32-element block rotation before quantizing")
     ap.add_argument("--workload", default="qwen1.5b_prefill_linears_m2048")
     ap.add_argument("--linear", default="gate_up")
@@ -63,6 +105,9 @@ def main():
     a = ap.parse_args()
     dev = torch.device("cuda", 0)
     torch.cuda.set_device(dev)
+    if a.kernel == "quantize_timeline":
+        _quantize_timeline(a, dev)
+        return
     if a.kernel == "gemm_swiglu":
         # gate_up of the workload with SwiGLU + NVFP4 quantization of the down
         # projection's input in the epilogue, against the same GEMM with bf16

@@ -17,6 +17,23 @@ namespace {
 
 constexpr int kThreads = 256;
 constexpr int kUnroll = 4;
+// Timeline build (-DNVFP4_TIMELINE): quantize_dynamic_kernel records, per
+// block, the globaltimer at entry, when its phase-1 loads are done, when it
+// has arrived at the grid barrier, when the barrier released it and when its
+// stores are issued.  The release build compiles the stamps away.
+#ifdef NVFP4_TIMELINE
+constexpr int kTimelineBlocks = 2048;
+__device__ unsigned long long g_quantize_timeline[kTimelineBlocks][5];
+__device__ __forceinline__ void timeline_stamp(int event) {
+  if (threadIdx.x == 0 && blockIdx.x < kTimelineBlocks) g_quantize_timeline[blockIdx.x][event] = globaltimer_ns();
+}
+#else
+__device__ __forceinline__ void timeline_stamp(int) {}
+#endif
+
+#ifndef NVFP4_BARRIER_POLL_NS
+#define NVFP4_BARRIER_POLL_NS 100  // sleep between polls of the one-launch quantizer's grid barrier
+#endif
 
 // Chunk c (8 elements) of a [rows, cols] tensor with leading dimension ld.
 struct ChunkMap {
@@ -211,6 +228,15 @@ __device__ __forceinline__ unsigned long long ld_acquire_u64(const unsigned long
   return v;
 }
 
+// The waiting blocks need only the value of the word they poll (the release
+// store carries the new epoch and the amax together), so they poll with
+// relaxed loads: no acquire per poll.
+__device__ __forceinline__ unsigned long long ld_relaxed_u64(const unsigned long long* p) {
+  unsigned long long v;
+  asm volatile("ld.relaxed.gpu.global.u64 %0, [%1];" : "=l"(v) : "l"(p) : "memory");
+  return v;
+}
+
 __device__ __forceinline__ unsigned long long atom_add_acq_rel_u64(unsigned long long* p, unsigned long long v) {
   unsigned long long old;
   asm volatile("atom.acq_rel.gpu.global.add.u64 %0, [%1], %2;" : "=l"(old) : "l"(p), "l"(v) : "memory");
@@ -245,6 +271,7 @@ __global__ void __launch_bounds__(kThreads) quantize_dynamic_kernel(
   // iterations, [iteration * kUnroll + slot][half][thread] as 16-byte words.
   extern __shared__ uint4 stash[];
   griddep_wait_and_release();
+  timeline_stamp(0);
   const uint32_t lane = threadIdx.x & 31;
   const uint32_t stride = gridDim.x * blockDim.x;
   unsigned long long epoch = 0;
@@ -273,6 +300,10 @@ __global__ void __launch_bounds__(kThreads) quantize_dynamic_kernel(
   m = __reduce_max_sync(0xffffffffu, m);
   __shared__ uint32_t warp_max[kThreads / 32];
   __shared__ uint32_t s_amax;
+#ifdef NVFP4_TIMELINE
+  __syncthreads();
+  timeline_stamp(1);
+#endif
   __shared__ int s_ok;
   if ((threadIdx.x & 31) == 0) warp_max[threadIdx.x >> 5] = m;
   __syncthreads();
@@ -282,6 +313,7 @@ __global__ void __launch_bounds__(kThreads) quantize_dynamic_kernel(
     if (threadIdx.x == 0) {
       red_max_u64(&state[1], (epoch << 32) | m);
       const unsigned long long old = atom_add_acq_rel_u64(&state[0], 1ull);
+      timeline_stamp(2);
       int ok = (old >> 32) == epoch;
       uint32_t amax_bits = 0;
       if (ok && static_cast<uint32_t>(old & 0xFFFFu) == gridDim.x - 1) {
@@ -290,10 +322,15 @@ __global__ void __launch_bounds__(kThreads) quantize_dynamic_kernel(
         amax_bits = static_cast<uint32_t>(a) & 0xFFFFu;
         if (ok) st_release_u64(&state[0], ((epoch + 1) << 32) | (static_cast<unsigned long long>(amax_bits) << 16));
       } else if (ok) {
+        // Every waiting block polls the one word the last arrival will
+        // release; a short sleep between polls keeps the polls from queueing
+        // ahead of the arrivals' atomics and the release store at L2.
         const uint64_t t0 = globaltimer_ns();
         unsigned long long v;
-        for (uint32_t it = 0; ((v = ld_acquire_u64(&state[0])) >> 32) == epoch; ++it)
+        for (uint32_t it = 0; ((v = ld_relaxed_u64(&state[0])) >> 32) == epoch; ++it) {
+          __nanosleep(NVFP4_BARRIER_POLL_NS);
           if ((it & 63u) == 63u && globaltimer_ns() - t0 > kWaitLimitNs) { ok = 0; break; }
+        }
         if (ok && (v >> 32) != epoch + 1) ok = 0;
         amax_bits = static_cast<uint32_t>(v >> 16) & 0xFFFFu;
       }
@@ -303,6 +340,7 @@ __global__ void __launch_bounds__(kThreads) quantize_dynamic_kernel(
     }
   }
   __syncthreads();
+  timeline_stamp(3);
   if (!s_ok) return;
   const float amax = __uint_as_float(s_amax << 16);
   const float g = amax > 0.0f ? __fdiv_rn(amax, 2688.0f) : 1.0f;
@@ -330,6 +368,10 @@ __global__ void __launch_bounds__(kThreads) quantize_dynamic_kernel(
     quantize_loaded<kMMA>(t, total_blocks, kblocks_div.d, bidx0, stride, lane, g, six_g, true, codes, scales, status);
   }
   if (kMMA) zero_scale_padding(rows, kblocks_div.d, scales, status);
+#ifdef NVFP4_TIMELINE
+  __syncthreads();
+  timeline_stamp(4);
+#endif
 }
 
 // Blocks of quantize_dynamic_kernel that fit on the device at once (a
@@ -574,12 +616,18 @@ NVFP4_API nvfp4_status nvfp4_quantize_dynamic(const void* x_bf16, int64_t rows, 
   }
   if (grid > cap) grid = cap;
   if (grid > 0xFFFF) grid = 0xFFFF;  // the barrier counts arrivals in 16 bits
-  // Cooperative: every block is resident at once, so the grid barrier can
-  // complete.  (Without programmatic serialization: measured no faster.)
+  // The grid never exceeds the blocks the device holds at once, so every
+  // block becomes resident and the grid barrier completes: blocks that find
+  // their SM still occupied by the previous kernel in the stream (programmatic
+  // dependent launch) start when it retires, and that kernel does not wait on
+  // this one.  A cooperative launch gives the same guarantee up front but
+  // measured 2-4 us slower per four-quantization step (its launch does not
+  // overlap the previous kernel).  Work on other streams that holds SMs for
+  // longer than the barrier's 2 s bound makes the call report TIMEOUT.
   cudaLaunchConfig_t cfg = {};
   cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeCooperative;
-  attr[0].val.cooperative = 1;
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.gridDim = dim3(grid);
   cfg.blockDim = dim3(kThreads);
   cfg.dynamicSmemBytes = stash_iters * kStashIterBytes;
@@ -653,3 +701,17 @@ NVFP4_API nvfp4_status mxfp4_quantize(const void* x_bf16, int64_t rows, int64_t 
   count_launches(1);
   return launch_status();
 }
+
+#ifdef NVFP4_TIMELINE
+// Timeline build only (not part of the C ABI of include/nvfp4.h): copy the
+// per-block stamps of the last nvfp4_quantize_dynamic launch to host memory
+// ([2048][5] uint64, nanoseconds, zero where a block did not run), then clear
+// them.  Synchronizes the device.
+extern "C" __attribute__((visibility("default"))) int nvfp4_timeline_quantize_dynamic(unsigned long long* host) {
+  if (cudaDeviceSynchronize() != cudaSuccess) return 1;
+  if (cudaMemcpyFromSymbol(host, nvfp4::g_quantize_timeline, sizeof(nvfp4::g_quantize_timeline)) != cudaSuccess)
+    return 1;
+  static unsigned long long zero[nvfp4::kTimelineBlocks * 5];
+  return cudaMemcpyToSymbol(nvfp4::g_quantize_timeline, zero, sizeof(zero)) == cudaSuccess ? 0 : 1;
+}
+#endif

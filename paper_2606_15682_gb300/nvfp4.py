@@ -14,8 +14,10 @@ import os
 import torch
 
 _PKG = os.path.dirname(os.path.abspath(__file__))
-# NVFP4_DEBUG=1 selects the bounds-checked build (paper_2606_15682_gb300.build).
-LIB_PATH = os.path.join(_PKG, "_build_debug" if os.environ.get("NVFP4_DEBUG") == "1" else "_build", "libnvfp4.so")
+# NVFP4_DEBUG=1 selects the bounds-checked build, NVFP4_TIMELINE=1 the
+# timeline build (paper_2606_15682_gb300.build).
+LIB_PATH = os.path.join(_PKG, "_build_debug" if os.environ.get("NVFP4_DEBUG") == "1" else
+                        ("_build_timeline" if os.environ.get("NVFP4_TIMELINE") == "1" else "_build"), "libnvfp4.so")
 
 SCALES_ROWMAJOR = 0
 SCALES_MMA = 1

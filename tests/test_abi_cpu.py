@@ -37,6 +37,24 @@ def test_bounds_checked_build_compiles_and_exports_every_call():
     assert b"bounds" in so.nvfp4_status_string(8)
 
 
+def test_timeline_build_compiles_and_exports_every_call():
+    """The NVFP4_TIMELINE variant (per-block stamps in the one-launch
+    quantizer) builds, exports the same C ABI plus its stamp reader, and the
+    release build does not export the reader."""
+    import os
+    import pytest
+    from paper_2606_15682_gb300 import build as B
+    path = B.build(timeline=True)
+    assert os.path.basename(os.path.dirname(path)) == "_build_timeline"
+    so = ctypes.CDLL(path)
+    for name in header_functions():
+        assert hasattr(so, name), name
+    assert hasattr(so, "nvfp4_timeline_quantize_dynamic")
+    assert not hasattr(ctypes.CDLL(B.build(timeline=False, debug=False)), "nvfp4_timeline_quantize_dynamic")
+    with pytest.raises(ValueError):
+        B.build(debug=True, timeline=True)
+
+
 def test_status_strings_and_sizes():
     N = lib()
     assert N.nvfp4_status_string(0) == "ok"
