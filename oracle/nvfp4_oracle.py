@@ -502,16 +502,22 @@ def qfit_transform(q_pre, k_pre, s, m, positions, theta=1.0e6):
 # paired pre-RoPE scale S and the post-RoPE key shift m that minimize the MSE
 # between a reference attention and the attention over the KV4 cache.
 # Readings where the algorithm leaves a choice open:
+#   * the calibration set is B sequences of T tokens at positions 0..T-1;
+#     inputs are [B, T, heads, d];
+#   * Attn is the causal attention of a decoder layer.  It is scored at the
+#     last token of every sequence, which attends to all T tokens of its own
+#     sequence: one decode step over the cached sequence.  (The paper averages
+#     over every position of its calibration samples; the last-token subset
+#     keeps the KV4 side a plain decode over one cache per grid point.)
+#     Softmax scale 1/sqrt(d).
 #   * RoPE is the fp32 table form ``rope_f32`` (tables from ``rope_table``);
 #     the scaled keys K_pre / S_K are rounded to bf16 before RoPE, as a key
-#     projection with S folded into its weights would produce them.
-#   * Attn(Q, K, V) is evaluated for the queries at positions ``q_pos``, each
-#     attending to all T cached tokens, with softmax scale 1/sqrt(d) (decode
-#     form; the calibration sequence is the cache).
+#     projection with S folded into its weights would produce them, and the
+#     scaled, RoPE'd queries are rounded to bf16, the attention's input type.
 #   * Q_KV4 uses a static tensor scale per grid point: g = amax / (qmax * 448)
-#     of the tensor being cached (K~ - m, or V).
-#   * the shift template mu is the token mean of RoPE(K_pre) (unscaled keys),
-#     as written; m(alpha_m) = alpha_m * mu at every alpha_s.
+#     of the tensor being cached (K~ - m over all sequences, or V).
+#   * the shift template mu is the mean over all tokens of RoPE(K_pre), the
+#     unscaled keys, as written; m(alpha_m) = alpha_m * mu at every alpha_s.
 # ---------------------------------------------------------------------------
 
 
@@ -522,55 +528,96 @@ def _bf16_round(x):
     return (b << 16).astype(np.uint32).view(np.float32)
 
 
+def _tokens(x):
+    """[B, T, H, d] -> [B * T, H, d]."""
+    x = np.asarray(x)
+    return x.reshape((-1,) + x.shape[-2:])
+
+
 def qfit_init_scale(k_pre, eps):
-    """S_K^0[h, r] = max(max_t |K[t,h,r]|, max_t |K[t,h,r+d/2]|, eps), shared by the
-    pair (r, r + d/2) so the scaling commutes with RoPE.  k_pre [T, H_kv, d]."""
-    k = np.abs(np.asarray(k_pre, dtype=np.float64))
+    """S_K^0[h, r] = max(max_t |K[t,h,r]|, max_t |K[t,h,r+d/2]|, eps) over every
+    token of every sequence, shared by the pair (r, r + d/2) so the scaling
+    commutes with RoPE.  k_pre [..., H_kv, d] -> [H_kv, d]."""
+    k = np.abs(_tokens(k_pre).astype(np.float64))
     half = k.shape[-1] // 2
     m = np.maximum(k[..., :half].max(axis=0), k[..., half:].max(axis=0))
     s0 = np.maximum(m, eps)
-    return np.concatenate([s0, s0], axis=-1)                       # [H_kv, d]
+    return np.concatenate([s0, s0], axis=-1)
 
 
-def qfit_attention_error(q_pre, k_pre, v, table, q_pos, s_k, s_q, m, element="e2m1"):
-    """MSE between the reference attention (RoPE'd Q and K, exact V) and the
-    attention over the KV4 cache holding Q_KV4(RoPE(K_pre / s_k) - m), Q_KV4(V)
-    for queries RoPE(Q_pre * s_q) (one grid point of Algorithm 1)."""
-    T, hkv, d = k_pre.shape
-    hq = q_pre.shape[1]
+def qfit_shift_template(k_pre, table):
+    """mu = E_t[RoPE(K_pre)_t], the channel-wise mean of the post-RoPE keys over
+    every token of every sequence (token t of a sequence at position t).
+    k_pre [B, T, H_kv, d] -> fp64 [H_kv, d]."""
+    k = np.asarray(k_pre, dtype=np.float32)
+    B, T = k.shape[:2]
     pos = np.arange(T)
-    qmax = 6.0 if element == "e2m1" else E1M2_MAX
-    # reference: unscaled, unshifted, unquantized
-    k0 = rope_f32(k_pre, pos, table).astype(np.float64)
-    q0 = rope_f32(q_pre[q_pos], q_pos, table).astype(np.float64)
-    scale = 1.0 / np.sqrt(d)
+    rot = np.stack([rope_f32(k[b], pos, table) for b in range(B)])
+    return rot.astype(np.float64).reshape((-1,) + k.shape[-2:]).mean(axis=0)
+
+
+def qfit_reference(q_pre, k_pre, v, table):
+    """Y_ref: the unquantized attention of the last token of each sequence,
+    RoPE'd query against the RoPE'd keys and the values of all T tokens, fp64.
+    Returns [B, H_q, d]."""
+    q = np.asarray(q_pre, np.float32)
+    k = np.asarray(k_pre, np.float32)
+    vv = np.asarray(v, np.float64)
+    B, T, hq, d = q.shape
+    hkv = k.shape[2]
     group = hq // hkv
-    y_ref = np.stack([[attention_fp64(q0[i, h], k0[:, h // group], np.asarray(v, np.float64)[:, h // group], scale)
-                       for h in range(hq)] for i in range(len(q_pos))])
-    # transformed and quantized
-    k_in = _bf16_round(np.asarray(k_pre, np.float32) / np.asarray(s_k, np.float32)[None])
-    kt = rope_f32(k_in, pos, table)
-    kt = (kt - np.asarray(m, np.float32)[None]).astype(np.float32)
-    g_k = np.float32(np.abs(kt).max() / (qmax * 448))
-    g_v = np.float32(np.abs(np.asarray(v, np.float32)).max() / (qmax * 448))
-    kc, ks = quantize(kt.reshape(T * hkv, d), g_k, element)
-    vc, vs = quantize(np.asarray(v, np.float32).reshape(T * hkv, d), g_v, element)
-    K = dequantize(kc, ks, g_k, element).reshape(T, hkv, d)
-    V = dequantize(vc, vs, g_v, element).reshape(T, hkv, d)
-    q_in = np.asarray(q_pre, np.float32)[q_pos] * np.repeat(np.asarray(s_q, np.float32), 1, axis=0)[None]
-    qt = _bf16_round(rope_f32(q_in.astype(np.float32), q_pos, table)).astype(np.float64)
-    y = np.stack([[attention_fp64(qt[i, h], K[:, h // group], V[:, h // group], scale) for h in range(hq)]
-                  for i in range(len(q_pos))])
+    pos = np.arange(T)
+    scale = 1.0 / np.sqrt(d)
+    out = np.zeros((B, hq, d))
+    for b in range(B):
+        k0 = rope_f32(k[b], pos, table).astype(np.float64)
+        q0 = rope_f32(q[b, T - 1:T], np.array([T - 1]), table)[0].astype(np.float64)
+        for h in range(hq):
+            out[b, h] = attention_fp64(q0[h], k0[:, h // group], vv[b, :, h // group], scale)
+    return out
+
+
+def qfit_attention_error(q_pre, k_pre, v, table, s_k, s_q, m, element="e2m1", y_ref=None):
+    """MSE between Y_ref and the attention of the last token of each sequence
+    over the KV4 cache holding Q_KV4(RoPE(bf16(K_pre / s_k)) - m) and Q_KV4(V),
+    with query bf16(RoPE(Q_pre * s_q)) (one grid point of Algorithm 1)."""
+    q = np.asarray(q_pre, np.float32)
+    k = np.asarray(k_pre, np.float32)
+    vv = np.asarray(v, np.float32)
+    B, T, hq, d = q.shape
+    hkv = k.shape[2]
+    group = hq // hkv
+    qmax = 6.0 if element == "e2m1" else E1M2_MAX
+    pos = np.arange(T)
+    if y_ref is None:
+        y_ref = qfit_reference(q_pre, k_pre, v, table)
+    k_in = _bf16_round(k / np.asarray(s_k, np.float32)[None, None])
+    kt = np.stack([rope_f32(k_in[b], pos, table) for b in range(B)])
+    kt = (kt - np.asarray(m, np.float32)[None, None]).astype(np.float32)
+    g_k = np.float32(np.abs(kt).max() / np.float32(qmax * 448))
+    g_v = np.float32(np.abs(vv).max() / np.float32(qmax * 448))
+    kc, ks = quantize(kt.reshape(-1, d), g_k, element)
+    vc, vs = quantize(vv.reshape(-1, d), g_v, element)
+    K = dequantize(kc, ks, g_k, element).reshape(B, T, hkv, d)
+    V = dequantize(vc, vs, g_v, element).reshape(B, T, hkv, d)
+    q_in = (q[:, T - 1] * np.asarray(s_q, np.float32)[None]).astype(np.float32)       # [B, H_q, d]
+    qt = _bf16_round(rope_f32(q_in, np.full(B, T - 1), table)).astype(np.float64)
+    scale = 1.0 / np.sqrt(d)
+    y = np.stack([[attention_fp64(qt[b, h], K[b, :, h // group], V[b, :, h // group], scale) for h in range(hq)]
+                  for b in range(B)])
     return float(np.mean((y - y_ref) ** 2))
 
 
-def qfit_calibrate(q_pre, k_pre, v, table, q_pos, grid_s, grid_m, eps=1e-6, element="e2m1"):
-    """Algorithm 1: returns (s_q, s_k, m, errors[grid_s, grid_m])."""
-    hkv = k_pre.shape[1]
-    hq = q_pre.shape[1]
+def qfit_calibrate(q_pre, k_pre, v, table, grid_s, grid_m, eps=1e-6, element="e2m1"):
+    """Algorithm 1 on B calibration sequences ([B, T, heads, d] inputs).
+    Returns (s_q [H_q, d], s_k [H_kv, d], m [H_kv, d], errors[grid_s, grid_m]);
+    the first grid point (in alpha_s-major order) with the least error wins."""
+    hkv = np.asarray(k_pre).shape[2]
+    hq = np.asarray(q_pre).shape[2]
     s0_k = qfit_init_scale(k_pre, eps)
     s0_q = np.repeat(s0_k, hq // hkv, axis=0)                      # Replicate to query heads
-    mu = rope_f32(k_pre, np.arange(k_pre.shape[0]), table).astype(np.float64).mean(axis=0)
+    mu = qfit_shift_template(k_pre, table)
+    y_ref = qfit_reference(q_pre, k_pre, v, table)
     errors = np.full((grid_s, grid_m), np.inf)
     best = None
     for a in range(grid_s):
@@ -580,7 +627,7 @@ def qfit_calibrate(q_pre, k_pre, v, table, q_pos, grid_s, grid_m, eps=1e-6, elem
         for b in range(grid_m):
             alpha_m = b / grid_m
             m = (alpha_m * mu).astype(np.float32)
-            e = qfit_attention_error(q_pre, k_pre, v, table, q_pos, s_k, s_q, m, element)
+            e = qfit_attention_error(q_pre, k_pre, v, table, s_k, s_q, m, element, y_ref=y_ref)
             errors[a, b] = e
             if best is None or e < best[0]:
                 best = (e, s_q, s_k, m)

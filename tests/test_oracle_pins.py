@@ -495,12 +495,13 @@ def test_qfit_init_scale_pairs_and_floor():
     assert np.array_equal(s0[0], [0.5, 7, 0.5, 2, 0.5, 7, 0.5, 2])
 
 
-def _qfit_data(T=96, hq=4, hkv=2, d=128, seed=3, offset=3.0):
+def _qfit_data(B=3, T=64, hq=4, hkv=2, d=128, seed=3, offset=3.0):
+    """B calibration sequences [B, T, heads, d] with per-channel outliers and a common key offset."""
     rng = np.random.default_rng(seed)
     spread = np.exp(rng.standard_normal((hkv, d)))                 # channel outliers (paired scaling helps)
-    k = (rng.standard_normal((T, hkv, d)) * spread + offset).astype(np.float32)   # a mean (the shift helps)
-    q = rng.standard_normal((T, hq, d)).astype(np.float32)
-    v = rng.standard_normal((T, hkv, d)).astype(np.float32)
+    k = (rng.standard_normal((B, T, hkv, d)) * spread + offset).astype(np.float32)   # a mean (the shift helps)
+    q = rng.standard_normal((B, T, hq, d)).astype(np.float32)
+    v = rng.standard_normal((B, T, hkv, d)).astype(np.float32)
     return _bf(q), _bf(k), _bf(v)
 
 
@@ -508,21 +509,98 @@ def _bf(x):
     return O._bf16_round(x)
 
 
-def test_qfit_identity_point_and_invariance_without_quantization(monkeypatch):
+def _inverse_rope(c, positions, theta=1.0e6):
+    """Keys whose RoPE at each position is the fixed vector c: rotate c by minus
+    the RoPE angle pos * theta^(-2i/d) of each pair (i, i + d/2), in fp64."""
+    c = np.asarray(c, np.float64)
+    d = c.shape[-1]
+    half = d // 2
+    ang = -np.asarray(positions, np.float64)[:, None] * theta ** (-np.arange(half) * 2.0 / d)[None, :]
+    cs, sn = np.cos(ang)[:, None, :], np.sin(ang)[:, None, :]       # [T, 1, half] over heads
+    c1, c2 = c[None, ..., :half], c[None, ..., half:]
+    return np.concatenate([c1 * cs - c2 * sn, c1 * sn + c2 * cs], axis=-1)
+
+
+def test_qfit_shift_template_is_the_mean_of_the_post_rope_keys():
+    # Keys built so that RoPE maps every token to the same vector c: the
+    # template must be c, while the pre-RoPE keys (rotating with position)
+    # average to something else.
+    rng = np.random.default_rng(21)
+    B, T, hkv, d = 2, 48, 2, 128
+    c = rng.standard_normal((hkv, d)) * 2.0 + 1.0
+    k = np.stack([_inverse_rope(c, np.arange(T)) for _ in range(B)]).astype(np.float32)
+    mu = O.qfit_shift_template(k, O.rope_table(T))
+    assert mu.shape == (hkv, d)
+    assert np.abs(mu - c).max() < 1e-5 * np.abs(c).max()
+    assert np.abs(k.astype(np.float64).reshape(-1, hkv, d).mean(axis=0) - c).max() > 0.1
+
+
+def test_qfit_shift_template_at_position_zero_is_the_plain_mean():
+    # One token per sequence, at position 0 where RoPE is the identity.
+    rng = np.random.default_rng(22)
+    k = _bf(rng.standard_normal((5, 1, 2, 128)).astype(np.float32))
+    mu = O.qfit_shift_template(k, O.rope_table(1))
+    assert np.array_equal(mu, k.astype(np.float64)[:, 0].mean(axis=0))
+
+
+def test_qfit_reference_is_the_last_token_over_its_own_sequence():
+    q, k, v = _qfit_data(B=2, T=9)
+    tab = O.rope_table(9)
+    y = O.qfit_reference(q, k, v, tab)
+    # a single cached token: the output is that token's value (softmax of one logit)
+    y1 = O.qfit_reference(q[:, :1], k[:, :1], v[:, :1], tab)
+    assert np.allclose(y1, np.repeat(v[:, 0], 2, axis=1), rtol=0, atol=0)
+    # each sequence attends to its own tokens only: changing sequence 1 leaves sequence 0
+    k2, v2 = k.copy(), v.copy()
+    k2[1] += 1.0
+    v2[1] *= -1.0
+    y2 = O.qfit_reference(q, k2, v2, tab)
+    assert np.array_equal(y2[0], y[0]) and not np.allclose(y2[1], y[1])
+    # causal: the last token's output depends on every earlier token of its sequence
+    v3 = v.copy()
+    v3[0, 0] += 1.0
+    assert not np.array_equal(O.qfit_reference(q, k, v3, tab)[0], y[0])
+
+
+def test_qfit_identity_point_is_plain_kv4_attention():
+    # alpha_s = alpha_m = 0: the error is that of RoPE'd keys and values in the
+    # KV4 cache, with the cache and the attention taken from the separately
+    # pinned kv_append and decode_attention.
+    q, k, v = _qfit_data(B=2, T=40)
+    B, T, hq, d = q.shape
+    hkv = k.shape[2]
+    tab = O.rope_table(T)
+    ones_k, ones_q, zero = np.ones((hkv, d), np.float32), np.ones((hq, d), np.float32), np.zeros((hkv, d), np.float32)
+    e = O.qfit_attention_error(q, k, v, tab, ones_k, ones_q, zero)
+    kr = np.stack([O.rope_f32(k[b], np.arange(T), tab) for b in range(B)])
+    g_k = np.float32(np.abs(kr).max() / np.float32(2688.0))
+    g_v = np.float32(np.abs(v).max() / np.float32(2688.0))
+    kc = np.zeros((B, hkv, T, 64), np.uint8); ks = np.zeros((B, hkv, T, 8), np.uint8)
+    vc, vs = kc.copy(), ks.copy()
+    seq = np.repeat(np.arange(B), T); pos = np.tile(np.arange(T), B)
+    O.kv_append(kc, ks, vc, vs, kr.reshape(-1, hkv, d), v.reshape(-1, hkv, d), seq, pos, g_k, g_v)
+    qt = _bf(O.rope_f32(q[:, T - 1], np.full(B, T - 1), tab))
+    y = O.decode_attention(qt, kc, ks, vc, vs, np.full(B, T), g_k, g_v, 1.0 / np.sqrt(d))
+    expect = np.mean((y - O.qfit_reference(q, k, v, tab)) ** 2)
+    # decode_attention takes the softmax scale as an fp32 argument (1/sqrt(128)
+    # rounded to fp32); the calibration uses it in fp64: a ~1e-8 relative effect
+    assert np.isclose(e, expect, rtol=1e-6, atol=0)
+
+
+def test_qfit_grid_points_preserve_attention_without_quantization(monkeypatch):
     q, k, v = _qfit_data()
-    tab = O.rope_table(k.shape[0])
-    qp = np.array([10, 50, 95])
+    tab = O.rope_table(k.shape[1])
     # With the quantizer replaced by the identity, every grid point reproduces the
     # reference (paired scaling and the shift leave attention unchanged), up to the
     # bf16 rounding of the scaled inputs.
-    e_q = O.qfit_attention_error(q, k, v, tab, qp, np.ones((2, 128), np.float32), np.ones((4, 128), np.float32),
-                                 np.zeros((2, 128), np.float32))     # with the KV4 quantizer: ~4e-2
+    e_q = O.qfit_attention_error(q, k, v, tab, np.ones((2, 128), np.float32), np.ones((4, 128), np.float32),
+                                 np.zeros((2, 128), np.float32))     # with the KV4 quantizer
     monkeypatch.setattr(O, "quantize", lambda x, g, element="e2m1": (np.asarray(x, np.float32), g))
     monkeypatch.setattr(O, "dequantize", lambda c, s, g, element="e2m1": np.asarray(c, np.float64))
     s0 = O.qfit_init_scale(k, 1e-6)
-    mu = O.rope_f32(k, np.arange(k.shape[0]), tab).astype(np.float64).mean(axis=0)
+    mu = O.qfit_shift_template(k, tab)
     for alpha_s, alpha_m in [(0.0, 0.0), (0.5, 0.5), (0.8, 0.8)]:
-        e = O.qfit_attention_error(q, k, v, tab, qp, (s0 ** alpha_s).astype(np.float32),
+        e = O.qfit_attention_error(q, k, v, tab, (s0 ** alpha_s).astype(np.float32),
                                    np.repeat(s0 ** alpha_s, 2, axis=0).astype(np.float32),
                                    (alpha_m * mu).astype(np.float32))
         # bf16 rounding of the scaled q and k (relative 2^-9) is all that remains
@@ -531,10 +609,25 @@ def test_qfit_identity_point_and_invariance_without_quantization(monkeypatch):
 
 def test_qfit_calibration_prefers_the_shift_for_offset_keys():
     q, k, v = _qfit_data(offset=6.0)
-    tab = O.rope_table(k.shape[0])
-    qp = np.arange(80, 96)
-    s_q, s_k, m, err = O.qfit_calibrate(q, k, v, tab, qp, grid_s=3, grid_m=4)
+    tab = O.rope_table(k.shape[1])
+    s_q, s_k, m, err = O.qfit_calibrate(q, k, v, tab, grid_s=3, grid_m=4)
     assert err.shape == (3, 4) and np.isfinite(err).all()
     # keys with a large common offset: some shift beats none at alpha_s = 0
     assert err[0, 1:].min() < err[0, 0]
-    assert np.isclose(err.min(), O.qfit_attention_error(q, k, v, tab, qp, s_k, s_q, m))
+    # the returned transformation is the first least-error grid point's:
+    # S = S0^alpha_s (paired, replicated to the query heads), m = alpha_m * mu
+    a, b = np.unravel_index(err.argmin(), err.shape)
+    s0 = O.qfit_init_scale(k, 1e-6)
+    assert np.array_equal(s_k, (s0 ** (a / 3)).astype(np.float32))
+    assert np.array_equal(s_q, np.repeat(s_k, 2, axis=0))
+    assert np.array_equal(m, ((b / 4) * O.qfit_shift_template(k, tab)).astype(np.float32))
+    assert b > 0
+
+
+def test_qfit_calibration_avoids_the_shift_for_centred_keys():
+    # Without a common offset the template is ~0 and shifting buys nothing: the
+    # errors along alpha_m stay within the KV4 noise of the alpha_m = 0 column.
+    q, k, v = _qfit_data(offset=0.0, seed=9)
+    tab = O.rope_table(k.shape[1])
+    _, _, _, err = O.qfit_calibrate(q, k, v, tab, grid_s=2, grid_m=3)
+    assert np.all(err[:, 1:] > 0.8 * err[:, :1])
