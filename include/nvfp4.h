@@ -431,6 +431,44 @@ nvfp4_status decode_attention_nvfp4_static_scratch(const nvfp4_kv_cache* cache, 
                                                    int32_t num_q_heads, float softmax_scale, void* out_bf16,
                                                    void* stream);
 
+/*
+ * f4. Q-FIT calibration (Algorithm 1; Eq. 2): choose the paired pre-RoPE
+ * scale S (S_Q for the query heads, S_K for the KV heads, equal on each RoPE
+ * pair) and the post-RoPE key shift m by a grid search over (alpha_s,
+ * alpha_m) = (a / grid_s, b / grid_m): S = S0^alpha_s with S0[h, r] =
+ * max(max_t |K_pre[t,h,r]|, max_t |K_pre[t,h,r+64]|, eps); m = alpha_m * mu
+ * with mu the mean over tokens of RoPE(K_pre).  A grid point's error is the
+ * mean squared difference between the unquantized attention and the
+ * attention over the KV4 cache of Q_KV4(RoPE(bf16(K_pre / S_K)) - m) and
+ * Q_KV4(V) (static scales amax / (qmax * 448); kv_format as the cache's),
+ * with queries bf16(RoPE(Q_pre * S_Q)).  The calibration set is `batch`
+ * sequences of `tokens` tokens at positions 0..tokens-1; the causal
+ * attention is scored at the last token of each sequence, which attends to
+ * its whole sequence.  The KV4 side runs kv_append_rope_nvfp4 and
+ * decode_attention_nvfp4.  The first grid point (alpha_s-major) with the
+ * least error wins.
+ *   q_pre_bf16 : [batch, tokens, num_q_heads, 128] bf16 (pre-RoPE queries).
+ *   k_pre_bf16, v_bf16 : [batch, tokens, num_kv_heads, 128] bf16.
+ *   rope_table : nvfp4_rope_table output with rope_positions >= tokens
+ *                rounded up to even, 16-B aligned.
+ *   s_q [num_q_heads, 128], s_k [num_kv_heads, 128], m [num_kv_heads, 128]:
+ *                fp32 device outputs (S_Q, S_K, m of the chosen point).
+ *   errors_host: NULL or host fp64 [grid_s, grid_m], every point's error.
+ *   workspace  : nvfp4_qfit_workspace_size(...) bytes, 256-B aligned.
+ * Offline: the call synchronizes `stream` once per grid point (the key scale
+ * of a point is a host argument of the cache).  1 <= grid_s, grid_m <= 64,
+ * tokens <= 8192, head_dim == 128, num_q_heads % num_kv_heads == 0 with a
+ * group of at most 8 (SHAPE otherwise); eps > 0 and finite (INVALID_ARG).
+ * Device-side errors of the append and the attention set the status word.
+ */
+size_t nvfp4_qfit_workspace_size(int32_t batch, int32_t tokens, int32_t num_q_heads, int32_t num_kv_heads,
+                                 int32_t grid_s, int32_t grid_m);
+nvfp4_status nvfp4_qfit_calibrate(const void* q_pre_bf16, const void* k_pre_bf16, const void* v_bf16, int32_t batch,
+                                  int32_t tokens, int32_t num_q_heads, int32_t num_kv_heads, int32_t head_dim,
+                                  const float* rope_table, int64_t rope_positions, int32_t grid_s, int32_t grid_m,
+                                  double eps, int32_t kv_format, float* s_q, float* s_k, float* m,
+                                  double* errors_host, void* workspace, size_t workspace_bytes, void* stream);
+
 /* Synchronize `stream`, copy the device status word of the current device to
  * *status_host (an nvfp4_status value) and clear it. */
 nvfp4_status nvfp4_get_device_status(int32_t* status_host, void* stream);

@@ -594,8 +594,10 @@ def qfit_attention_error(q_pre, k_pre, v, table, s_k, s_q, m, element="e2m1", y_
     k_in = _bf16_round(k / np.asarray(s_k, np.float32)[None, None])
     kt = np.stack([rope_f32(k_in[b], pos, table) for b in range(B)])
     kt = (kt - np.asarray(m, np.float32)[None, None]).astype(np.float32)
-    g_k = np.float32(np.abs(kt).max() / np.float32(qmax * 448))
-    g_v = np.float32(np.abs(vv).max() / np.float32(qmax * 448))
+    # static scales; an all-zero tensor gets scale 1 (the tensor-scale convention)
+    a_k, a_v = np.abs(kt).max(), np.abs(vv).max()
+    g_k = np.float32(a_k / np.float32(qmax * 448)) if a_k > 0 else np.float32(1.0)
+    g_v = np.float32(a_v / np.float32(qmax * 448)) if a_v > 0 else np.float32(1.0)
     kc, ks = quantize(kt.reshape(-1, d), g_k, element)
     vc, vs = quantize(vv.reshape(-1, d), g_v, element)
     K = dequantize(kc, ks, g_k, element).reshape(B, T, hkv, d)

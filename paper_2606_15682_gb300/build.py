@@ -32,7 +32,7 @@ BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(BUILD, "libnvfp4.so")
 BUILD_DEBUG = os.path.join(PKG, "_build_debug")
 BUILD_TIMELINE = os.path.join(PKG, "_build_timeline")
-SOURCES = ["api.cu", "quantize.cu", "kv_append.cu", "attention.cu", "gemm.cu"]
+SOURCES = ["api.cu", "quantize.cu", "kv_append.cu", "attention.cu", "gemm.cu", "qfit.cu"]
 HEADERS = ["common.cuh", "nvfp4_quant.cuh", os.path.join("..", "..", "include", "nvfp4.h")]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC,-fvisibility=hidden", "-Xptxas", "-v"]

@@ -68,6 +68,9 @@ _attn = _sig("decode_attention_nvfp4", [ctypes.POINTER(KVCacheStruct), _p, _i32,
 _attn_quant = _sig("decode_attention_nvfp4_quantize",
                    [ctypes.POINTER(KVCacheStruct), _p, _i32, _f32, _p, _p, _p, _p, _sz, _p])
 _attn_static = _sig("decode_attention_nvfp4_static_scratch", [ctypes.POINTER(KVCacheStruct), _p, _i32, _f32, _p, _p])
+_qfit_ws = _sig("nvfp4_qfit_workspace_size", [_i32, _i32, _i32, _i32, _i32, _i32], _sz)
+_qfit = _sig("nvfp4_qfit_calibrate", [_p, _p, _p, _i32, _i32, _i32, _i32, _i32, _p, _i64, _i32, _i32,
+                                      ctypes.c_double, _i32, _p, _p, _p, _p, _p, _sz, _p])
 _get_status = _sig("nvfp4_get_device_status", [ctypes.POINTER(_i32), _p])
 _status_string = _sig("nvfp4_status_string", [ctypes.c_int], ctypes.c_char_p)
 _launch_count = _sig("nvfp4_launch_count", [], ctypes.c_uint64)
@@ -237,6 +240,26 @@ def decode_attention_nvfp4_static_scratch(cache, q, softmax_scale, out, stream=N
                                                                  _ptr(out), _stream(stream)))
 
 
+def nvfp4_qfit_workspace_size(batch, tokens, num_q_heads, num_kv_heads, grid_s, grid_m):
+    return int(_qfit_ws(batch, tokens, num_q_heads, num_kv_heads, grid_s, grid_m))
+
+
+def nvfp4_qfit_calibrate(q_pre, k_pre, v, rope_table, grid_s, grid_m, eps, kv_format, s_q, s_k, m, errors,
+                         workspace, stream=None):
+    """q_pre [B, T, H_q, 128], k_pre and v [B, T, H_kv, 128] bf16; rope_table fp32 [n, 64, 2];
+    s_q, s_k, m fp32 device outputs; errors: a host (CPU) float64 tensor of grid_s * grid_m, or None."""
+    B, T, hq, d = q_pre.shape
+    hkv = k_pre.shape[2]
+    if errors is not None and (errors.device.type != "cpu" or errors.dtype != torch.float64 or
+                               not errors.is_contiguous() or errors.numel() != grid_s * grid_m):
+        raise ValueError("errors must be a contiguous CPU float64 tensor of grid_s * grid_m")
+    _check("nvfp4_qfit_calibrate",
+           _qfit(_ptr(q_pre), _ptr(k_pre), _ptr(v), B, T, hq, hkv, d, _ptr(rope_table), rope_table.shape[0], grid_s,
+                 grid_m, float(eps), kv_format, _ptr(s_q), _ptr(s_k), _ptr(m),
+                 None if errors is None else ctypes.c_void_p(errors.data_ptr()), _ptr(workspace),
+                 workspace.numel() * workspace.element_size(), _stream(stream)))
+
+
 def nvfp4_get_device_status(stream=None):
     v = _i32(0)
     _check("nvfp4_get_device_status", _get_status(ctypes.byref(v), _stream(stream)))
@@ -278,5 +301,5 @@ EXPORTED = ["nvfp4_scales_bytes", "nvfp4_tensor_scale", "nvfp4_quantize", "nvfp4
             "mxfp4_scales_bytes", "mxfp4_quantize", "mxfp4_linear", "mxfp4_linear_swiglu_quantize",
             "kv_append_nvfp4", "kv_append_rope_nvfp4", "nvfp4_rope_table", "decode_attention_nvfp4_workspace_size", "decode_attention_nvfp4",
             "decode_attention_nvfp4_quantize",
-            "decode_attention_nvfp4_static_scratch",
+            "decode_attention_nvfp4_static_scratch", "nvfp4_qfit_workspace_size", "nvfp4_qfit_calibrate",
             "nvfp4_get_device_status", "nvfp4_status_string", "nvfp4_launch_count", "nvfp4_debug_inject_fault"]

@@ -179,6 +179,25 @@ def test_kv_and_attention_validation():
     assert L.decode_attention_nvfp4_quantize(ctypes.byref(cache()), p, 4, f, p, p, p, p, ws - 16, s) == 2   # workspace
     assert L.decode_attention_nvfp4_quantize(ctypes.byref(cache()), p, 4, f, p, odd, p, p, ws, s) == 3      # codes align
     assert L.decode_attention_nvfp4_quantize(ctypes.byref(cache(kv_format=5)), p, 4, f, p, p, p, p, ws, s) == 1
+    # Q-FIT calibration: arguments checked before any CUDA call
+    qws = N.nvfp4_qfit_workspace_size(2, 64, 4, 2, 3, 3)
+    assert qws > 0 and N.nvfp4_qfit_workspace_size(2, 64, 4, 3, 3, 3) == 0          # 4 % 3
+    assert N.nvfp4_qfit_workspace_size(2, 8193, 4, 2, 3, 3) == 0                        # > 8192 tokens
+    assert N.nvfp4_qfit_workspace_size(2, 64, 4, 2, 0, 3) == 0                          # empty grid
+    Q = L.nvfp4_qfit_calibrate
+    ok = (p, p, p, 2, 64, 4, 2, 128, p, 64, 3, 3, ctypes.c_double(1e-6), 0, p, p, p, None, p, qws, s)
+    def qcall(**kw):
+        a = list(ok)
+        for i, val in kw.items():
+            a[int(i[1:])] = val
+        return Q(*a)
+    assert qcall(a0=None) == 1                                   # no queries
+    assert qcall(a13=2) == 1                                     # kv format
+    assert qcall(a12=ctypes.c_double(0.0)) == 1                  # eps
+    assert qcall(a7=64) == 2                                     # head_dim
+    assert qcall(a9=63) == 2                                     # table shorter than the cache
+    assert qcall(a19=qws - 1) == 2                               # workspace
+    assert qcall(a18=ctypes.c_void_p(0x10010)) == 3              # workspace alignment
     # static-scratch attention: a problem whose partials exceed the fixed
     # scratch is refused on the host, before any CUDA call
     big = cache(batch=64, num_kv_heads=1, capacity=131072)

@@ -413,30 +413,41 @@ def test_decode_attention_e1m2_matches_fp64(N, B, hq, hkv, lens):
 
 # ------------------------------------------------ Q-FIT calibration (Alg. 1) ---
 
-def test_qfit_calibration_matches_oracle_grid(N):
-    """The GPU grid search (library kernels for the KV4 path) against the oracle's:
-    per-point errors close, and the same best point."""
-    from paper_2606_15682_gb300 import qfit
-    rng = np.random.default_rng(5)
-    T, hq, hkv, d = 256, 8, 2, 128
+def _qfit_case(B, T, hq, hkv, seed, offset=6.0):
+    rng = np.random.default_rng(seed)
+    d = 128
     spread = np.exp(rng.standard_normal((hkv, d)))
-    k = O._bf16_round((rng.standard_normal((T, hkv, d)) * spread + 6.0).astype(np.float32))
-    q = O._bf16_round(rng.standard_normal((T, hq, d)).astype(np.float32))
-    v = O._bf16_round(rng.standard_normal((T, hkv, d)).astype(np.float32))
-    table = O.rope_table(T)
-    q_pos = np.arange(T - 16, T)
+    k = O._bf16_round((rng.standard_normal((B, T, hkv, d)) * spread + offset).astype(np.float32))
+    q = O._bf16_round(rng.standard_normal((B, T, hq, d)).astype(np.float32))
+    v = O._bf16_round(rng.standard_normal((B, T, hkv, d)).astype(np.float32))
+    return q, k, v
+
+
+@pytest.mark.parametrize("kv_format", ["e2m1", "e1m2"])
+def test_qfit_calibration_matches_oracle_grid(N, kv_format):
+    """nvfp4_qfit_calibrate (every step in the library's kernels) against the
+    oracle's Algorithm 1: per-point errors close, the same best point, and the
+    same transformation."""
+    from paper_2606_15682_gb300 import qfit
+    B, T, hq, hkv = 4, 255, 8, 2                          # odd T: the cache capacity rounds up
+    q, k, v = _qfit_case(B, T, hq, hkv, seed=5)
+    table = O.rope_table(T + 1)
     dev = "cuda"
+    fmt = N.KV_E2M1 if kv_format == "e2m1" else N.KV_E1M2
     s_q, s_k, m, err = qfit.qfit_calibrate(torch.from_numpy(q).to(dev).to(torch.bfloat16),
                                            torch.from_numpy(k).to(dev).to(torch.bfloat16),
                                            torch.from_numpy(v).to(dev).to(torch.bfloat16),
-                                           torch.from_numpy(table).to(dev), torch.from_numpy(q_pos).to(dev),
-                                           grid_s=3, grid_m=3)
-    r_sq, r_sk, r_m, r_err = O.qfit_calibrate(q, k, v, table, q_pos, grid_s=3, grid_m=3)
+                                           torch.from_numpy(table).to(dev), grid_s=3, grid_m=3, kv_format=fmt)
+    torch.cuda.synchronize()
+    assert N.nvfp4_get_device_status() == 0
+    r_sq, r_sk, r_m, r_err = O.qfit_calibrate(q, k, v, table, grid_s=3, grid_m=3, element=kv_format)
     err = err.numpy()
-    # the GPU attention rounds its output to bf16 and multiplies in f16: small relative differences
-    assert np.allclose(err, r_err, rtol=0.05, atol=1e-6), (err, r_err)
+    # the GPU attention multiplies in f16 and rounds its output to bf16, its
+    # reference is fp32: small relative differences in each point's error
+    assert np.allclose(err, r_err, rtol=0.05, atol=1e-7), (err, r_err)
     assert np.unravel_index(err.argmin(), err.shape) == np.unravel_index(r_err.argmin(), r_err.shape)
-    assert np.allclose(s_k.cpu().numpy(), r_sk, rtol=1e-6) and np.allclose(m.cpu().numpy(), r_m, rtol=1e-5, atol=1e-6)
+    assert np.allclose(s_k.cpu().numpy(), r_sk, rtol=1e-6) and np.allclose(s_q.cpu().numpy(), r_sq, rtol=1e-6)
+    assert np.allclose(m.cpu().numpy(), r_m, rtol=1e-5, atol=1e-6)
     assert r_err.min() < r_err[0, 0]            # the calibration improves on no transform
 
 
