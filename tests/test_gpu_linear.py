@@ -9,7 +9,7 @@ import numpy as np
 import pytest
 import torch
 
-from _util import TOL, assert_close, errors, f32, lib, u8
+from _util import TOL, assert_close, assert_nvfp4_within, errors, f32, lib, swiglu_tolerance, u8
 from oracle import nvfp4_oracle as O
 from paper_2606_15682_gb300 import synth
 
@@ -219,23 +219,21 @@ def swiglu_case(N, M, I, K, seed, rows=None):
                                    M, I, K, torch.tensor([g_out], device=dev), out_c, out_s)
     torch.cuda.synchronize()
     assert N.nvfp4_get_device_status() == 0
-    return h, g_out, rows, u8(out_c), u8(out_s)
+    return h, g_out, rows, u8(out_c), u8(out_s), swiglu_tolerance(G, U, h)
 
 
 @pytest.mark.parametrize("M,I,K", [(256, 128, 256), (129, 384, 512), (300, 256, 1024), (640, 512, 768)])
 def test_linear_swiglu_quantize(N, M, I, K):
-    """h = SiLU(gate) * up from the fp32 accumulators, quantized with a static scale:
-    scales within one E4M3 step of the oracle's, elements within the quantization
-    error bound of the fp64 h, almost all codes identical, padding scales zero."""
-    h, g_out, rows, out_c, out_s = swiglu_case(N, M, I, K, seed=M + I + K)
+    """h = SiLU(gate) * up from the fp32 accumulators, quantized with a static
+    scale.  The kernel's SiLU uses the hardware tanh approximation, so every
+    block scale and code must be one the recipe gives for some h' within that
+    approximation's error of the exact fp64 h; no other difference is allowed.
+    Most equal the oracle's quantization of h; padding scales are zero."""
+    h, g_out, rows, out_c, out_s, tol = swiglu_case(N, M, I, K, seed=M + I + K)
     rc, rs = O.quantize(h.astype(np.float32), g_out)
     gs = O.scales_from_mma(out_s, M, I)
-    assert np.abs(gs.astype(int) - rs.astype(int)).max() <= 1
-    assert (gs == rs).mean() > 0.99
-    assert (out_c == rc).mean() > 0.99
-    deq = O.dequantize(out_c, gs, g_out)
-    S = O.e4m3_decode(gs).repeat(16, axis=1)
-    assert np.all(np.abs(deq - h) <= 1.5 * S * np.float64(g_out) + 1e-6 * np.abs(h))
+    assert_nvfp4_within(out_c, gs, h, tol, g_out, what=f"swiglu {M}x{I}x{K}")
+    assert (gs == rs).mean() > 0.99 and (out_c == rc).mean() > 0.99
     pad = np.setdiff1d(np.arange(O.mma_scale_bytes(M, I)), O._mma_offsets(M, I // 16).ravel())
     assert not out_s[pad].any(), "padding rows of the output scales must be zero"
 
@@ -245,13 +243,9 @@ def test_linear_swiglu_quantize_prefill_shape_then_down(N):
     then fed to the down projection as its A operand."""
     M, I, K, Hd = 2048, 8960, 1536, 1536
     rows = np.sort(np.r_[np.random.default_rng(2).choice(M, 48, replace=False), M - 1])
-    h, g_out, rows, out_c, out_s = swiglu_case(N, M, I, K, seed=99, rows=rows)
+    h, g_out, rows, out_c, out_s, tol = swiglu_case(N, M, I, K, seed=99, rows=rows)
     gs = O.scales_from_mma(out_s, M, I)[rows]
-    rc, rs = O.quantize(h.astype(np.float32), g_out)
-    assert np.abs(gs.astype(int) - rs.astype(int)).max() <= 1 and (out_c[rows] == rc).mean() > 0.99
-    deq = O.dequantize(out_c[rows], gs, g_out)
-    S = O.e4m3_decode(gs).repeat(16, axis=1)
-    assert np.all(np.abs(deq - h) <= 1.5 * S * np.float64(g_out) + 1e-6 * np.abs(h))
+    assert_nvfp4_within(out_c[rows], gs, h, tol, g_out, what="swiglu 1.5B prefill")
     # down projection straight from the fused output
     gen = torch.Generator().manual_seed(7)
     wd_c, wd_s = random_operand(Hd, I, gen)
