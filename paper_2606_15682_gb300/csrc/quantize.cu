@@ -616,18 +616,16 @@ NVFP4_API nvfp4_status nvfp4_quantize_dynamic(const void* x_bf16, int64_t rows, 
   }
   if (grid > cap) grid = cap;
   if (grid > 0xFFFF) grid = 0xFFFF;  // the barrier counts arrivals in 16 bits
-  // The grid never exceeds the blocks the device holds at once, so every
-  // block becomes resident and the grid barrier completes: blocks that find
-  // their SM still occupied by the previous kernel in the stream (programmatic
-  // dependent launch) start when it retires, and that kernel does not wait on
-  // this one.  A cooperative launch gives the same guarantee up front but
-  // measured 2-4 us slower per four-quantization step (its launch does not
-  // overlap the previous kernel).  Work on other streams that holds SMs for
-  // longer than the barrier's 2 s bound makes the call report TIMEOUT.
+  // Cooperative: every block is resident at once, so the grid barrier can
+  // complete.  A plain launch with programmatic dependent launch (the grid is
+  // capped at the co-resident blocks anyway) was measured too: 2-4 us faster
+  // per four back-to-back quantizations, but slower inside a step that
+  // alternates quantizations and GEMMs (32B prefill layer: 1697 vs 1658-1679
+  // us graph-replayed), so the cooperative launch stays.
   cudaLaunchConfig_t cfg = {};
   cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  attr[0].id = cudaLaunchAttributeCooperative;
+  attr[0].val.cooperative = 1;
   cfg.gridDim = dim3(grid);
   cfg.blockDim = dim3(kThreads);
   cfg.dynamicSmemBytes = stash_iters * kStashIterBytes;
