@@ -48,7 +48,7 @@ CSRC = os.path.join(ROOT, "paper_2606_15682_gb300", "csrc")
 # same kernel and shape (commands in profiles/).  Each entry holds only while the kernel sources
 # hash to the value they had at capture time; otherwise the line reports traffic = null.
 NCU_TRAFFIC = {
-    "gemm": {"bytes": None, "sources": ("gemm.cu", "common.cuh"), "sha": None,
+    "gemm": {"bytes": 661180000 + 863110000, "sources": ("gemm.cu", "common.cuh"), "sha": "283b225788dd4181",
              "shape": (8192, 55296, 5120),
              "profile": "profiles/gemm_qwen32b_prefill_gate_up_m8192_n55296_k5120.md"},
     "attention": {"bytes": 1208783616 + 22233856, "sources": ("attention.cu", "common.cuh"),
