@@ -9,6 +9,7 @@
     python -m paper_2606_15682_gb300.cases mx_quantize --workload qwen32b_prefill_linears_m8192 --linear down --rotate
     python -m paper_2606_15682_gb300.cases mx_gemm_swiglu --workload qwen32b_prefill_linears_m8192 --rotate
     NVFP4_TIMELINE=1 python -m paper_2606_15682_gb300.cases quantize_timeline --workload qwen1.5b_prefill_linears_m2048 --linear qkv
+    NVFP4_TIMELINE=1 python -m paper_2606_15682_gb300.cases gemm_timeline --workload w4a4_linear_m16_k1536_n1536 --linear linear
 
 Inputs are seeded synthetic tensors (paper_2606_15682_gb300.synth); for the
 attention case the cache is filled with seeded random codes and scales
@@ -16,7 +17,9 @@ directly, which is enough to time the kernel.  Prints the mean CUDA-event time
 of the measured call.  quantize_timeline (timeline build, NVFP4_TIMELINE=1)
 prints, for one launch of the one-launch dynamic quantizer after an L2 flush,
 when its blocks started, finished their loads, arrived at the grid barrier,
-were released and issued their stores.
+were released and issued their stores; gemm_timeline the same for one
+single-CTA GEMM launch (set-up, first stage issued and landed, last MMA
+issued, last accumulator seen by the epilogue, stores complete, exit).
 """
 from __future__ import annotations
 
@@ -91,10 +94,52 @@ def _quantize_timeline(a, dev):
         print(f"  {name:13s} min {v[0] / 1e3:6.2f}  median {v[len(v) // 2] / 1e3:6.2f}  max {v[-1] / 1e3:6.2f} us")
 
 
+def _gemm_timeline(a, dev):
+    import ctypes
+    if not hasattr(N._lib, "nvfp4_timeline_gemm"):
+        raise SystemExit("gemm_timeline needs the timeline build: run with NVFP4_TIMELINE=1")
+    read = N._lib.nvfp4_timeline_gemm
+    read.argtypes = [ctypes.c_void_p]
+    read.restype = ctypes.c_int
+    x, W = synth.linear_inputs(a.workload, a.linear, device=dev)
+    M, K = x.shape
+    Nn = W.shape[0]
+    ac, asf, ga = _quantized(x)
+    wc, wsf, gw = _quantized(W)
+    out = torch.empty(M, Nn, dtype=torch.bfloat16, device=dev)
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    for _ in range(3):
+        N.nvfp4_linear(ac, asf, ga, wc, wsf, gw, out, M, Nn, K)
+    host = (ctypes.c_ulonglong * (1024 * 8))()
+    read(host)  # clears the warm-up launches' stamps
+    flush.zero_()
+    torch.cuda._sleep(1_000_000)
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
+    ev[0].record()
+    N.nvfp4_linear(ac, asf, ga, wc, wsf, gw, out, M, Nn, K)
+    ev[1].record()
+    if read(host) != 0:
+        raise SystemExit("reading the timeline failed")
+    assert N.nvfp4_get_device_status() == 0
+    rows = [host[8 * c:8 * c + 8] for c in range(1024) if host[8 * c] != 0]
+    if not rows:
+        raise SystemExit("no stamps: this shape does not run the single-CTA GEMM kernel")
+    t0 = min(r[0] for r in rows)
+    print(f"{a.workload}/{a.linear}: {M}x{Nn}x{K}, {len(rows)} CTAs, event {ev[0].elapsed_time(ev[1]) * 1e3:.2f} us, "
+          f"in-kernel span {(max(r[7] for r in rows) - t0) / 1e3:.2f} us")
+    names = ["entry", "set-up done", "1st stage issued", "1st stage landed", "last MMA issued",
+             "last acc. seen", "stores done", "exit"]
+    for e, name in enumerate(names):
+        v = sorted(r[e] - t0 for r in rows if r[e] != 0)
+        if v:
+            print(f"  {name:16s} min {v[0] / 1e3:6.2f}  median {v[len(v) // 2] / 1e3:6.2f}  max {v[-1] / 1e3:6.2f} us")
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("kernel", choices=["gemm", "gemm_swiglu", "quantize", "quantize_dynamic", "tensor_scale",
-                                       "attention", "mx_gemm", "mx_quantize", "mx_gemm_swiglu", "quantize_timeline"])
+                                       "attention", "mx_gemm", "mx_quantize", "mx_gemm_swiglu", "quantize_timeline",
+                                       "gemm_timeline"])
     ap.add_argument("--rotate", action="store_true", help="MXFP4: 32-element block rotation before quantizing")
     ap.add_argument("--workload", default="qwen1.5b_prefill_linears_m2048")
     ap.add_argument("--linear", default="gate_up")
@@ -107,6 +152,9 @@ def main():
     torch.cuda.set_device(dev)
     if a.kernel == "quantize_timeline":
         _quantize_timeline(a, dev)
+        return
+    if a.kernel == "gemm_timeline":
+        _gemm_timeline(a, dev)
         return
     if a.kernel == "gemm_swiglu":
         # gate_up of the workload with SwiGLU + NVFP4 quantization of the down

@@ -139,6 +139,22 @@ __device__ __forceinline__ void unit_coords(int u, int msup, int tiles_n, int gr
   *nb = r / rows;
 }
 
+// Timeline build (-DNVFP4_TIMELINE): the 1-CTA kernel records, per CTA, the
+// globaltimer at kernel entry (0), after its set-up (barriers, TMEM, the
+// previous kernel's completion) (1), when the producer issued the first stage
+// (2), when the first stage's data had landed for the MMA issuer (3), when the
+// last MMA was issued (4), when the first epilogue warp saw the last tile's
+// accumulator (5), when its stores had completed (6) and at exit (7).
+#ifdef NVFP4_TIMELINE
+constexpr int kGemmTimelineCtas = 1024;
+__device__ unsigned long long g_gemm_timeline[kGemmTimelineCtas][8];
+__device__ __forceinline__ void gemm_stamp(int event) {
+  if (blockIdx.x < kGemmTimelineCtas) g_gemm_timeline[blockIdx.x][event] = globaltimer_ns();
+}
+#else
+__device__ __forceinline__ void gemm_stamp(int) {}
+#endif
+
 // Scale-format bit of the block-scaled MMA instruction descriptor (bit 23: UE8M0).
 constexpr uint32_t kScaleE8M0 = 1u << 23;
 
@@ -207,6 +223,7 @@ __global__ void __launch_bounds__(C::kThreads, 1)
   const int msup = args.tiles_m;
   const int total_units = msup * args.tiles_n;
   const int cta_id = blockIdx.x, n_ctas = gridDim.x;
+  if (threadIdx.x == 0) gemm_stamp(0);
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
@@ -234,6 +251,7 @@ __global__ void __launch_bounds__(C::kThreads, 1)
   __syncthreads();
   tc_fence_after();
   griddep_wait_and_release();
+  if (threadIdx.x == 0) gemm_stamp(1);
   const uint32_t tmem = *tmem_slot;
 
   auto fail = [&]() {
@@ -248,6 +266,9 @@ __global__ void __launch_bounds__(C::kThreads, 1)
     uint32_t issued_parity[kStages];
     bool issued[kStages];
     for (int s = 0; s < kStages; ++s) issued[s] = false;
+#ifdef NVFP4_TIMELINE
+    bool first_issue = true;
+#endif
     for (int u = cta_id; u < total_units && !abort_flag; u += n_ctas) {
       int ms, nb;
       unit_coords(u, msup, args.tiles_n, args.group_m, &ms, &nb);
@@ -267,6 +288,10 @@ __global__ void __launch_bounds__(C::kThreads, 1)
                     sfb_tiles + (static_cast<size_t>(j) * kgroups) * 512 + static_cast<size_t>(kb) * C::kSfaBytes,
                     C::kSfaBytes, &full[stage]);
         tma_load_2d(sB + stage * C::kTileBytesB, &tmap_b, &full[stage], kb * (BK / 2), nb * BN);
+#ifdef NVFP4_TIMELINE
+        if (first_issue) gemm_stamp(2);
+        first_issue = false;
+#endif
         issued[stage] = true;
         issued_parity[stage] = phase;
         if (++stage == kStages) { stage = 0; phase ^= 1u; }
@@ -292,6 +317,7 @@ __global__ void __launch_bounds__(C::kThreads, 1)
       bool ok = true;
       for (int kb = 0; kb < kblocks; ++kb) {
         if (!mbar_wait_bounded(&sfready[stage], phase, &abort_flag)) { fail(); ok = false; break; }
+        if (local == 0 && kb == 0) gemm_stamp(3);
         tc_fence_after();
         const uint32_t sfa_col = tmem + C::kSfTmemCol + stage * C::kSfCols;
         const uint32_t sfb_col = sfa_col + 16;
@@ -306,6 +332,7 @@ __global__ void __launch_bounds__(C::kThreads, 1)
       }
       if (!ok) break;
       tc_commit(&tfull[acc]);
+      gemm_stamp(4);
     }
     // Wait until every MMA issued above has retired before TMEM is freed.
     tc_commit(drain);
@@ -361,6 +388,7 @@ __global__ void __launch_bounds__(C::kThreads, 1)
         if (!ok && !abort_flag) fail();
       }
       if (!__shfl_sync(0xffffffffu, ok, 0)) break;
+      if (warp == 3 && lane == 0) gemm_stamp(5);
       tc_fence_after();
       // Drain 128 columns into registers, then hand the accumulator back.
       uint32_t r[128];
@@ -397,11 +425,13 @@ __global__ void __launch_bounds__(C::kThreads, 1)
       }
     }
     if (lane == 0) bulk_wait_all();
+    if (warp == 3 && lane == 0) gemm_stamp(6);
   }
 
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
+  if (threadIdx.x == 0) gemm_stamp(7);
   if (warp == 1) tmem_dealloc(tmem, kTmemCols);
 }
 
@@ -1278,3 +1308,16 @@ NVFP4_API nvfp4_status nvfp4_interleave_gate_up(const void* w_gate, const void* 
   count_launches(1);
   return launch_status();
 }
+
+#ifdef NVFP4_TIMELINE
+// Timeline build only (not part of the C ABI of include/nvfp4.h): copy the
+// per-CTA stamps of the last 1-CTA GEMM launch ([1024][8] uint64, ns, zero
+// where a CTA or event did not occur) to host memory, then clear them.
+// Synchronizes the device.
+extern "C" __attribute__((visibility("default"))) int nvfp4_timeline_gemm(unsigned long long* host) {
+  if (cudaDeviceSynchronize() != cudaSuccess) return 1;
+  if (cudaMemcpyFromSymbol(host, nvfp4::g_gemm_timeline, sizeof(nvfp4::g_gemm_timeline)) != cudaSuccess) return 1;
+  static unsigned long long zero[nvfp4::kGemmTimelineCtas * 8];
+  return cudaMemcpyToSymbol(nvfp4::g_gemm_timeline, zero, sizeof(zero)) == cudaSuccess ? 0 : 1;
+}
+#endif

@@ -49,7 +49,7 @@ def test_timeline_build_compiles_and_exports_every_call():
     so = ctypes.CDLL(path)
     for name in header_functions():
         assert hasattr(so, name), name
-    assert hasattr(so, "nvfp4_timeline_quantize_dynamic")
+    assert hasattr(so, "nvfp4_timeline_quantize_dynamic") and hasattr(so, "nvfp4_timeline_gemm")
     assert not hasattr(ctypes.CDLL(B.build(timeline=False, debug=False)), "nvfp4_timeline_quantize_dynamic")
     with pytest.raises(ValueError):
         B.build(debug=True, timeline=True)
