@@ -146,7 +146,11 @@ nvfp4_status nvfp4_scales_relayout(const uint8_t* src, uint8_t* dst, int64_t row
  * paper's compute speedup comes from, Sec. 5.3):
  *   out[m, n] = bf16_rne( (g_a * g_w) * sum_k a[m,k] * w[n,k] )
  * with a[m,k] = e2m1 * e4m3 of A (no g) and likewise for W; the sum is
- * accumulated in fp32 by the tensor core (tcgen05 block-scaled MMA).
+ * accumulated in fp32 by the tensor core (tcgen05 block-scaled MMA).  When
+ * N % 256 == 0, K >= 4096 and the 256 x 256 tiles are too few to occupy the
+ * GPU (decode-sized M), K is split into 2-4 contiguous ranges whose fp32 partial
+ * sums are added in range order in the cluster's shared memory: the result
+ * is deterministic for a given shape.
  *   a_codes  : [M, K/2] bytes (K-major), 16-B aligned.
  *   a_scales : MMA layout for [M, K].
  *   w_codes  : [N, K/2] bytes (K-major, i.e. the nn.Linear weight [N, K]).
@@ -483,8 +487,9 @@ nvfp4_status nvfp4_get_device_status(int32_t* status_host, void* stream);
  *     undefined, and the device stays usable.
  *   NVFP4_FAULT_GEMM_SKIP_STAGE: in the next launch of a CTA-pair GEMM kernel
  *     (the 256 x 256 tiles that nvfp4_linear / mxfp4_linear use when N % 256
- *     == 0 and the tiles fill the GPU, and the fused SwiGLU calls), both CTAs
- *     of pair 0 leave their first ring stage neither armed nor loaded; the MMA
+ *     == 0, with or without a split of K across a cluster, and the fused
+ *     SwiGLU calls), both CTAs of the first pair leave their first ring stage
+ *     of their K range neither armed nor loaded; the MMA
  *     issuer's and the scale copiers' bounded waits run out after ~2 s, every
  *     role of the pair stops, the MMAs issued so far drain and TMEM is freed.
  *     The call reports NVFP4_ERR_TIMEOUT, its output is undefined, and the

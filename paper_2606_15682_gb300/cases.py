@@ -18,8 +18,9 @@ of the measured call.  quantize_timeline (timeline build, NVFP4_TIMELINE=1)
 prints, for one launch of the one-launch dynamic quantizer after an L2 flush,
 when its blocks started, finished their loads, arrived at the grid barrier,
 were released and issued their stores; gemm_timeline the same for one
-single-CTA GEMM launch (set-up, first stage issued and landed, last MMA
-issued, last accumulator seen by the epilogue, stores complete, exit).
+single-CTA or split-K GEMM launch (set-up, first stage issued and landed, last
+MMA issued, last accumulator seen by the epilogue or, split-K, the partial
+drained into shared memory, stores complete, exit).
 """
 from __future__ import annotations
 
@@ -123,12 +124,12 @@ def _gemm_timeline(a, dev):
     assert N.nvfp4_get_device_status() == 0
     rows = [host[8 * c:8 * c + 8] for c in range(1024) if host[8 * c] != 0]
     if not rows:
-        raise SystemExit("no stamps: this shape does not run the single-CTA GEMM kernel")
+        raise SystemExit("no stamps: this shape runs neither the single-CTA nor the split-K GEMM kernel")
     t0 = min(r[0] for r in rows)
     print(f"{a.workload}/{a.linear}: {M}x{Nn}x{K}, {len(rows)} CTAs, event {ev[0].elapsed_time(ev[1]) * 1e3:.2f} us, "
           f"in-kernel span {(max(r[7] for r in rows) - t0) / 1e3:.2f} us")
     names = ["entry", "set-up done", "1st stage issued", "1st stage landed", "last MMA issued",
-             "last acc. seen", "stores done", "exit"]
+             "acc. seen/drained", "stores done", "exit"]
     for e, name in enumerate(names):
         v = sorted(r[e] - t0 for r in rows if r[e] != 0)
         if v:

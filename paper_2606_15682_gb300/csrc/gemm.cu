@@ -144,7 +144,10 @@ __device__ __forceinline__ void unit_coords(int u, int msup, int tiles_n, int gr
 // previous kernel's completion) (1), when the producer issued the first stage
 // (2), when the first stage's data had landed for the MMA issuer (3), when the
 // last MMA was issued (4), when the first epilogue warp saw the last tile's
-// accumulator (5), when its stores had completed (6) and at exit (7).
+// accumulator (5), when its stores had completed (6) and at exit (7).  The
+// split-K kernel uses the same slots: 3 and 4 in the pair's leader only, 5
+// when the first epilogue warp has drained the partial into shared memory,
+// 6 when it has reduced and stored its box (CTAs that store one).
 #ifdef NVFP4_TIMELINE
 constexpr int kGemmTimelineCtas = 1024;
 __device__ unsigned long long g_gemm_timeline[kGemmTimelineCtas][8];
@@ -182,6 +185,8 @@ struct GemmArgs {
   int fault_skip_stage;
   // Row super-tiles per raster group (unit_coords).
   int group_m;
+  // Split-K kernel: CTA pairs per cluster, each taking one range of K.
+  int splits;
 };
 
 // Raster group for a GEMM with this K: with K <= 5120 the whole of A (M x K
@@ -935,6 +940,346 @@ __global__ void __launch_bounds__(C::kThreads, 1)
   if (warp == 1) tmem_dealloc_pair(tmem, kTmemCols);
 }
 
+// ------------------------------------------------- split-K cluster kernel ---
+// For decode-sized M the 256 x 256 pair tiles are too few to occupy the GPU,
+// and 128 x 128 tiles on single CTAs make every SM receive all of A and a W
+// tile for the whole K (the k-loop is bound by the bytes each SM must take
+// in).  Here a cluster of 2S CTAs computes one 256 x 256 tile: its S CTA
+// pairs (ranks 2s and 2s + 1) each run the pair kernel's pipeline over one
+// contiguous range of the k-blocks, so each W byte is still read once and
+// each SM takes in 1/S of the tile's operands.  The S fp32 partial
+// accumulators are then summed across the cluster in distributed shared
+// memory: every CTA drains its 128 x 256 partial from TMEM into its own
+// (now idle) operand ring, and after a cluster barrier the S CTAs holding the
+// same 128 rows each reduce a share of the 32 x 64 output boxes, reading the
+// other partials remotely and adding them in split order (so the result does
+// not depend on which CTA reduces), scale by g_a g_w, round to bf16 and store
+// with TMA.  One tile per cluster; no persistent loop.
+
+// 16-byte chunk j of partial-buffer row `row` (1 KiB rows of 256 fp32): the
+// chunk index is XOR-ed with row % 8 so that both the row-per-lane drain and
+// the row-contiguous reduction touch every bank once per 8 lanes.
+__device__ __forceinline__ uint32_t part_offset(uint32_t row, uint32_t j) {
+  return row * 1024u + ((j ^ (row & 7u)) << 4);
+}
+
+// Load from a shared::cluster address (a CTA's shared memory mapped with mapa).
+__device__ __forceinline__ float4 ld_cluster_f4(uint32_t cluster_addr) {
+  float4 v;
+  asm volatile("ld.shared::cluster.v4.f32 {%0, %1, %2, %3}, [%4];"
+               : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+               : "r"(cluster_addr)
+               : "memory");
+  return v;
+}
+__device__ __forceinline__ void st_shared_v2(uint32_t addr, uint32_t a, uint32_t b) {
+  asm volatile("st.shared.v2.b32 [%0], {%1, %2};" ::"r"(addr), "r"(a), "r"(b) : "memory");
+}
+// The pair-form TMA load of the pair kernel, completing on the barrier at
+// offset `bar` in cluster CTA `lead_rank` (the pair's even rank).
+__device__ __forceinline__ void tma_load_2d_to(void* smem_dst, const void* tmap, uint64_t* bar, int x, int y,
+                                               uint32_t lead_rank) {
+  uint32_t remote;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(smem_u32(bar)), "r"(lead_rank));
+  asm volatile(
+      "cp.async.bulk.tensor.2d.cta_group::2.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%3, %4}], [%2];" ::"r"(smem_u32(smem_dst)),
+      "l"(reinterpret_cast<uint64_t>(tmap)), "r"(remote), "r"(x), "r"(y)
+      : "memory");
+}
+
+// One 32 x 64 output box of the split-K reduction: rows 32q .. 32q + 31 of
+// the CTA's slice, 16-byte column chunk j (lane & 15 picks the chunk, lane >> 4
+// the row of a pair).  The S partials (cluster ranks 2t + half) are read in
+// batches of B row pairs with all S x B loads of a batch in flight, added in
+// split order (the result does not depend on which CTA reduces), scaled,
+// rounded to bf16 and written to the 128-byte-swizzled staging box.
+template <int S, int B>
+__device__ __forceinline__ void reduce_box(uint32_t part0, uint32_t half, int q, uint32_t j, int lane, float scale,
+                                           uint32_t buf) {
+  uint32_t base[S];
+#pragma unroll
+  for (int t = 0; t < S; ++t)
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(base[t]) : "r"(part0), "r"(2u * t + half));
+  const uint32_t cchunk = static_cast<uint32_t>((lane & 15) >> 1);
+#pragma unroll 1
+  for (int b = 0; b < 16 / B; ++b) {
+    float4 v[S][B];
+#pragma unroll
+    for (int t = 0; t < S; ++t)
+#pragma unroll
+      for (int i = 0; i < B; ++i) {
+        const uint32_t rr = static_cast<uint32_t>(2 * (b * B + i) + (lane >> 4));
+        v[t][i] = ld_cluster_f4(base[t] + part_offset(static_cast<uint32_t>(q * 32) + rr, j));
+      }
+#pragma unroll
+    for (int i = 0; i < B; ++i) {
+      float4 acc = v[0][i];
+#pragma unroll
+      for (int t = 1; t < S; ++t) {
+        acc.x += v[t][i].x;
+        acc.y += v[t][i].y;
+        acc.z += v[t][i].z;
+        acc.w += v[t][i].w;
+      }
+      const uint32_t rr = static_cast<uint32_t>(2 * (b * B + i) + (lane >> 4));
+      st_shared_v2(buf + rr * 128 + ((cchunk ^ (rr & 7u)) << 4) + (lane & 1) * 8,
+                   pack_bf16x2(acc.x * scale, acc.y * scale), pack_bf16x2(acc.z * scale, acc.w * scale));
+    }
+  }
+}
+
+template <class C>
+__global__ void __launch_bounds__(C::kThreads, 1)
+    nvfp4_gemm_splitk_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_constant__ CUtensorMap tmap_b,
+                             const __grid_constant__ CUtensorMap tmap_sfa,
+                             const __grid_constant__ CUtensorMap tmap_sfb,
+                             const __grid_constant__ CUtensorMap tmap_out, const GemmArgs args) {
+  constexpr int BN = C::BN;
+  constexpr int kStages = C::kStages;
+  constexpr int kEpi0 = 2 + C::kCopyWarps;
+  static_assert(!C::kRes, "streaming form only");
+  static_assert(C::kEpiWarps == 8, "eight reduction warps");
+  static_assert(128u * 1024u <= kStages * (C::kTileBytesA + C::kTileBytesB), "the partial fits in the ring");
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* sA = smem;
+  uint8_t* sB = sA + kStages * C::kTileBytesA;
+  uint8_t* sEpi = sB + kStages * C::kTileBytesB;
+  uint8_t* sSFA = sEpi + C::kEpiWarps * kEpiBufBytes;
+  uint8_t* sSFB = sSFA + kStages * C::kSfaBytes;
+  uint64_t* full = reinterpret_cast<uint64_t*>(sSFB + kStages * C::kSfbBytes);
+  uint64_t* empty = full + kStages;
+  uint64_t* sfready = empty + kStages;
+  uint64_t* sffull = sfready + kStages;
+  uint64_t* tfull = sffull + kStages;
+  uint64_t* drain = tfull + 1;
+  uint64_t* drain_cp = drain + 1;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain_cp + 1);
+  __shared__ volatile int abort_flag;
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int S = args.splits;
+  const int kblocks = args.K / BK;
+  const int kgroups = args.K / 64;
+  const uint32_t rank = cluster_ctarank();
+  const uint32_t half = rank & 1u, split = rank >> 1, lead = rank & ~1u;
+  const bool leader = half == 0;
+  const int tile = blockIdx.x / (2 * S);
+  const int msup = (args.tiles_m + 1) / 2;
+  int ms, nb;
+  unit_coords(tile, msup, args.tiles_n, args.group_m, &ms, &nb);
+  const int k0 = static_cast<int>(split) * kblocks / S, k1 = (static_cast<int>(split) + 1) * kblocks / S;
+  const int mb = ms * 2 + static_cast<int>(half);  // mb >= tiles_m: a spare CTA, nothing is stored
+  if (threadIdx.x == 0) gemm_stamp(0);
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+      mbar_init(&sfready[s], C::kCopyWarps);
+      mbar_init(&sffull[s], 1);
+    }
+    mbar_init(tfull, 1);
+    mbar_init(drain, 1);
+    mbar_init(drain_cp, C::kCopyWarps);
+    abort_flag = 0;
+    fence_mbar_init();
+    prefetch_tmap(&tmap_a);
+    prefetch_tmap(&tmap_b);
+    prefetch_tmap(&tmap_sfa);
+    prefetch_tmap(&tmap_sfb);
+    prefetch_tmap(&tmap_out);
+  }
+  if (warp == 1) {
+    tmem_alloc_pair(tmem_slot, kTmemCols);
+    tmem_relinquish_pair();
+  }
+  tc_fence_before();
+  cluster_sync_all();
+  tc_fence_after();
+  griddep_wait_and_release();
+  if (threadIdx.x == 0) gemm_stamp(1);
+  const uint32_t tmem = *tmem_slot;
+
+  auto fail = [&]() {
+    set_status(args.status, NVFP4_ERR_TIMEOUT);
+    abort_flag = 1;
+  };
+
+  bool have_partial = false;  // epilogue warps: this CTA's partial is in shared memory
+  if (warp == 0 && lane == 0) {
+    // ------------------------------------------------------ TMA producer ---
+    int stage = 0;
+    uint32_t phase = 0;
+    uint32_t issued_parity[kStages];
+    bool issued[kStages];
+    for (int s = 0; s < kStages; ++s) issued[s] = false;
+    const int a_row = min(mb, args.tiles_m - 1) * BM;  // a spare CTA reloads the last tile
+    const int sfa_row = min(mb, args.tiles_m - 1) * kgroups * 2;
+    const int sfb_row = nb * 2 * kgroups * 2;
+    const int b_row = nb * BN + static_cast<int>(half) * 128;
+    for (int kb = k0; kb < k1; ++kb) {
+      if (!mbar_wait_bounded(&empty[stage], phase ^ 1u, &abort_flag)) { fail(); break; }
+      if (args.fault_skip_stage && tile == 0 && split == 0 && kb == k0) {
+        // Test-only injected fault, as in the pair kernel: the first stage of
+        // the first pair is neither armed nor loaded.
+        if (++stage == kStages) { stage = 0; phase ^= 1u; }
+        continue;
+      }
+      uint8_t* a_dst = sA + stage * C::kTileBytesA;
+      uint8_t* b_dst = sB + stage * C::kTileBytesB;
+      uint8_t* sfa_dst = sSFA + stage * C::kSfaBytes;
+      uint8_t* sfb_dst = sSFB + stage * C::kSfbBytes;
+      const int kx = kb * (BK / 2);
+      if (leader) {
+        // Both CTAs' loads land on the leader's barriers.
+        mbar_arrive_expect_tx(&sffull[stage], 2 * (C::kSfaBytes + C::kSfbBytes));
+        mbar_arrive_expect_tx(&full[stage], 2 * (C::kTileBytesA + C::kTileBytesB));
+        tma_load_2d(sfa_dst, &tmap_sfa, &sffull[stage], 0, sfa_row + kb * 8);
+        tma_load_2d(sfb_dst, &tmap_sfb, &sffull[stage], 0, sfb_row + kb * 8);
+        tma_load_2d(sfb_dst + C::kSfaBytes, &tmap_sfb, &sffull[stage], 0, sfb_row + kgroups * 2 + kb * 8);
+        tma_load_2d(a_dst, &tmap_a, &full[stage], kx, a_row);
+        tma_load_2d(b_dst, &tmap_b, &full[stage], kx, b_row);
+      } else {
+        tma_load_2d_to(sfa_dst, &tmap_sfa, &sffull[stage], 0, sfa_row + kb * 8, lead);
+        tma_load_2d_to(sfb_dst, &tmap_sfb, &sffull[stage], 0, sfb_row + kb * 8, lead);
+        tma_load_2d_to(sfb_dst + C::kSfaBytes, &tmap_sfb, &sffull[stage], 0, sfb_row + kgroups * 2 + kb * 8,
+                       lead);
+        tma_load_2d_to(a_dst, &tmap_a, &full[stage], kx, a_row, lead);
+        tma_load_2d_to(b_dst, &tmap_b, &full[stage], kx, b_row, lead);
+      }
+      if (kb == k0) gemm_stamp(2);
+      issued[stage] = true;
+      issued_parity[stage] = phase;
+      if (++stage == kStages) { stage = 0; phase ^= 1u; }
+    }
+    if (abort_flag && leader) {
+      for (int s = 0; s < kStages; ++s)
+        if (issued[s]) {
+          mbar_wait_bounded(&sffull[s], issued_parity[s], nullptr);
+          mbar_wait_bounded(&full[s], issued_parity[s], nullptr);
+        }
+    }
+  } else if (warp == 1 && lane == 0 && leader) {
+    // ------------------------------------------------ MMA issuer (leader) ---
+    int stage = 0;
+    uint32_t phase = 0;
+    const uint32_t sA0 = smem_u32(sA), sB0 = smem_u32(sB);
+    bool ok = true;
+    for (int kb = k0; kb < k1; ++kb) {
+      if (!mbar_wait_bounded(&full[stage], phase, &abort_flag) ||
+          !mbar_wait_bounded(&sfready[stage], phase, &abort_flag)) { fail(); ok = false; break; }
+      if (kb == k0) gemm_stamp(3);
+      tc_fence_after();
+      const uint32_t sfa_col = tmem + C::kSfTmemCol + stage * C::kSfCols;
+      const uint32_t sfb_col = sfa_col + 16;
+#pragma unroll
+      for (int kk = 0; kk < 4; ++kk)
+        mma_fp4_pair(tmem, desc_sw128(sA0 + stage * C::kTileBytesA + kk * 32),
+                     desc_sw128(sB0 + stage * C::kTileBytesB + kk * 32), C::kIdesc | args.idesc_fmt,
+                     sfa_col + kk * 4, sfb_col + kk * 8, (kb != k0) | (kk != 0));
+      tc_commit_pair(&empty[stage], static_cast<uint16_t>(3u << lead));
+      if (++stage == kStages) { stage = 0; phase ^= 1u; }
+    }
+    if (ok) tc_commit_pair(tfull, static_cast<uint16_t>(3u << lead));
+    gemm_stamp(4);
+    tc_commit_pair(drain, static_cast<uint16_t>(1u << lead));
+    mbar_wait_bounded(drain, 0, nullptr);
+  } else if (warp >= 2 && warp < kEpi0 && lane == 0 && leader) {
+    // ------------------------------------- leader: block scales -> TMEM ---
+    constexpr int kPerWarp = 4 / C::kCopyWarps;
+    const int kk0 = (warp - 2) * kPerWarp;
+    int stage = 0;
+    uint32_t phase = 0;
+    const uint32_t sSFA0 = smem_u32(sSFA), sSFB0 = smem_u32(sSFB);
+    for (int kb = k0; kb < k1; ++kb) {
+      if (!mbar_wait_bounded(&sffull[stage], phase, &abort_flag)) { fail(); break; }
+      tc_fence_after();
+      const uint32_t sfa_col = tmem + C::kSfTmemCol + stage * C::kSfCols;
+      const uint32_t sfb_col = sfa_col + 16;
+#pragma unroll
+      for (int kk = kk0; kk < kk0 + kPerWarp; ++kk) {
+        copy_sf_to_tmem_pair(sfa_col + kk * 4, desc_sf(sSFA0 + stage * C::kSfaBytes + kk * 512));
+#pragma unroll
+        for (int j = 0; j < 2; ++j)
+          copy_sf_to_tmem_pair(sfb_col + kk * 8 + j * 4,
+                               desc_sf(sSFB0 + stage * C::kSfbBytes + j * C::kSfaBytes + kk * 512));
+      }
+      tc_commit_pair(&sfready[stage], static_cast<uint16_t>(1u << lead));
+      if (++stage == kStages) { stage = 0; phase ^= 1u; }
+    }
+    tc_commit_pair(drain_cp, static_cast<uint16_t>(1u << lead));
+    mbar_wait_bounded(drain_cp, 0, nullptr);
+  } else if (warp >= kEpi0) {
+    // ------------------------------- drain the partial into shared memory ---
+    // The last MMA has completed (tfull), so every operand copy has landed
+    // and been read: the ring is free for the partial.
+    const int quarter = warp & 3;
+    const int colbase = ((warp - kEpi0) >> 2) * 128;
+    int ok = 1;
+    if (lane == 0) {
+      ok = !abort_flag && mbar_wait_bounded(tfull, 0, &abort_flag);
+      if (!ok && !abort_flag) fail();
+    }
+    if (__shfl_sync(0xffffffffu, ok, 0)) {
+      tc_fence_after();
+      uint32_t r[128];
+      const uint32_t taddr = tmem + (static_cast<uint32_t>(quarter * 32) << 16) + colbase;
+#pragma unroll
+      for (int c = 0; c < 4; ++c) tmem_ld32(taddr + c * 32, r + 32 * c);
+      tmem_ld_wait();
+      const uint32_t row = static_cast<uint32_t>(quarter * 32 + lane);
+      const uint32_t part0 = smem_u32(smem);
+#pragma unroll
+      for (int c = 0; c < 32; ++c)
+        st_shared_v4(part0 + part_offset(row, static_cast<uint32_t>(colbase / 4 + c)), r[4 * c], r[4 * c + 1],
+                     r[4 * c + 2], r[4 * c + 3]);
+      have_partial = true;
+      if (warp == kEpi0 && lane == 0) gemm_stamp(5);
+    }
+  }
+
+  // Every CTA's partial is written (or its CTA gave up) before any is read.
+  tc_fence_before();
+  cluster_sync_all();
+  tc_fence_after();
+
+  if (warp >= kEpi0 && !abort_flag) {
+    // ------------------------------------------ reduce and store (one box) ---
+    // Box p (0..15) covers rows 32 (p % 4) .. +31 and columns 64 (p / 4) .. +63
+    // of this CTA's 128 x 256 slice; split s reduces boxes s, s + S, ...
+    const int p = static_cast<int>(split) + (warp - kEpi0) * S;
+    const bool all_ok = __all_sync(0xffffffffu, have_partial ? 1 : 0);
+    if (p < 16 && mb < args.tiles_m && all_ok) {
+      const int q = p & 3, pc = p >> 2;
+      const float scale = args.ga ? __fmul_rn(__ldg(args.ga), __ldg(args.gb)) : 1.0f;
+      uint8_t* buf_ptr = sEpi + (warp - kEpi0) * kEpiBufBytes;
+      const uint32_t buf = smem_u32(buf_ptr), part0 = smem_u32(smem);
+      const uint32_t j = static_cast<uint32_t>(pc * 16 + (lane & 15));
+      if (S == 2) reduce_box<2, 8>(part0, half, q, j, lane, scale, buf);
+      else if (S == 3) reduce_box<3, 4>(part0, half, q, j, lane, scale, buf);
+      else reduce_box<4, 4>(part0, half, q, j, lane, scale, buf);
+      fence_proxy_async_smem();
+      __syncwarp();
+      const int x = nb * BN + pc * 64, y = mb * BM + q * 32;
+      if (lane == 0 && x < args.N && y < args.M) {
+        tma_store_2d(&tmap_out, buf_ptr, x, y);
+        bulk_commit_group();
+        bulk_wait_all();
+        if (warp == kEpi0) gemm_stamp(6);
+      }
+    }
+  }
+
+  // No CTA leaves while another may still read its partial.
+  tc_fence_before();
+  cluster_sync_all();
+  tc_fence_after();
+  if (threadIdx.x == 0) gemm_stamp(7);
+  if (warp == 1) tmem_dealloc_pair(tmem, kTmemCols);
+}
+
 // ------------------------------------------------------------------- host ---
 
 PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
@@ -1136,8 +1481,114 @@ nvfp4_status launch_pair(const uint8_t* a_codes, const uint8_t* a_scales, const 
   return launch_status();
 }
 
+using SplitCfg = PairCfg<NVFP4_GEMM_PAIR_STAGES>;
+
+// Clusters of `size` CTAs of the split-K kernel that are resident on the GPU
+// at once (0 if that cluster shape cannot be launched).
+int resident_split_clusters(int size) {
+  static std::mutex mu;
+  static std::map<std::pair<int, int>, int> cache;
+  int d = 0;
+  if (cudaGetDevice(&d) != cudaSuccess) return 0;
+  std::lock_guard<std::mutex> lock(mu);
+  auto it = cache.find({d, size});
+  if (it != cache.end()) return it->second;
+  int clusters = 0;
+  if (cudaFuncSetAttribute(nvfp4_gemm_splitk_kernel<SplitCfg>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           static_cast<int>(SplitCfg::kSmemBytes)) == cudaSuccess) {
+    cudaLaunchConfig_t cfg = {};
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = size;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.gridDim = dim3(size * (sm_count() / size), 1, 1);
+    cfg.blockDim = dim3(SplitCfg::kThreads, 1, 1);
+    cfg.dynamicSmemBytes = SplitCfg::kSmemBytes;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    if (cudaOccupancyMaxActiveClusters(&clusters, nvfp4_gemm_splitk_kernel<SplitCfg>, &cfg) != cudaSuccess)
+      clusters = 0;
+  }
+  cudaGetLastError();
+  cache[{d, size}] = clusters;
+  return clusters;
+}
+
+// Pairs per tile for the split-K kernel: among S = 2..4 with every tile's
+// cluster of 2S CTAs resident at once, the one with the fewest k-blocks per
+// pair (ties: the smaller S, less to reduce); 0 if none.  On GB300 clusters
+// of 4, 6 and 8 CTAs of this kernel fit about 36, 24 and 16 at a time, so the
+// 14B decode qkv (28 tiles) takes S = 2 and the o and down GEMMs (20 tiles)
+// S = 3.  The cross-CTA reduction costs ~3-4 us, which only pays with a long
+// K: measured back to back on GB300, 256 x 7168 x 5120 11.9 -> 11.1 us,
+// 256 x 5120 x 5120 11.8 -> 10.7 us, 256 x 5120 x 13824 24.8 -> 15.2 us, but
+// 16 x 1536 x 1536 (6 k-blocks) 5.7 -> 7.2 us; so K needs 16 k-blocks.
+constexpr int64_t kSplitMinKblocks = 16;
+int choose_splits(int64_t tiles, int64_t kblocks) {
+  if (kblocks < kSplitMinKblocks) return 0;
+  int best = 0;
+  int64_t best_kb = kblocks;
+  for (int S = 2; S <= 4; ++S) {
+    if (kblocks < S || tiles > resident_split_clusters(2 * S)) continue;
+    const int64_t kb = (kblocks + S - 1) / S;
+    if (kb < best_kb) { best = S; best_kb = kb; }
+  }
+  return best;
+}
+
+nvfp4_status launch_splitk(const uint8_t* a_codes, const uint8_t* a_scales, const float* g_a, const uint8_t* w_codes,
+                           const uint8_t* w_scales, const float* g_w, int64_t M, int64_t N, int64_t K, void* out_bf16,
+                           int64_t ldo, cudaStream_t stream, uint32_t idesc_fmt, int splits) {
+  using C = SplitCfg;
+  const int64_t tiles_m = (M + BM - 1) / BM, tiles_n = N / C::BN;
+  const int64_t tiles = ((tiles_m + 1) / 2) * tiles_n;
+  if (tiles * 2 * splits >= (1ll << 31)) return NVFP4_ERR_SHAPE;
+  CUtensorMap ma, mb, msa, msb, mo;
+  if (!make_code_map(&ma, a_codes, M, K, BM) || !make_code_map(&mb, w_codes, N, K, 128) ||
+      !make_scale_map(&msa, a_scales, M, K) || !make_scale_map(&msb, w_scales, N, K) ||
+      !make_out_map(&mo, out_bf16, M, N, ldo))
+    return NVFP4_ERR_CUDA;
+  GemmArgs args = {};
+  args.idesc_fmt = idesc_fmt;
+  args.sfa = a_scales;
+  args.sfb = w_scales;
+  args.ga = g_a;
+  args.gb = g_w;
+  args.M = static_cast<int>(M);
+  args.N = static_cast<int>(N);
+  args.K = static_cast<int>(K);
+  args.tiles_m = static_cast<int>(tiles_m);
+  args.tiles_n = static_cast<int>(tiles_n);
+  args.group_m = raster_group(K, tiles / tiles_n);
+  args.splits = splits;
+  args.status = status_word_dev();
+  args.fault_skip_stage = take_fault(NVFP4_FAULT_GEMM_SKIP_STAGE) ? 1 : 0;
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr[2];
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2 * splits;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.gridDim = dim3(static_cast<unsigned>(tiles * 2 * splits), 1, 1);
+  cfg.blockDim = dim3(C::kThreads, 1, 1);
+  cfg.dynamicSmemBytes = C::kSmemBytes;
+  cfg.stream = stream;
+  cfg.attrs = attr;
+  cfg.numAttrs = 2;
+  if (cudaLaunchKernelEx(&cfg, nvfp4_gemm_splitk_kernel<C>, ma, mb, msa, msb, mo, args) != cudaSuccess)
+    return NVFP4_ERR_CUDA;
+  count_launches(1);
+  return launch_status();
+}
+
 #ifndef NVFP4_GEMM_BN
 #define NVFP4_GEMM_BN 0  // 0: choose per shape
+#endif
+#ifndef NVFP4_GEMM_SPLITK
+#define NVFP4_GEMM_SPLITK 1  // 0: never use the split-K kernel
 #endif
 #ifndef NVFP4_GEMM_PAIR
 #define NVFP4_GEMM_PAIR 1  // 0: never use the CTA-pair kernel
@@ -1173,8 +1624,9 @@ nvfp4_status linear_dispatch(const uint8_t* a_codes, const uint8_t* a_scales, co
                              int64_t K, void* out_bf16, int64_t ldo, cudaStream_t s, uint32_t idesc_fmt) {
   const int64_t tiles_m = (M + BM - 1) / BM;
   // The CTA pair, unless its 256 x 256 tiles would leave most pairs idle
-  // (decode-sized M): then 128 x 128 tiles on single CTAs spread the W stream
-  // over more SMs (measured faster at M = 256 with N = 5120 or 7168, slower
+  // (decode-sized M): then, with a long K, the split-K clusters, else 128 x
+  // 128 tiles on single CTAs, which spread the W stream over more SMs than
+  // the pairs would (measured faster at M = 256 with N = 5120 or 7168, slower
   // with N = 27648).
   using Pair = PairCfg<NVFP4_GEMM_PAIR_STAGES>;
   if (NVFP4_GEMM_PAIR && N % 256 == 0 && tiles_m >= 2) {
@@ -1185,6 +1637,13 @@ nvfp4_status linear_dispatch(const uint8_t* a_codes, const uint8_t* a_scales, co
     if (2 * pair_units >= resident_pairs<Pair, false>())
       return launch_pair<Pair>(a_codes, a_scales, g_a, w_codes, w_scales, g_w, M, N, K, out_bf16, ldo, s, nullptr,
                                idesc_fmt);
+  }
+  // Too few pair tiles for the GPU: split K across clusters of CTA pairs.
+  if (NVFP4_GEMM_SPLITK && N % 256 == 0) {
+    const int splits = choose_splits(((tiles_m + 1) / 2) * (N / 256), K / BK);
+    if (splits)
+      return launch_splitk(a_codes, a_scales, g_a, w_codes, w_scales, g_w, M, N, K, out_bf16, ldo, s, idesc_fmt,
+                           splits);
   }
   // Single CTAs: BN = 128 (measured faster than 256 at M <= 256 on GB300).
   const int bn = NVFP4_GEMM_BN ? NVFP4_GEMM_BN : 128;

@@ -47,8 +47,14 @@ def run_linear(N, a_codes, a_scales_rm, g_a, w_codes, w_scales_rm, g_w, M, Nn, K
 
 @pytest.mark.parametrize("M,Nn,K", [(128, 128, 256), (1, 16, 256), (16, 128, 512), (130, 144, 512),
                                     (257, 384, 1024), (300, 272, 2304), (128, 1024, 256),
-                                    # N % 256 == 0 with few 256 x 256 tiles: single CTAs
+                                    # N % 256 == 0 with too few 256 x 256 tiles for the pairs and a short
+                                    # K: single CTAs
                                     (256, 256, 512), (300, 512, 1024), (640, 768, 768), (129, 1280, 2048),
+                                    (16, 1536, 1536), (256, 5120, 3584),
+                                    # ... and with K >= 4096: split-K clusters of 2, 3 or 4 pairs, even
+                                    # and uneven K ranges, M tails, a spare CTA per pair when M <= 128
+                                    (256, 512, 4096), (16, 1536, 4608), (1, 256, 4096), (300, 768, 5120),
+                                    (100, 512, 6400), (256, 7168, 4096), (256, 5120, 4352),
                                     # CTA-pair path (enough 256 x 256 tiles to occupy the pairs):
                                     # M tails with a spare CTA, odd super-tile counts, one-row tail
                                     (256, 10240, 512), (300, 10240, 1024), (640, 5120, 768), (129, 12800, 256),
@@ -157,6 +163,41 @@ def test_injected_missing_stage_times_out_and_next_call_is_exact(N):
     import time
     M, Nn, K = 640, 10240, 2048  # a CTA-pair shape with more tiles than resident pairs
     gen = torch.Generator().manual_seed(31)
+    a_c, a_s = random_operand(M, K, gen)
+    w_c, w_s = random_operand(Nn, K, gen)
+    dev = "cuda"
+    args = (torch.from_numpy(a_c).to(dev), torch.from_numpy(O.scales_to_mma(a_s)).to(dev),
+            torch.ones(1, device=dev), torch.from_numpy(w_c).to(dev),
+            torch.from_numpy(O.scales_to_mma(w_s)).to(dev), torch.ones(1, device=dev))
+    out = torch.full((M, Nn), float("nan"), dtype=torch.bfloat16, device=dev)
+    torch.cuda.synchronize()
+    assert N.nvfp4_get_device_status() == 0
+    N.nvfp4_debug_inject_fault(N.FAULT_GEMM_SKIP_STAGE)
+    try:
+        t0 = time.time()
+        N.nvfp4_linear(*args, out, M, Nn, K)
+        torch.cuda.synchronize()
+        waited = time.time() - t0
+    finally:
+        N.nvfp4_debug_inject_fault(N.FAULT_NONE)
+    assert N.nvfp4_get_device_status() == 6
+    assert 1.0 < waited < 20.0, f"bounded wait expected (~2-4 s), took {waited:.1f} s"
+    out.fill_(float("nan"))
+    N.nvfp4_linear(*args, out, M, Nn, K)
+    torch.cuda.synchronize()
+    assert N.nvfp4_get_device_status() == 0
+    assert_close(f32(out), O.linear(a_c, a_s, 1.0, w_c, w_s, 1.0), what="after the injected timeout")
+
+
+def test_injected_missing_stage_in_split_k_cluster_times_out(N):
+    """The same fault in the split-K cluster kernel (a decode-sized shape with
+    three CTA pairs per tile): the first pair of the first cluster leaves its
+    first stage unissued; the other pairs of that cluster finish and wait at
+    the cluster barrier, the faulted pair's bounded waits run out, the call
+    reports NVFP4_ERR_TIMEOUT and the next call is exact."""
+    import time
+    M, Nn, K = 256, 5120, 4352
+    gen = torch.Generator().manual_seed(37)
     a_c, a_s = random_operand(M, K, gen)
     w_c, w_s = random_operand(Nn, K, gen)
     dev = "cuda"
