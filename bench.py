@@ -48,11 +48,11 @@ CSRC = os.path.join(ROOT, "paper_2606_15682_gb300", "csrc")
 # same kernel and shape (commands in profiles/).  Each entry holds only while the kernel sources
 # hash to the value they had at capture time; otherwise the line reports traffic = null.
 NCU_TRAFFIC = {
-    "gemm": {"bytes": 661180000 + 863110000, "sources": ("gemm.cu", "common.cuh"), "sha": "283b225788dd4181",
+    "gemm": {"bytes": 207516672 + 862637568, "sources": ("gemm.cu", "common.cuh"), "sha": "43fb355ab491de1b",
              "shape": (8192, 55296, 5120),
              "profile": "profiles/gemm_qwen32b_prefill_gate_up_m8192_n55296_k5120.md"},
-    "attention": {"bytes": 1208783616 + 22233856, "sources": ("attention.cu", "common.cuh"),
-                  "sha": "b4d25eaf23259ae3", "shape": (64, 16384),
+    "attention": {"bytes": 1208723200 + 22190592, "sources": ("attention.cu", "common.cuh"),
+                  "sha": "9e8c99fa4fbebd08", "shape": (64, 16384),
                   "profile": "profiles/attention_qwen14b_decode_b64_t16384.md (attn_partial_kernel)"},
 }
 
