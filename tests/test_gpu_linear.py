@@ -104,11 +104,14 @@ def test_single_block_structure(N):
     assert_close(f32(out), ref)
 
 
-def test_deterministic(N):
-    M, Nn, K = 256, 256, 1024
+@pytest.mark.parametrize("M,Nn,K", [(256, 256, 1024),    # single CTAs
+                                    (256, 5120, 4352)])  # split-K clusters: partials summed in split order
+def test_deterministic(N, M, Nn, K):
     gen = torch.Generator().manual_seed(11)
-    a_c, a_s = random_operand(M, K, gen)
-    w_c, w_s = random_operand(Nn, K, gen)
+    # Wide scale range: partial sums that round in fp32, so a change of
+    # summation order would show.
+    a_c, a_s = random_operand(M, K, gen, 0x20, 0x58)
+    w_c, w_s = random_operand(Nn, K, gen, 0x20, 0x58)
     o1 = run_linear(N, a_c, a_s, 1.0, w_c, w_s, 1.0, M, Nn, K)
     o2 = run_linear(N, a_c, a_s, 1.0, w_c, w_s, 1.0, M, Nn, K)
     assert torch.equal(o1, o2)

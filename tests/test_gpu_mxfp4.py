@@ -128,7 +128,9 @@ def run_mx_linear(N, a_codes, a_scales_rm, w_codes, w_scales_rm, M, Nn, K, ldo=N
                                     # N % 256 == 0: 256 x 256 CTA-pair tiles (enough of them)
                                     (2048, 1280, 1024),
                                     # more pair tiles than pairs with 6 k-blocks: the W-resident form
-                                    (2048, 2560, 1536)])
+                                    (2048, 2560, 1536),
+                                    # too few pair tiles with a long K: split-K clusters (S = 4, 2)
+                                    (256, 768, 4096), (200, 7168, 4608)])
 def test_mx_linear_random_operands(N, M, Nn, K):
     """Seeded random codes and E8M0 scales (isolates the GEMM from the quantizer)."""
     gen = torch.Generator().manual_seed(7400 + M + Nn + K)
