@@ -75,8 +75,10 @@ def test_random_codes(N, M, Nn, K):
     assert_close(f32(out), ref, what=f"{M}x{Nn}x{K}")
 
 
-def test_ldo_padding_untouched(N):
-    M, Nn, K, ldo = 200, 160, 512, 200
+@pytest.mark.parametrize("M,Nn,K,ldo", [(200, 160, 512, 200),     # single CTAs
+                                        (200, 512, 4096, 520),    # split-K clusters
+                                        (640, 10240, 1024, 10248)])  # CTA pairs
+def test_ldo_padding_untouched(N, M, Nn, K, ldo):
     gen = torch.Generator().manual_seed(5)
     a_c, a_s = random_operand(M, K, gen)
     w_c, w_s = random_operand(Nn, K, gen)
