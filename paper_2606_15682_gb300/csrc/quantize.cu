@@ -349,18 +349,22 @@ __global__ void __launch_bounds__(kThreads) quantize_dynamic_kernel(
   if (bidx_last < total_blocks)
     quantize_loaded<kMMA>(sl, total_blocks, kblocks_div.d, bidx_last, stride, lane, g, six_g, true, codes, scales,
                           status);
-  it = 0;
-  for (uint32_t bidx0 = bidx_first; bidx0 < bidx_last; bidx0 += stride * kUnroll, ++it) {
+  // The iterations between the stashed ones and the last are read from x
+  // again, most recent first: when x does not fit in L2, phase 1 left the
+  // latest of them in L2.  The stashed ones come from shared memory.
+  const int n_iter = it;
+  for (int k = n_iter - 2; k >= 0; --k) {
+    const uint32_t bidx0 = bidx_first + static_cast<uint32_t>(k) * stride * kUnroll;
     BlockSlots t;
-    if (it < stash_iters) {
+    if (k < stash_iters) {
       const uint32_t kblocks = kblocks_div.d;
 #pragma unroll
       for (int u = 0; u < kUnroll; ++u) {
         const uint32_t b = bidx0 + u * stride + lane;
         t.row[u] = kblocks_div.div(b);
         t.kb[u] = b - t.row[u] * kblocks;
-        t.v0[u] = stash[((it * kUnroll + u) * 2) * kThreads + threadIdx.x];
-        t.v1[u] = stash[((it * kUnroll + u) * 2 + 1) * kThreads + threadIdx.x];
+        t.v0[u] = stash[((k * kUnroll + u) * 2) * kThreads + threadIdx.x];
+        t.v1[u] = stash[((k * kUnroll + u) * 2 + 1) * kThreads + threadIdx.x];
       }
     } else {
       load_blocks(x, kblocks_div, total_blocks, ld, dense, bidx0, stride, lane, t);
