@@ -51,8 +51,8 @@ NCU_TRAFFIC = {
     "gemm": {"bytes": 205137408 + 862096896, "sources": ("gemm.cu", "common.cuh"), "sha": "16b5f730c8ca69b4",
              "shape": (8192, 55296, 5120),
              "profile": "profiles/gemm_qwen32b_prefill_gate_up_m8192_n55296_k5120.md"},
-    "attention": {"bytes": 1208723200 + 22190592, "sources": ("attention.cu", "common.cuh"),
-                  "sha": "9e8c99fa4fbebd08", "shape": (64, 16384),
+    "attention": {"bytes": 1208885248 + 22256640, "sources": ("attention.cu", "common.cuh"),
+                  "sha": "76e8785bf56696d1", "shape": (64, 16384),
                   "profile": "profiles/attention_qwen14b_decode_b64_t16384.md (attn_partial_kernel)"},
 }
 

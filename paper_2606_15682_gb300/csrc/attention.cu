@@ -315,7 +315,11 @@ __global__ void __launch_bounds__(kThreads, NVFP4_ATTN_MIN_CTAS) attn_partial_ke
       }
       if (!__shfl_sync(0xffffffffu, ok, 0)) return;
       const uint8_t* st = ring + stage * kStageBytes;
-#pragma unroll 1
+      // The warp's two tiles of the stage, unrolled: the second tile's loads,
+      // decode and score MMAs interleave with the first tile's softmax and
+      // value MMAs (same 96 registers, same 4 CTAs per SM): B=64, T=16384
+      // 248.4 -> 241.3 us, bit-identical.
+#pragma unroll
       for (int sub = 0; sub < kStageTok / (16 * kConsumers); ++sub) {
       const int r0 = 16 * (cw + kConsumers * sub);  // this warp's tile within the stage
       const int tile = t0 + r0;
