@@ -145,14 +145,16 @@ __device__ __forceinline__ uint4 ld_shared_v4(uint32_t addr) {
 // Write one staged 32 x 64 bf16 box (rows of 128 B whose 16-byte chunks sit at
 // chunk ^ (row % 8)) to out[y.., x..] with coalesced 16-byte stores: per
 // instruction the warp writes 4 rows x 128 B; rows at or past M are skipped.
-__device__ __forceinline__ void store_box_lsu(uint32_t buf, uint16_t* out, int64_t ldo, int x, int y, int M,
-                                              int lane) {
+// (In the bounds-checked build each store is also checked against [M, N].)
+__device__ __forceinline__ void store_box_lsu(uint32_t buf, uint16_t* out, int64_t ldo, int x, int y, int M, int N,
+                                              int lane, int* status) {
   const int cc = lane & 7;
 #pragma unroll
   for (int it = 0; it < 8; ++it) {
     const int rr = 4 * it + (lane >> 3);
     const uint4 v = ld_shared_v4(buf + rr * 128 + ((cc ^ (rr & 7)) << 4));
-    if (y + rr < M) *reinterpret_cast<uint4*>(out + static_cast<int64_t>(y + rr) * ldo + x + cc * 8) = v;
+    if (y + rr < M && in_bounds(status, x + cc * 8 + 8 <= N))
+      *reinterpret_cast<uint4*>(out + static_cast<int64_t>(y + rr) * ldo + x + cc * 8) = v;
   }
 }
 
@@ -957,7 +959,7 @@ __global__ void __launch_bounds__(C::kThreads, 1)
         const int x = nb * BN + colbase + h * kEpiCols, y = mb * BM + quarter * 32;
         if (NVFP4_GEMM_LSU_STORE) {
           __syncwarp();
-          if (x < args.N && y < args.M) store_box_lsu(buf, args.out, args.ldo, x, y, args.M, lane);
+          if (x < args.N && y < args.M) store_box_lsu(buf, args.out, args.ldo, x, y, args.M, args.N, lane, args.status);
           __syncwarp();  // the next box overwrites the staging buffer
         } else {
           fence_proxy_async_smem();
