@@ -88,8 +88,15 @@ _mx_linear = _sig("mxfp4_linear", [_p, _p, _p, _p, _i64, _i64, _i64, _p, _i64, _
 _mx_linear_swiglu = _sig("mxfp4_linear_swiglu_quantize", [_p, _p, _p, _p, _i64, _i64, _i64, ctypes.c_int, _p, _p, _p])
 
 
+# The current stream's raw handle without building a torch.cuda.Stream object
+# (0.1 us instead of ~3 us per call); the public call where it is absent.
+_raw_current_stream = getattr(torch._C, "_cuda_getCurrentRawStream", None)
+
+
 def _stream(stream):
     if stream is None:
+        if _raw_current_stream is not None:
+            return ctypes.c_void_p(_raw_current_stream(torch.cuda.current_device()))
         stream = torch.cuda.current_stream()
     return ctypes.c_void_p(stream.cuda_stream if hasattr(stream, "cuda_stream") else int(stream))
 
