@@ -478,6 +478,20 @@ def run_ours(args, rank, world):
     seq = torch.arange(Bq, dtype=torch.int32, device=dev).repeat_interleave(T)
     pos = torch.arange(T, dtype=torch.int32, device=dev).repeat(Bq)
     N.kv_append_nvfp4(cache, K_all.view(-1, hkv, 128), V_all.view(-1, hkv, 128), seq, pos)
+    # The cache fill itself (a4 at prefill size: every token of every sequence,
+    # K and V quantized and written), timed as a single launch after an L2 flush.
+    fill_ms = []
+    with torch.cuda.stream(stream):
+        for _ in range(3):
+            flush_buf.zero_()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
+            N.kv_append_nvfp4(cache, K_all.view(-1, hkv, 128), V_all.view(-1, hkv, 128), seq, pos)
+            e1.record()
+            stream.synchronize()
+            fill_ms.append(e0.elapsed_time(e1))
+    fill_bytes = Bq * T * hkv * 2 * (256 + 72)  # bf16 K and V rows in; codes and scales out
+    fill_gbs = fill_bytes / (statistics.median(fill_ms) * 1e-3) / 1e9
     del K_all, V_all, seq, pos
     cache.seq_lens.fill_(T)
     q = rec.queries(Bq, hq, seed=synth.seed_for(ATTN_WL, "q") % (1 << 62))
@@ -577,6 +591,9 @@ def run_ours(args, rank, world):
                          "frac": attn_gbs / peaks["hbm_gbs"], "traffic": ncu_traffic("attention", (Bq, T)),
                          "kernel": "attn_partial_kernel + attn_combine_kernel (one decode_attention_nvfp4 call)"},
             "gpu_launches": attn_launches * args.steps,
+            "kv_fill": {"step": "kv_append_nvfp4 of the whole cache (B x T tokens, H_kv heads, K and V)",
+                        "tokens": Bq * T, "us": 1e3 * statistics.median(fill_ms), "algorithmic_bytes": fill_bytes,
+                        "gbs": fill_gbs, "frac": fill_gbs / peaks["hbm_gbs"]},
         },
         "attention_gbs": world * attn_gbs,
         "attention_frac": attn_gbs / peaks["hbm_gbs"],

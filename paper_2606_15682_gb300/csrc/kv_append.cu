@@ -2,9 +2,9 @@
 // m, Eq. 2) and write them into the NVFP4 KV cache; optionally rotate K by
 // RoPE first (the fused RoPE -> shift -> quantize -> append step).
 //
-// Work item = one 8-element chunk of one 128-channel row; the 16 lanes that
-// hold a row cover its 8 blocks.  Item order (token, kv head, K|V, chunk) keeps
-// each warp's 512-byte bf16 read contiguous in the [n_new, H_kv, 128] inputs.
+// Work item = one 16-element block of one 128-channel row (one thread per
+// block: the block scale is computed once).  Item order (token, kv head, K|V,
+// block) keeps each warp's reads contiguous in the [n_new, H_kv, 128] inputs.
 #include <cfloat>
 
 #include "common.cuh"
@@ -14,10 +14,17 @@ namespace nvfp4 {
 namespace {
 
 constexpr int kThreads = 256;
+constexpr int kUnroll = 4;  // items (16-element blocks) per thread per pass
 
 // kRope: K arrives before RoPE and is rotated here (rotate-half pairing,
 // channel i with i + 64) with the (cos, sin) table row of its position, in
 // fp32: y_i = x_i c_i - x_{i+64} s_i, y_{i+64} = x_i s_i + x_{i+64} c_i.
+//
+// Work item = one 16-element block of one row (row = token, KV head, K or V):
+// 16 items per (token, head), so a warp covers two.  Lane l of a warp takes
+// (token-head 2w + l/16, K or V by bit 3, block l % 8); the RoPE partner block
+// (channels 64 apart) is on lane l ^ 4.  kUnroll items per thread per pass,
+// all their loads issued first.
 template <bool kRope, bool kE1M2>
 __global__ void __launch_bounds__(kThreads) kv_append_kernel(
     const uint16_t* __restrict__ k_in, const uint16_t* __restrict__ v_in, const int32_t* __restrict__ seq_idx,
@@ -25,72 +32,100 @@ __global__ void __launch_bounds__(kThreads) kv_append_kernel(
     uint32_t n_rows /* n_new*H_kv */, FastDiv hkv, uint32_t batch, uint32_t capacity, uint8_t* __restrict__ kc,
     uint8_t* __restrict__ ks, uint8_t* __restrict__ vc, uint8_t* __restrict__ vs, float gk, float gv, int* status) {
   griddep_wait_and_release();
-  const uint32_t total = n_rows * 32u;  // 2 tensors x 16 chunks per row: a multiple of the warp
+  const uint32_t total = n_rows * 16u;  // 2 tensors x 8 blocks per row: a multiple of the warp
   const uint32_t lane = threadIdx.x & 31;
   const float qmax = kE1M2 ? 3.5f : 6.0f;  // largest element magnitude of the grid
   const float six_gk = __fmul_rn(qmax, gk), six_gv = __fmul_rn(qmax, gv);
-  for (uint32_t c0 = blockIdx.x * blockDim.x + (threadIdx.x & ~31u); c0 < total; c0 += gridDim.x * blockDim.x) {
-    const uint32_t c = c0 + lane;
-    const bool live = c < total;
-    const uint32_t j = c & 15u;          // chunk within the 128-channel row
-    const bool is_v = (c >> 4) & 1u;
-    const uint32_t rr = c >> 5;          // token * H_kv + head
-    const uint32_t tok = hkv.div(rr);
-    const uint32_t h = rr - tok * hkv.d;
-    uint4 raw = make_uint4(0, 0, 0, 0);
-    if (live) raw = __ldg(reinterpret_cast<const uint4*>((is_v ? v_in : k_in) + static_cast<uint64_t>(rr) * 128 + j * 8));
-    float x[8];
-    unpack_bf16x8(raw, x);
-    if (kRope) {
-      // The partner chunk (channels 64 apart) is held by lane ^ 8; the whole warp is live.
-      uint4 pr;
-      pr.x = __shfl_xor_sync(0xffffffffu, raw.x, 8);
-      pr.y = __shfl_xor_sync(0xffffffffu, raw.y, 8);
-      pr.z = __shfl_xor_sync(0xffffffffu, raw.z, 8);
-      pr.w = __shfl_xor_sync(0xffffffffu, raw.w, 8);
-      if (live && !is_v) {
-        float xp[8];
-        unpack_bf16x8(pr, xp);
-        int32_t p = __ldg(pos + tok);
-        if (p < 0 || static_cast<uint32_t>(p) >= capacity) p = 0;  // reported as CAPACITY below
-        const float4* cs = reinterpret_cast<const float4*>(rope + (static_cast<uint64_t>(p) * 64 + (j & 7u) * 8) * 2);
-        float cv[8], sv[8];
+  const uint32_t stride = gridDim.x * blockDim.x;
+  // Item indices are formed in 64 bits: a pass may reach past 2^32 near the end.
+  for (uint64_t c00 = blockIdx.x * blockDim.x + (threadIdx.x & ~31u); c00 < total;
+       c00 += static_cast<uint64_t>(stride) * kUnroll) {
+    uint4 lo[kUnroll], hi[kUnroll];
+#pragma unroll
+    for (int u = 0; u < kUnroll; ++u) {
+      const uint64_t c = c00 + static_cast<uint64_t>(u) * stride + lane;
+      const uint32_t rr = static_cast<uint32_t>(c >> 4);
+      const bool is_v = (c >> 3) & 1u;
+      const uint4* src = reinterpret_cast<const uint4*>((is_v ? v_in : k_in) + static_cast<uint64_t>(rr) * 128 +
+                                                        (c & 7u) * 16);
+      const bool in = c < total;
+      lo[u] = in ? __ldg(src) : make_uint4(0, 0, 0, 0);
+      hi[u] = in ? __ldg(src + 1) : make_uint4(0, 0, 0, 0);
+    }
+#pragma unroll
+    for (int u = 0; u < kUnroll; ++u) {
+      const uint64_t c0 = c00 + static_cast<uint64_t>(u) * stride;
+      if (c0 >= total) continue;  // warp-uniform: c0 is the warp's first item
+      const uint32_t c = static_cast<uint32_t>(c0) + lane;  // c0 < total < 2^32
+      const bool live = c < total;         // an odd row count leaves half of the last warp idle
+      const uint32_t blk = c & 7u;         // block within the 128-channel row
+      const bool is_v = (c >> 3) & 1u;
+      const uint32_t rr = c >> 4;          // token * H_kv + head
+      const uint32_t tok = hkv.div(rr);
+      const uint32_t h = rr - tok * hkv.d;
+      float x[16];
+      unpack_bf16x8(lo[u], x);
+      unpack_bf16x8(hi[u], x + 8);
+      if (kRope) {
+        // The partner block (channels 64 apart) is on lane ^ 4; every lane of the warp is live.
+        uint4 plo, phi;
+        plo.x = __shfl_xor_sync(0xffffffffu, lo[u].x, 4);
+        plo.y = __shfl_xor_sync(0xffffffffu, lo[u].y, 4);
+        plo.z = __shfl_xor_sync(0xffffffffu, lo[u].z, 4);
+        plo.w = __shfl_xor_sync(0xffffffffu, lo[u].w, 4);
+        phi.x = __shfl_xor_sync(0xffffffffu, hi[u].x, 4);
+        phi.y = __shfl_xor_sync(0xffffffffu, hi[u].y, 4);
+        phi.z = __shfl_xor_sync(0xffffffffu, hi[u].z, 4);
+        phi.w = __shfl_xor_sync(0xffffffffu, hi[u].w, 4);
+        if (live && !is_v) {
+          float xp[16];
+          unpack_bf16x8(plo, xp);
+          unpack_bf16x8(phi, xp + 8);
+          int32_t p = __ldg(pos + tok);
+          if (p < 0 || static_cast<uint32_t>(p) >= capacity) p = 0;  // reported as CAPACITY below
+          const float4* cs =
+              reinterpret_cast<const float4*>(rope + (static_cast<uint64_t>(p) * 64 + (blk & 3u) * 16) * 2);
+#pragma unroll
+          for (int q = 0; q < 8; ++q) {
+            const float4 t = __ldg(cs + q);
+            const float cv0 = t.x, sv0 = t.y, cv1 = t.z, sv1 = t.w;
+            const int e = 2 * q;
+            x[e] = blk < 4 ? __fsub_rn(__fmul_rn(x[e], cv0), __fmul_rn(xp[e], sv0))
+                           : __fadd_rn(__fmul_rn(xp[e], sv0), __fmul_rn(x[e], cv0));
+            x[e + 1] = blk < 4 ? __fsub_rn(__fmul_rn(x[e + 1], cv1), __fmul_rn(xp[e + 1], sv1))
+                               : __fadd_rn(__fmul_rn(xp[e + 1], sv1), __fmul_rn(x[e + 1], cv1));
+          }
+        }
+      }
+      if (live && !is_v && k_shift) {
+        const float4* m4 = reinterpret_cast<const float4*>(k_shift + h * 128u + blk * 16u);
 #pragma unroll
         for (int q = 0; q < 4; ++q) {
-          const float4 t = __ldg(cs + q);
-          cv[2 * q] = t.x; sv[2 * q] = t.y; cv[2 * q + 1] = t.z; sv[2 * q + 1] = t.w;
+          const float4 m = __ldg(m4 + q);
+          x[4 * q] = __fsub_rn(x[4 * q], m.x);
+          x[4 * q + 1] = __fsub_rn(x[4 * q + 1], m.y);
+          x[4 * q + 2] = __fsub_rn(x[4 * q + 2], m.z);
+          x[4 * q + 3] = __fsub_rn(x[4 * q + 3], m.w);
         }
-#pragma unroll
-        for (int e = 0; e < 8; ++e)
-          x[e] = j < 8 ? __fsub_rn(__fmul_rn(x[e], cv[e]), __fmul_rn(xp[e], sv[e]))
-                       : __fadd_rn(__fmul_rn(xp[e], sv[e]), __fmul_rn(x[e], cv[e]));
       }
-    }
-    if (live && !is_v && k_shift) {
-      const float4* m4 = reinterpret_cast<const float4*>(k_shift + h * 128u + j * 8u);
-      const float4 m0 = __ldg(m4), m1 = __ldg(m4 + 1);
-      x[0] = __fsub_rn(x[0], m0.x); x[1] = __fsub_rn(x[1], m0.y);
-      x[2] = __fsub_rn(x[2], m0.z); x[3] = __fsub_rn(x[3], m0.w);
-      x[4] = __fsub_rn(x[4], m1.x); x[5] = __fsub_rn(x[5], m1.y);
-      x[6] = __fsub_rn(x[6], m1.z); x[7] = __fsub_rn(x[7], m1.w);
-    }
-    float amax = 0.0f;
+      float amax = 0.0f;
 #pragma unroll
-    for (int i = 0; i < 8; ++i) amax = fmaxf(amax, fabsf(x[i]));
-    uint32_t sc;
-    const uint32_t packed = quantize8_pair<kE1M2>(x, amax, is_v ? gv : gk, is_v ? six_gv : six_gk, &sc);
-    if (!live) continue;
-    const int32_t b = __ldg(seq_idx + tok), p = __ldg(pos + tok);
-    if (b < 0 || static_cast<uint32_t>(b) >= batch || p < 0 || static_cast<uint32_t>(p) >= capacity) {
-      if (j == 0 && !is_v) set_status(status, NVFP4_ERR_CAPACITY);
-      continue;
+      for (int i = 0; i < 16; ++i) amax = fmaxf(amax, fabsf(x[i]));
+      const BlockScale bs = block_scale(amax, is_v ? gv : gk, is_v ? six_gv : six_gk);
+#pragma unroll
+      for (int i = 0; i < 16; ++i) x[i] = __fmul_rn(x[i], bs.mult);
+      const uint2 packed = kE1M2 ? make_uint2(e1m2x8(x), e1m2x8(x + 8)) : make_uint2(e2m1x8(x), e2m1x8(x + 8));
+      if (!live) continue;
+      const int32_t b = __ldg(seq_idx + tok), p = __ldg(pos + tok);
+      if (b < 0 || static_cast<uint32_t>(b) >= batch || p < 0 || static_cast<uint32_t>(p) >= capacity) {
+        if (blk == 0 && !is_v) set_status(status, NVFP4_ERR_CAPACITY);
+        continue;
+      }
+      const uint64_t row = (static_cast<uint64_t>(b) * hkv.d + h) * capacity + static_cast<uint32_t>(p);
+      if (!in_bounds(status, row < static_cast<uint64_t>(batch) * hkv.d * capacity && blk < 8u)) continue;
+      reinterpret_cast<uint2*>((is_v ? vc : kc) + row * 64)[blk] = packed;
+      (is_v ? vs : ks)[row * 8 + blk] = static_cast<uint8_t>(bs.code);
     }
-    const uint64_t row = (static_cast<uint64_t>(b) * hkv.d + h) * capacity + static_cast<uint32_t>(p);
-    if (!in_bounds(status, row < static_cast<uint64_t>(batch) * hkv.d * capacity && j < 16u)) continue;
-    uint8_t* codes = is_v ? vc : kc;
-    uint8_t* scales = is_v ? vs : ks;
-    reinterpret_cast<uint32_t*>(codes + row * 64)[j] = packed;
-    if ((j & 1u) == 0) scales[row * 8 + (j >> 1)] = static_cast<uint8_t>(sc);
   }
 }
 
@@ -110,8 +145,8 @@ nvfp4_status append(const nvfp4_kv_cache* cache, const void* k_bf16, const void*
     return NVFP4_ERR_ALIGN;
   if (n_new == 0) return NVFP4_OK;
   const uint32_t n_rows = static_cast<uint32_t>(n_new * cache->num_kv_heads);
-  const uint64_t items = static_cast<uint64_t>(n_rows) * 32;
-  uint64_t grid = (items + kThreads - 1) / kThreads;
+  const uint64_t items = static_cast<uint64_t>(n_rows) * 16;
+  uint64_t grid = (items + kThreads * kUnroll - 1) / (kThreads * kUnroll);
   const uint64_t cap = static_cast<uint64_t>(sm_count()) * 8;
   if (grid > cap) grid = cap;
   const bool e1m2 = cache->kv_format == NVFP4_KV_E1M2;

@@ -62,6 +62,40 @@ def test_kv_append_bit_exact(N, shifted):
     assert np.array_equal(u8(cache.v_codes), rvc) and np.array_equal(u8(cache.v_scales), rvs)
 
 
+@pytest.mark.parametrize("rope", [False, True])
+@pytest.mark.parametrize("n", [1, 7, 33])
+def test_kv_append_odd_row_counts_bit_exact(N, rope, n):
+    """One KV head and an odd number of new tokens: the last warp of the
+    append has idle lanes, which must neither read past the inputs nor write."""
+    B, hkv, cap = 2, 1, 40
+    rec = synth.KVRecipe(hkv, seed=13)
+    k, v = rec.kv(n, seed=4)
+    seq = np.arange(n) % B
+    pos = (np.arange(n) // B) * 3 % cap
+    table = O.rope_table(cap)
+    kq = O.rope_f32(f32(k), pos, table) if rope else f32(k)
+    shift = (kq.mean(axis=0) * 0.5).astype(np.float32)
+    gk = O.tensor_scale((kq - shift).astype(np.float32))
+    gv = O.tensor_scale(f32(v))
+    cache = N.KVCache(B, hkv, cap, gk, gv)
+    args = (k.cuda(), v.cuda(), torch.as_tensor(seq, dtype=torch.int32, device="cuda"),
+            torch.as_tensor(pos, dtype=torch.int32, device="cuda"))
+    if rope:
+        N.kv_append_rope_nvfp4(cache, *args, torch.from_numpy(table).cuda(), torch.from_numpy(shift).cuda())
+    else:
+        N.kv_append_nvfp4(cache, *args, torch.from_numpy(shift).cuda())
+    torch.cuda.synchronize()
+    assert N.nvfp4_get_device_status() == 0
+    rkc, rks, rvc, rvs = oracle_cache(B, hkv, cap)
+    if rope:
+        O.kv_append_rope(rkc, rks, rvc, rvs, f32(k), f32(v), seq, pos, np.float32(gk), np.float32(gv), table,
+                         k_shift=shift)
+    else:
+        O.kv_append(rkc, rks, rvc, rvs, f32(k), f32(v), seq, pos, np.float32(gk), np.float32(gv), k_shift=shift)
+    assert np.array_equal(u8(cache.k_codes), rkc) and np.array_equal(u8(cache.k_scales), rks)
+    assert np.array_equal(u8(cache.v_codes), rvc) and np.array_equal(u8(cache.v_scales), rvs)
+
+
 def test_kv_append_out_of_range_sets_capacity_and_skips(N):
     B, hkv, cap = 2, 1, 8
     k = torch.randn(3, hkv, 128).to(torch.bfloat16)
