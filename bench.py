@@ -48,7 +48,7 @@ CSRC = os.path.join(ROOT, "paper_2606_15682_gb300", "csrc")
 # same kernel and shape (commands in profiles/).  Each entry holds only while the kernel sources
 # hash to the value they had at capture time; otherwise the line reports traffic = null.
 NCU_TRAFFIC = {
-    "gemm": {"bytes": 204993536 + 861905664, "sources": ("gemm.cu", "common.cuh"), "sha": "49e35d7b86aa45c7",
+    "gemm": {"bytes": 205745920 + 861377536, "sources": ("gemm.cu", "common.cuh"), "sha": "1dc61211627969f1",
              "shape": (8192, 55296, 5120),
              "profile": "profiles/gemm_qwen32b_prefill_gate_up_m8192_n55296_k5120.md"},
     "attention": {"bytes": 1208885248 + 22256640, "sources": ("attention.cu", "common.cuh"),
@@ -374,6 +374,20 @@ def run_ours(args, rank, world):
                                                                        gemm_bytes(Mw, L["N"], L["K"]),
                                                                        b2b[L["name"]]) for L in lw},
                  "algorithmic_gemm_bytes": byt}
+        if Mw <= 32 and all(L["K"] <= 1536 for L in lw):
+            # The same step through nvfp4_linear_dynamic: tensor scale,
+            # quantization and GEMM of each linear in one launch (bit-identical
+            # outputs, checked in the GPU tests).
+            def one_launch_step(lw=lw):
+                for L in lw:
+                    N.nvfp4_linear_dynamic(L["a"], L["wc"], L["ws"], L["gw"], L["out"], L["N"], g_a=L["ga"])
+
+            gf = graph_of(one_launch_step)
+            ms_f = statistics.mean(timed_loop(gf.replay, other_steps, args.warmup))
+            entry["one_launch"] = {"step": "per linear: nvfp4_linear_dynamic (tensor scale, quantization and "
+                                           "GEMM in one launch)",
+                                   "ms_per_step": ms_f, "tflops": fw / (ms_f * 1e-3) / 1e12}
+            del gf
         kva = synth.WORKLOADS[wl].get("kv_append")
         if kva:
             # One new token for each of n_new sequences, K and V quantized and appended.

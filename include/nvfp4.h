@@ -166,6 +166,32 @@ nvfp4_status nvfp4_linear(const uint8_t* a_codes, const uint8_t* a_scales, const
                           void* stream);
 
 /*
+ * a1 + a2 + a3 in one launch for a small activation: the tensor scale of x,
+ * its NVFP4 quantization and the linear layer with W (Appendix A format,
+ * Appendix D.1 linears; the tensor-scale reduction fused into the GEMM's
+ * prologue).  Every CTA reduces the amax of the whole of x and quantizes it
+ * into its own shared memory, so no grid barrier is needed.  g_a, the
+ * quantized A and out are bit-identical to nvfp4_quantize_dynamic (MMA
+ * scales) followed by nvfp4_linear; the quantized A is not written to
+ * global memory.
+ *   x_bf16   : [M, K] bf16, leading dimension ld_x >= K (elements), 16-B
+ *              aligned, ld_x % 8 == 0.
+ *   w_codes, w_scales, g_w, out_bf16, ldo : as nvfp4_linear.
+ *   g_a_out  : device float that receives g_a, or NULL.
+ * 1 <= M <= 32 and K <= 1536 (UNSUPPORTED otherwise: each CTA holds all of
+ * x in registers and all of A in shared memory, and quantizes it itself;
+ * measured on GB300 at N = K = 1536, one launch is faster than the two calls
+ * up to M = 16, on par at M = 32 and 1.7x slower at M = 64); K % 256 == 0, N % 16 == 0, ldo >= N, ldo % 8 == 0
+ * (SHAPE); pointers 16-B aligned, g_w and g_a_out 4-B aligned (ALIGN).  A
+ * bounded on-device wait that expires sets NVFP4_ERR_TIMEOUT and leaves out
+ * undefined.
+ */
+nvfp4_status nvfp4_linear_dynamic(const void* x_bf16, int64_t M, int64_t K, int64_t ld_x,
+                                  const uint8_t* w_codes, const uint8_t* w_scales, const float* g_w,
+                                  int64_t N, void* out_bf16, int64_t ldo, float* g_a_out,
+                                  void* stream);
+
+/*
  * a3 for the gate_up projection, with the down projection's input produced in
  * the epilogue: h[m, i] = SiLU(G[m, i]) * U[m, i], where G and U are the gate
  * and up halves of the block-scaled product exactly as nvfp4_linear forms them

@@ -10,6 +10,7 @@
     python -m paper_2606_15682_gb300.cases mx_gemm_swiglu --workload qwen32b_prefill_linears_m8192 --rotate
     NVFP4_TIMELINE=1 python -m paper_2606_15682_gb300.cases quantize_timeline --workload qwen1.5b_prefill_linears_m2048 --linear qkv
     NVFP4_TIMELINE=1 python -m paper_2606_15682_gb300.cases gemm_timeline --workload w4a4_linear_m16_k1536_n1536 --linear linear
+    python -m paper_2606_15682_gb300.cases linear_dynamic --workload w4a4_linear_m16_k1536_n1536 --linear linear
 
 Inputs are seeded synthetic tensors (paper_2606_15682_gb300.synth); for the
 attention case the cache is filled with seeded random codes and scales
@@ -140,7 +141,7 @@ def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("kernel", choices=["gemm", "gemm_swiglu", "quantize", "quantize_dynamic", "tensor_scale",
                                        "attention", "mx_gemm", "mx_quantize", "mx_gemm_swiglu", "quantize_timeline",
-                                       "gemm_timeline"])
+                                       "gemm_timeline", "linear_dynamic"])
     ap.add_argument("--rotate", action="store_true", help="MXFP4: 32-element block rotation before quantizing")
     ap.add_argument("--workload", default="qwen1.5b_prefill_linears_m2048")
     ap.add_argument("--linear", default="gate_up")
@@ -242,6 +243,27 @@ def main():
             ms = _time(lambda: N.mxfp4_linear(ac, asf, wc, wsf, out, M, Nn, K), a.iters)
             print(f"mx_gemm {a.workload}/{a.linear} {M}x{Nn}x{K}: {ms * 1e3:.1f} us, "
                   f"{2 * M * Nn * K / ms / 1e9:.1f} TFLOP/s")
+    elif a.kernel == "linear_dynamic":
+        # Tensor scale, quantization and GEMM in one launch (M <= 32), against
+        # the one-launch quantizer followed by the GEMM.
+        x, W = synth.linear_inputs(a.workload, a.linear, device=dev)
+        M, K = x.shape
+        Nn = W.shape[0]
+        wc, wsf, gw = _quantized(W)
+        del W
+        out = torch.empty(M, Nn, dtype=torch.bfloat16, device=dev)
+        ga = torch.empty(1, dtype=torch.float32, device=dev)
+        ms_f = _time(lambda: N.nvfp4_linear_dynamic(x, wc, wsf, gw, out, Nn, g_a=ga), a.iters)
+        st = torch.zeros(N.DYNAMIC_STATE_BYTES, dtype=torch.uint8, device=dev)
+        ac = torch.empty(M, K // 2, dtype=torch.uint8, device=dev)
+        asf = torch.empty(N.nvfp4_scales_bytes(M, K, N.SCALES_MMA), dtype=torch.uint8, device=dev)
+
+        def two_calls():
+            N.nvfp4_quantize_dynamic(x, st, ga, ac, asf, N.SCALES_MMA)
+            N.nvfp4_linear(ac, asf, ga, wc, wsf, gw, out, M, Nn, K)
+        ms_u = _time(two_calls, a.iters)
+        print(f"linear_dynamic {a.workload}/{a.linear} {M}x{Nn}x{K}: one launch {ms_f * 1e3:.1f} us, "
+              f"quantize_dynamic + linear {ms_u * 1e3:.1f} us")
     elif a.kernel in ("gemm", "quantize", "quantize_dynamic", "tensor_scale"):
         x, W = synth.linear_inputs(a.workload, a.linear, device=dev)
         M, K = x.shape

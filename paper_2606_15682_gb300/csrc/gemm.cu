@@ -1320,6 +1320,358 @@ __global__ void __launch_bounds__(C::kThreads, 1)
   if (warp == 1) tmem_dealloc_pair(tmem, kTmemCols);
 }
 
+// ------------------------------------- quantize-in-prologue linear kernel ---
+// a1 + a2 + a3 in one launch for an activation of at most 32 rows and K of
+// at most 1536: every CTA reads the whole bf16 activation x (at most 96 KB,
+// an L2 hit after the first CTA), reduces its amax, forms the tensor scale g_a
+// and quantizes x into its own shared memory in the MMA layout (codes in the
+// 128-byte-swizzled K-major tiles the tensor core reads, block scales in
+// 512-byte atoms), exactly as nvfp4_quantize_dynamic would; no grid barrier
+// is needed because each CTA does the reduction itself.  A and its scales then
+// stay resident (A scales in TMEM for the whole K) while the producer streams
+// only W through a 5-stage ring, from the kernel's first instruction on.
+//   warp 0      TMA producer for W codes and scales (skips the prologue)
+//   warps 1-11  prologue (amax, then quantization), then:
+//   warp 1      TMEM allocation; one lane issues the MMAs
+//   warp 2      one lane copies the A scales once, then each stage's W scales
+//   warps 3-6   epilogue (double-buffered 128-column accumulator)
+struct DynCfg {
+  static constexpr int BN = 128;
+  static constexpr int kStages = 5;
+  static constexpr int kMaxKb = 6;                          // K <= 1536
+  static constexpr int kMaxRows = 32;                       // M <= 32
+  static constexpr int kEpiWarps = 4;
+  // Warps 7-11 only help with the prologue, whose per-block arithmetic
+  // (E4M3 scale, reciprocal, 16 conversions) is latency-bound with few warps.
+  static constexpr int kThreads = 384;
+  static constexpr int kProThreads = kThreads - 32;          // warps 1-11
+  static constexpr uint32_t kTileBytesA = BM * BK / 2;       // 16 KiB per k-block
+  static constexpr uint32_t kTileBytesB = BN * BK / 2;       // 16 KiB per stage
+  static constexpr uint32_t kSfaBytes = 128 * (BK / 16);     // 2 KiB per k-block: four 512-byte atoms
+  static constexpr uint32_t kSfbBytes = kSfaBytes;
+  static constexpr uint32_t kSfaResCol = 2 * BN;             // A scales: 16 columns per k-block
+  static constexpr uint32_t kSfbCol = kSfaResCol + 16 * kMaxKb;  // W scales: 16 columns per stage
+  static constexpr size_t kSmemBytes = 1024 + kMaxKb * (kTileBytesA + kSfaBytes) +
+                                       kStages * (kTileBytesB + kSfbBytes) + kEpiWarps * kEpiBufBytes + 512;
+  static constexpr uint32_t kIdesc = (1u << 7) | (1u << 10) | (static_cast<uint32_t>(BN >> 3) << 17) |
+                                     (static_cast<uint32_t>(BM >> 4) << 24);
+  static_assert(kSfbCol + kStages * 16 <= kTmemCols, "TMEM budget");
+  static_assert(kSmemBytes <= 227 * 1024, "shared memory budget");
+};
+
+struct DynArgs {
+  const uint16_t* x;  // bf16 [M, K], row pitch ldx elements
+  int64_t ldx;
+  const uint8_t* sfb;
+  const float* gb;
+  float* g_out;  // optional: g_a
+  int M, N, K;
+  int tiles_n;
+  int* status;
+};
+
+__device__ __forceinline__ void named_barrier(uint32_t id, uint32_t threads) {
+  asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(threads) : "memory");
+}
+__device__ __forceinline__ void st_shared_v2_u32(uint32_t addr, uint32_t a, uint32_t b) {
+  asm volatile("st.shared.v2.b32 [%0], {%1, %2};" ::"r"(addr), "r"(a), "r"(b) : "memory");
+}
+__device__ __forceinline__ void st_shared_u32(uint32_t addr, uint32_t v) {
+  asm volatile("st.shared.u32 [%0], %1;" ::"r"(addr), "r"(v) : "memory");
+}
+__device__ __forceinline__ void st_shared_u8(uint32_t addr, uint32_t v) {
+  asm volatile("st.shared.u8 [%0], %1;" ::"r"(addr), "r"(v) : "memory");
+}
+
+template <class C>
+__global__ void __launch_bounds__(C::kThreads, 1)
+    nvfp4_linear_dyn_kernel(const __grid_constant__ CUtensorMap tmap_b, const __grid_constant__ CUtensorMap tmap_out,
+                            const DynArgs args) {
+  constexpr int BN = C::BN;
+  constexpr int kStages = C::kStages;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* sA = smem;                                        // resident A, one 16 KiB tile per k-block
+  uint8_t* sB = sA + C::kMaxKb * C::kTileBytesA;
+  uint8_t* sEpi = sB + kStages * C::kTileBytesB;
+  uint8_t* sSFA = sEpi + C::kEpiWarps * kEpiBufBytes;        // resident A scale atoms
+  uint8_t* sSFB = sSFA + C::kMaxKb * C::kSfaBytes;
+  uint64_t* full = reinterpret_cast<uint64_t*>(sSFB + kStages * C::kSfbBytes);
+  uint64_t* empty = full + kStages;
+  uint64_t* sfready = empty + kStages;
+  uint64_t* tfull = sfready + kStages;
+  uint64_t* tempty = tfull + 2;
+  uint64_t* aready = tempty + 2;
+  uint64_t* drain = aready + 1;
+  uint64_t* drain_cp = drain + 1;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain_cp + 1);
+  __shared__ volatile int abort_flag;
+  __shared__ uint32_t warp_max[C::kThreads / 32];
+  __shared__ float s_g;
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int kblocks = args.K / BK;
+  const int kgroups = args.K / 64;
+  const int total_units = args.tiles_n;
+  const int cta_id = blockIdx.x, n_ctas = gridDim.x;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+      mbar_init(&sfready[s], 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(&tfull[a], 1);
+      mbar_init(&tempty[a], C::kEpiWarps);
+    }
+    mbar_init(aready, 1);
+    mbar_init(drain, 1);
+    mbar_init(drain_cp, 1);
+    abort_flag = 0;
+    fence_mbar_init();
+    prefetch_tmap(&tmap_b);
+    prefetch_tmap(&tmap_out);
+  }
+  if (warp == 1) {
+    tmem_alloc(tmem_slot, kTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  griddep_wait_and_release();
+  const uint32_t tmem = *tmem_slot;
+
+  auto fail = [&]() {
+    set_status(args.status, NVFP4_ERR_TIMEOUT);
+    abort_flag = 1;
+  };
+
+  if (warp == 0) {
+    // ------------------------------------------------------ TMA producer ---
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t phase = 0;
+      uint32_t issued_parity[kStages];
+      bool issued[kStages];
+      for (int s = 0; s < kStages; ++s) issued[s] = false;
+      for (int u = cta_id; u < total_units && !abort_flag; u += n_ctas) {
+        const uint8_t* sfb_tile = args.sfb + (static_cast<size_t>(u) * kgroups) * 512;
+        for (int kb = 0; kb < kblocks; ++kb) {
+          if (!mbar_wait_bounded(&empty[stage], phase ^ 1u, &abort_flag)) { fail(); break; }
+          mbar_arrive_expect_tx(&full[stage], C::kTileBytesB + C::kSfbBytes);
+          bulk_load(sSFB + stage * C::kSfbBytes, sfb_tile + static_cast<size_t>(kb) * C::kSfbBytes, C::kSfbBytes,
+                    &full[stage]);
+          tma_load_2d(sB + stage * C::kTileBytesB, &tmap_b, &full[stage], kb * (BK / 2), u * BN);
+          issued[stage] = true;
+          issued_parity[stage] = phase;
+          if (++stage == kStages) { stage = 0; phase ^= 1u; }
+        }
+      }
+      if (abort_flag)
+        for (int s = 0; s < kStages; ++s)
+          if (issued[s]) mbar_wait_bounded(&full[s], issued_parity[s], nullptr);
+    }
+  } else {
+    // ------------------------------- prologue: g_a and A into shared memory ---
+    // Thread pt owns the 16-element blocks pt, pt + 352, ... of x in row-major
+    // block order; they stay in registers from the amax pass to the
+    // quantization pass, so x is read once.
+    constexpr int kKeep = 10;
+    static_assert(kKeep * C::kProThreads >= C::kMaxRows * C::kMaxKb * (BK / 16), "x fits in registers");
+    const uint32_t pt = threadIdx.x - 32;
+    const uint32_t kb16 = static_cast<uint32_t>(args.K) / 16;
+    const uint32_t M = static_cast<uint32_t>(args.M);
+    const uint32_t live = M * kb16;
+    auto block_src = [&](uint32_t b) {
+      const uint32_t r = b / kb16, j = b - r * kb16;
+      return reinterpret_cast<const uint4*>(args.x + static_cast<int64_t>(r) * args.ldx + j * 16);
+    };
+    uint4 lo[kKeep], hi[kKeep];
+#pragma unroll
+    for (int i = 0; i < kKeep; ++i) {
+      const uint32_t b = pt + i * C::kProThreads;
+      lo[i] = hi[i] = make_uint4(0, 0, 0, 0);
+      if (b < live) {
+        const uint4* src = block_src(b);
+        lo[i] = __ldg(src);
+        hi[i] = __ldg(src + 1);
+      }
+    }
+    const uint32_t sA0 = smem_u32(sA), sSFA0 = smem_u32(sSFA);
+    // Rows M..127 of the tile: zero codes and zero scales, as the two-call
+    // path gets from the TMA fill and the quantizer's padding rows.
+    {
+      const uint32_t pad_chunks = (128u - M) * 8u;  // 16-byte chunks per k-block
+      for (uint32_t i = pt; i < static_cast<uint32_t>(kblocks) * pad_chunks; i += C::kProThreads) {
+        const uint32_t kb = i / pad_chunks, c = i - kb * pad_chunks;
+        st_shared_v4(sA0 + kb * C::kTileBytesA + M * 128u + c * 16u, 0u, 0u, 0u, 0u);
+      }
+      const uint32_t pad_rows = 128u - M;
+      for (uint32_t i = pt; i < static_cast<uint32_t>(kgroups) * pad_rows; i += C::kProThreads) {
+        const uint32_t jg = i / pad_rows, r = M + (i - jg * pad_rows);
+        st_shared_u32(sSFA0 + jg * 512u + (r & 31u) * 16u + ((r >> 5) & 3u) * 4u, 0u);
+      }
+    }
+    uint32_t m = 0;
+#pragma unroll
+    for (int i = 0; i < kKeep; ++i) m = max(m, max(amax_bits_bf16x8(lo[i]), amax_bits_bf16x8(hi[i])));
+    m = __reduce_max_sync(0xffffffffu, m);
+    if (lane == 0) warp_max[warp] = m;
+    named_barrier(1, C::kProThreads);
+    if (pt == 0) {
+      uint32_t mm = 0;
+      for (int w = 1; w < C::kThreads / 32; ++w) mm = max(mm, warp_max[w]);
+      // g_a = amax / (6 * 448), or 1 for an all-zero tensor: the dynamic
+      // quantizer's tensor scale, bit for bit.
+      const float amax = __uint_as_float(mm << 16);
+      const float gv = amax > 0.0f ? __fdiv_rn(amax, 2688.0f) : 1.0f;
+      s_g = gv;
+      if (blockIdx.x == 0 && args.g_out) *args.g_out = gv;
+    }
+    named_barrier(1, C::kProThreads);
+    const float g = s_g, six_g = __fmul_rn(6.0f, g);
+    // One 16-element block: E4M3 scale and 16 E2M1 codes, stored where the
+    // TMA load of the two-call path would have put them (row r at r * 128 in
+    // its k-block tile, 16-byte chunk c at (c ^ r % 8) * 16) and the scale
+    // byte at its place in the 512-byte atom of its 64-element group.
+    auto quantize_block = [&](uint32_t b, const uint4 v0, const uint4 v1) {
+      const uint32_t r = b / kb16, j = b - r * kb16;
+      float xf[16];
+      unpack_bf16x8(v0, xf);
+      unpack_bf16x8(v1, xf + 8);
+      const float amax = __uint_as_float(max(amax_bits_bf16x8(v0), amax_bits_bf16x8(v1)) << 16);
+      const BlockScale bs = block_scale(amax, g, six_g);
+      float q[16];
+#pragma unroll
+      for (int i = 0; i < 16; ++i) q[i] = __fmul_rn(xf[i], bs.mult);
+      const uint32_t kb = j >> 4, e = j & 15u;
+      st_shared_v2_u32(sA0 + kb * C::kTileBytesA + r * 128u + (((e >> 1) ^ (r & 7u)) << 4) + (e & 1u) * 8u,
+                       e2m1x8(q), e2m1x8(q + 8));
+      st_shared_u8(sSFA0 + (j >> 2) * 512u + (r & 31u) * 16u + ((r >> 5) & 3u) * 4u + (j & 3u), bs.code);
+    };
+#pragma unroll
+    for (int i = 0; i < kKeep; ++i) {
+      const uint32_t b = pt + i * C::kProThreads;
+      if (b < live) quantize_block(b, lo[i], hi[i]);
+    }
+    fence_proxy_async_smem();  // the tensor core reads A and its scales through the async proxy
+    named_barrier(1, C::kProThreads);
+
+    if (warp == 1 && lane == 0) {
+      // ------------------------------------------------------- MMA issuer ---
+      int stage = 0;
+      uint32_t phase = 0;
+      int local = 0;
+      const uint32_t sB0 = smem_u32(sB);
+      bool ok = mbar_wait_bounded(aready, 0, &abort_flag);
+      if (!ok) fail();
+      for (int u = cta_id; ok && u < total_units && !abort_flag; u += n_ctas, ++local) {
+        const int acc = local & 1;
+        const uint32_t acc_phase = (local >> 1) & 1;
+        if (!mbar_wait_bounded(&tempty[acc], acc_phase ^ 1u, &abort_flag)) { fail(); break; }
+        tc_fence_after();
+        const uint32_t d_tmem = tmem + acc * BN;
+        for (int kb = 0; kb < kblocks; ++kb) {
+          if (!mbar_wait_bounded(&sfready[stage], phase, &abort_flag)) { fail(); ok = false; break; }
+          tc_fence_after();
+          const uint32_t sfa_col = tmem + C::kSfaResCol + kb * 16;
+          const uint32_t sfb_col = tmem + C::kSfbCol + stage * 16;
+#pragma unroll
+          for (int kk = 0; kk < 4; ++kk)
+            mma_fp4(d_tmem, desc_sw128(sA0 + kb * C::kTileBytesA + kk * 32),
+                    desc_sw128(sB0 + stage * C::kTileBytesB + kk * 32), C::kIdesc, sfa_col + kk * 4,
+                    sfb_col + kk * 4, (kb | kk) != 0);
+          tc_commit(&empty[stage]);
+          if (++stage == kStages) { stage = 0; phase ^= 1u; }
+        }
+        if (!ok) break;
+        tc_commit(&tfull[acc]);
+      }
+      tc_commit(drain);
+      mbar_wait_bounded(drain, 0, nullptr);
+    } else if (warp == 2 && lane == 0) {
+      // ------------------------------------------- block scales -> TMEM ---
+      for (int kb = 0; kb < kblocks; ++kb)
+#pragma unroll
+        for (int kk = 0; kk < 4; ++kk)
+          copy_sf_to_tmem(tmem + C::kSfaResCol + kb * 16 + kk * 4, desc_sf(sSFA0 + kb * C::kSfaBytes + kk * 512));
+      tc_commit(aready);
+      int stage = 0;
+      uint32_t phase = 0;
+      const uint32_t sSFB0 = smem_u32(sSFB);
+      bool ok = true;
+      for (int u = cta_id; ok && u < total_units && !abort_flag; u += n_ctas) {
+        for (int kb = 0; kb < kblocks; ++kb) {
+          if (!mbar_wait_bounded(&full[stage], phase, &abort_flag)) { fail(); ok = false; break; }
+          tc_fence_after();
+#pragma unroll
+          for (int kk = 0; kk < 4; ++kk)
+            copy_sf_to_tmem(tmem + C::kSfbCol + stage * 16 + kk * 4, desc_sf(sSFB0 + stage * C::kSfbBytes + kk * 512));
+          tc_commit(&sfready[stage]);
+          if (++stage == kStages) { stage = 0; phase ^= 1u; }
+        }
+      }
+      tc_commit(drain_cp);
+      mbar_wait_bounded(drain_cp, 0, nullptr);
+    } else if (warp >= 3 && warp < 3 + C::kEpiWarps) {
+      // --------------------------------------------------------- epilogue ---
+      const int quarter = warp & 3;
+      uint8_t* buf_ptr = sEpi + (warp - 3) * kEpiBufBytes;
+      const uint32_t buf = smem_u32(buf_ptr);
+      const float scale = __fmul_rn(g, __ldg(args.gb));
+      int local = 0;
+      for (int u = cta_id; u < total_units; u += n_ctas, ++local) {
+        const int acc = local & 1;
+        const uint32_t acc_phase = (local >> 1) & 1;
+        int ok = 1;
+        if (lane == 0) {
+          ok = !abort_flag && mbar_wait_bounded(&tfull[acc], acc_phase, &abort_flag);
+          if (!ok && !abort_flag) fail();
+        }
+        if (!__shfl_sync(0xffffffffu, ok, 0)) break;
+        tc_fence_after();
+        uint32_t r[128];
+        const uint32_t taddr = tmem + (static_cast<uint32_t>(quarter * 32) << 16) + acc * BN;
+#pragma unroll
+        for (int c = 0; c < 4; ++c) tmem_ld32(taddr + c * 32, r + 32 * c);
+        tmem_ld_wait();
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&tempty[acc]);
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+          if (lane == 0) bulk_wait_read_all();
+          __syncwarp();
+#pragma unroll
+          for (int c = 0; c < 8; ++c) {
+            const uint32_t* v = r + 64 * h + 8 * c;
+            st_shared_v4(buf + lane * 128 + ((c ^ (lane & 7)) << 4),
+                         pack_bf16x2(__uint_as_float(v[0]) * scale, __uint_as_float(v[1]) * scale),
+                         pack_bf16x2(__uint_as_float(v[2]) * scale, __uint_as_float(v[3]) * scale),
+                         pack_bf16x2(__uint_as_float(v[4]) * scale, __uint_as_float(v[5]) * scale),
+                         pack_bf16x2(__uint_as_float(v[6]) * scale, __uint_as_float(v[7]) * scale));
+          }
+          fence_proxy_async_smem();
+          __syncwarp();
+          const int x = u * BN + h * kEpiCols, y = quarter * 32;
+          if (lane == 0 && x < args.N && y < args.M) {
+            tma_store_2d(&tmap_out, buf_ptr, x, y);
+            bulk_commit_group();
+          }
+        }
+      }
+      if (lane == 0) bulk_wait_all();
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (warp == 1) tmem_dealloc(tmem, kTmemCols);
+}
+
 // ------------------------------------------------------------------- host ---
 
 PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
@@ -1626,6 +1978,49 @@ nvfp4_status launch_splitk(const uint8_t* a_codes, const uint8_t* a_scales, cons
   return launch_status();
 }
 
+// nvfp4_linear_dynamic: one persistent CTA per 128-column tile of W, at most
+// one per SM.
+nvfp4_status launch_dynamic(const uint16_t* x, int64_t M, int64_t K, int64_t ldx, const uint8_t* w_codes,
+                            const uint8_t* w_scales, const float* g_w, int64_t N, void* out_bf16, int64_t ldo,
+                            float* g_out, cudaStream_t stream) {
+  using C = DynCfg;
+  static std::mutex mu;
+  static std::map<int, bool> ready;
+  int d = 0;
+  if (cudaGetDevice(&d) != cudaSuccess) return NVFP4_ERR_CUDA;
+  {
+    std::lock_guard<std::mutex> lock(mu);
+    if (!ready[d]) {
+      if (cudaFuncSetAttribute(nvfp4_linear_dyn_kernel<C>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                               static_cast<int>(C::kSmemBytes)) != cudaSuccess)
+        return NVFP4_ERR_CUDA;
+      ready[d] = true;
+    }
+  }
+  const int64_t tiles_n = (N + C::BN - 1) / C::BN;
+  CUtensorMap mb, mo;
+  if (!make_code_map(&mb, w_codes, N, K, C::BN) || !make_out_map(&mo, out_bf16, M, N, ldo)) return NVFP4_ERR_CUDA;
+  DynArgs args = {};
+  args.x = x;
+  args.ldx = ldx;
+  args.sfb = w_scales;
+  args.gb = g_w;
+  args.g_out = g_out;
+  args.M = static_cast<int>(M);
+  args.N = static_cast<int>(N);
+  args.K = static_cast<int>(K);
+  args.tiles_n = static_cast<int>(tiles_n);
+  args.status = status_word_dev();
+  const int sms = sm_count();
+  if (sms <= 0) return NVFP4_ERR_CUDA;
+  const int ctas = static_cast<int>(tiles_n < sms ? tiles_n : sms);
+  if (launch_pdl(nvfp4_linear_dyn_kernel<C>, dim3(ctas), dim3(C::kThreads), C::kSmemBytes, stream, mb, mo, args) !=
+      cudaSuccess)
+    return NVFP4_ERR_CUDA;
+  count_launches(1);
+  return launch_status();
+}
+
 #ifndef NVFP4_GEMM_BN
 #define NVFP4_GEMM_BN 0  // 0: choose per shape
 #endif
@@ -1709,6 +2104,21 @@ NVFP4_API nvfp4_status nvfp4_linear(const uint8_t* a_codes, const uint8_t* a_sca
     return NVFP4_ERR_ALIGN;
   return linear_dispatch(a_codes, a_scales, g_a, w_codes, w_scales, g_w, M, N, K, out_bf16, ldo,
                          static_cast<cudaStream_t>(stream), 0);
+}
+
+NVFP4_API nvfp4_status nvfp4_linear_dynamic(const void* x_bf16, int64_t M, int64_t K, int64_t ld_x,
+                                            const uint8_t* w_codes, const uint8_t* w_scales, const float* g_w,
+                                            int64_t N, void* out_bf16, int64_t ldo, float* g_a_out, void* stream) {
+  NVFP4_TRACE("nvfp4_linear_dynamic");
+  if (!x_bf16 || !w_codes || !w_scales || !g_w || !out_bf16) return NVFP4_ERR_INVALID_ARG;
+  if (M <= 0 || N <= 0 || K <= 0 || K % BK || N % 16 || ldo < N || ldo % 8 || ld_x < K) return NVFP4_ERR_SHAPE;
+  if (M > DynCfg::kMaxRows || K > static_cast<int64_t>(DynCfg::kMaxKb) * BK) return NVFP4_ERR_UNSUPPORTED;
+  if (N >= (1ll << 31) || ld_x >= (1ll << 31)) return NVFP4_ERR_SHAPE;
+  if (!aligned(x_bf16, 16) || ld_x % 8 || !aligned(w_codes, 16) || !aligned(w_scales, 16) || !aligned(out_bf16, 16) ||
+      !aligned(g_w, 4) || !aligned(g_a_out, 4))
+    return NVFP4_ERR_ALIGN;
+  return launch_dynamic(static_cast<const uint16_t*>(x_bf16), M, K, ld_x, w_codes, w_scales, g_w, N, out_bf16, ldo,
+                        g_a_out, static_cast<cudaStream_t>(stream));
 }
 
 NVFP4_API nvfp4_status mxfp4_linear(const uint8_t* a_codes, const uint8_t* a_scales, const uint8_t* w_codes,

@@ -57,6 +57,7 @@ _quantize = _sig("nvfp4_quantize", [_p, _i64, _i64, _i64, _p, _p, _p, ctypes.c_i
 _quantize_dynamic = _sig("nvfp4_quantize_dynamic", [_p, _i64, _i64, _i64, _p, _p, _p, _p, ctypes.c_int, _p])
 _relayout = _sig("nvfp4_scales_relayout", [_p, _p, _i64, _i64, ctypes.c_int, ctypes.c_int, _p])
 _linear = _sig("nvfp4_linear", [_p, _p, _p, _p, _p, _p, _i64, _i64, _i64, _p, _i64, _p])
+_linear_dynamic = _sig("nvfp4_linear_dynamic", [_p, _i64, _i64, _i64, _p, _p, _p, _i64, _p, _i64, _p, _p])
 _linear_swiglu = _sig("nvfp4_linear_swiglu_quantize", [_p, _p, _p, _p, _p, _p, _i64, _i64, _i64, _p, _p, _p, _p])
 _interleave = _sig("nvfp4_interleave_gate_up", [_p, _p, _i64, _i64, _p, _p])
 _kv_append = _sig("kv_append_nvfp4", [ctypes.POINTER(KVCacheStruct), _p, _p, _p, _p, _i64, _p, _p])
@@ -160,6 +161,16 @@ def nvfp4_scales_relayout(src, dst, rows, cols, from_layout, to_layout, stream=N
 def nvfp4_linear(a_codes, a_scales, g_a, w_codes, w_scales, g_w, out, M, N, K, ldo=None, stream=None):
     _check("nvfp4_linear", _linear(_ptr(a_codes), _ptr(a_scales), _ptr(g_a), _ptr(w_codes), _ptr(w_scales),
                                    _ptr(g_w), M, N, K, _ptr(out), N if ldo is None else ldo, _stream(stream)))
+
+
+def nvfp4_linear_dynamic(x, w_codes, w_scales, g_w, out, N, ldo=None, g_a=None, stream=None):
+    """Tensor scale, quantization of the bf16 activation x [M, K] (M <= 32,
+    K <= 1536) and the linear layer with W in one launch; g_a (optional
+    device float) receives the tensor scale."""
+    ptr, M, K, ld = _mat(x)
+    _check("nvfp4_linear_dynamic", _linear_dynamic(ptr, M, K, ld, _ptr(w_codes), _ptr(w_scales), _ptr(g_w), N,
+                                                   _ptr(out), N if ldo is None else ldo, _ptr(g_a),
+                                                   _stream(stream)))
 
 
 def mxfp4_scales_bytes(rows, cols, layout):
@@ -304,6 +315,7 @@ class KVCache:
 
 
 EXPORTED = ["nvfp4_scales_bytes", "nvfp4_tensor_scale", "nvfp4_quantize", "nvfp4_quantize_dynamic", "nvfp4_scales_relayout", "nvfp4_linear",
+            "nvfp4_linear_dynamic",
             "nvfp4_linear_swiglu_quantize", "nvfp4_interleave_gate_up",
             "mxfp4_scales_bytes", "mxfp4_quantize", "mxfp4_linear", "mxfp4_linear_swiglu_quantize",
             "kv_append_nvfp4", "kv_append_rope_nvfp4", "nvfp4_rope_table", "decode_attention_nvfp4_workspace_size", "decode_attention_nvfp4",

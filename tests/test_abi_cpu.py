@@ -100,6 +100,20 @@ def test_argument_validation_before_launch():
     assert L.nvfp4_quantize_dynamic(p, 4, 32, 32, st, p, p, p, 1, s) == 2     # MMA layout needs cols % 64
     assert L.nvfp4_quantize_dynamic(p, 4, 64, 64, st, p, p, p, 9, s) == 1     # bad layout enum
     assert L.nvfp4_quantize_dynamic(p, 4, 64, 64, st, p, None, p, 1, s) == 1  # no codes
+    # one-launch quantize + linear: M <= 32 and K <= 1536, else UNSUPPORTED
+    ld = L.nvfp4_linear_dynamic
+    assert ld(None, 16, 1536, 1536, p, p, p, 1536, p, 1536, None, s) == 1
+    assert ld(p, 16, 1536, 1536, p, p, None, 1536, p, 1536, None, s) == 1
+    assert ld(p, 33, 1536, 1536, p, p, p, 1536, p, 1536, None, s) == 4
+    assert ld(p, 16, 1792, 1792, p, p, p, 1536, p, 1536, None, s) == 4
+    assert ld(p, 0, 1536, 1536, p, p, p, 1536, p, 1536, None, s) == 2
+    assert ld(p, 16, 1280 + 64, 1344, p, p, p, 1536, p, 1536, None, s) == 2   # K % 256
+    assert ld(p, 16, 1536, 1528, p, p, p, 1536, p, 1536, None, s) == 2        # ld_x < K
+    assert ld(p, 16, 1536, 1536, p, p, p, 1544, p, 1536, None, s) == 2        # ldo < N
+    assert ld(p, 16, 1536, 1536, p, p, p, 120 + 4, p, 128, None, s) == 2      # N % 16
+    assert ld(odd, 16, 1536, 1536, p, p, p, 1536, p, 1536, None, s) == 3
+    assert ld(p, 16, 1536, 1540, p, p, p, 1536, p, 1536, None, s) == 3        # ld_x % 8
+    assert ld(p, 16, 1536, 1536, p, p, p, 1536, p, 1536, odd, s) == 3         # g_a_out 4-B aligned
 
 
 def test_mxfp4_validation_before_launch():
