@@ -148,6 +148,8 @@ def main():
     ap.add_argument("--batch", type=int, default=64)
     ap.add_argument("--context", type=int, default=16384)
     ap.add_argument("--iters", type=int, default=3)
+    ap.add_argument("--rows", type=int, default=None,
+                    help="gemm/quantize: activation rows instead of the workload's M (smaller profiler cases)")
     ap.add_argument("--kv-format", choices=["e2m1", "e1m2"], default="e2m1")
     a = ap.parse_args()
     dev = torch.device("cuda", 0)
@@ -265,7 +267,7 @@ def main():
         print(f"linear_dynamic {a.workload}/{a.linear} {M}x{Nn}x{K}: one launch {ms_f * 1e3:.1f} us, "
               f"quantize_dynamic + linear {ms_u * 1e3:.1f} us")
     elif a.kernel in ("gemm", "quantize", "quantize_dynamic", "tensor_scale"):
-        x, W = synth.linear_inputs(a.workload, a.linear, device=dev)
+        x, W = synth.linear_inputs(a.workload, a.linear, M=a.rows, device=dev)
         M, K = x.shape
         Nn = W.shape[0]
         if a.kernel == "gemm":
