@@ -51,8 +51,8 @@ NCU_TRAFFIC = {
     "gemm": {"bytes": 205745920 + 861377536, "sources": ("gemm.cu", "common.cuh"), "sha": "1dc61211627969f1",
              "shape": (8192, 55296, 5120),
              "profile": "profiles/gemm_qwen32b_prefill_gate_up_m8192_n55296_k5120.md"},
-    "attention": {"bytes": 1208885248 + 22256640, "sources": ("attention.cu", "common.cuh"),
-                  "sha": "76e8785bf56696d1", "shape": (64, 16384),
+    "attention": {"bytes": 1208722432 + 22210816, "sources": ("attention.cu", "common.cuh"),
+                  "sha": "2e035c943bb67759", "shape": (64, 16384),
                   "profile": "profiles/attention_qwen14b_decode_b64_t16384.md (attn_partial_kernel)"},
 }
 

@@ -74,26 +74,36 @@ __device__ __forceinline__ void e2m1x8_to_f16x2(uint32_t w, uint32_t h[4]) {
 
 // E1M2 nibbles (two's complement n, value n/2) decode to f16 n; the 1/2 goes
 // into the block scale.  The nibble XOR 8 in the low mantissa bits of 1024.0
-// (0x6400) reads as 1032 + n, and one f16x2 subtraction of 1032 leaves n.
+// (0x6400) reads as 1032 + n, and one f16x2 subtraction of 1032 leaves n.  A
+// nibble in bits 4-7 of a half is decoded where it stands: 1024 + 16 (n + 8)
+// minus 1152 leaves 16 n, and its block scale carries a further 1/16.  Both
+// are exact, and the product with the scale is the same f16 either way
+// (16 n times s / 16 is n times s, and s / 16 is exact in f16 for every E4M3
+// scale), so the tensor-core operands are those of the shifted decode.
 __device__ __forceinline__ uint32_t hsub2(uint32_t a, uint32_t b) {
   uint32_t d;
   asm("sub.rn.f16x2 %0, %1, %2;" : "=r"(d) : "r"(a), "r"(b));
   return d;
 }
 // K side: the eight nibbles n0..n7 of w (n0 lowest) -> h[i] = (n_i, n_{i+4}),
-// one mask-and-xor and one subtraction per pair.  The channel order inside
-// each group of eight differs from the E2M1 path; the queries are paired the
-// same way, so every logit is the same sum.
+// with h[1] and h[3] holding 16 n (their scales carry the 1/16): one
+// mask-and-xor and one subtraction per pair, one shift per word.  The channel
+// order inside each group of eight differs from the E2M1 path; the queries
+// are paired the same way, so every logit is the same sum.
 __device__ __forceinline__ void e1m2x8_to_f16x2_paired(uint32_t w, uint32_t h[4]) {
-#pragma unroll
-  for (int i = 0; i < 4; ++i) h[i] = hsub2(((w >> (4 * i)) & 0x000F000Fu) ^ 0x64086408u, 0x64086408u);
+  const uint32_t t = w >> 8;
+  h[0] = hsub2((w & 0x000F000Fu) ^ 0x64086408u, 0x64086408u);
+  h[1] = hsub2((w & 0x00F000F0u) ^ 0x64806480u, 0x64806480u);
+  h[2] = hsub2((t & 0x000F000Fu) ^ 0x64086408u, 0x64086408u);
+  h[3] = hsub2((t & 0x00F000F0u) ^ 0x64806480u, 0x64806480u);
 }
 // V side: byte k of two tokens' words a and b -> lo = (a, b) of the byte's
-// low-nibble channel, hi = (a, b) of its high-nibble channel.
+// low-nibble channel, hi = 16 (a, b) of its high-nibble channel (its scale
+// carries the 1/16).
 __device__ __forceinline__ void e1m2_token_pair(uint32_t wa, uint32_t wb, int k, uint32_t* lo, uint32_t* hi) {
   const uint32_t x = __byte_perm(wa, wb, 0x4400u + 0x1111u * k);  // bytes: a_k, a_k, b_k, b_k
   *lo = hsub2((x & 0x000F000Fu) ^ 0x64086408u, 0x64086408u);
-  *hi = hsub2(((x >> 4) & 0x000F000Fu) ^ 0x64086408u, 0x64086408u);
+  *hi = hsub2((x & 0x00F000F0u) ^ 0x64806480u, 0x64806480u);
 }
 
 template <bool kE1M2>
@@ -342,10 +352,12 @@ __global__ void __launch_bounds__(kThreads, NVFP4_ATTN_MIN_CTAS) attn_partial_ke
           decode8<kE1M2>(kaw[w], ha);
           decode8<kE1M2>(kbw[w], hb);
           const uint32_t sa = w < 2 ? sa_lo : sa_hi, sb = w < 2 ? sb_lo : sb_hi;
+          // E1M2: the scales of the pairs decoded as 16 n (times 1/16, exact).
+          const uint32_t sa1 = kE1M2 ? hmul2(sa, 0x2C002C00u) : sa, sb1 = kE1M2 ? hmul2(sb, 0x2C002C00u) : sb;
 #pragma unroll
           for (int h = 0; h < 2; ++h) {  // k-step j = 2w + h uses bytes 2j and 2j+1
-            const uint32_t a[4] = {hmul2(ha[2 * h], sa), hmul2(hb[2 * h], sb), hmul2(ha[2 * h + 1], sa),
-                                   hmul2(hb[2 * h + 1], sb)};
+            const uint32_t a[4] = {hmul2(ha[2 * h], sa), hmul2(hb[2 * h], sb), hmul2(ha[2 * h + 1], sa1),
+                                   hmul2(hb[2 * h + 1], sb1)};
             const int j = 2 * w + h;
             mma16816(s, a, qf[2 * j], qf[2 * j + 1]);
           }
@@ -399,6 +411,9 @@ __global__ void __launch_bounds__(kThreads, NVFP4_ATTN_MIN_CTAS) attn_partial_ke
         // ---- O^T += V_hat^T P^T: 8 m-tiles, m-tile i = channels 16g+2i, 16g+2i+1
         uint32_t vs01 = e4m3x2_to_f16x2(vs01_raw), vs89 = e4m3x2_to_f16x2(vs89_raw);
         if (kE1M2) { vs01 = hmul2(vs01, 0x38003800u); vs89 = hmul2(vs89, 0x38003800u); }
+        // E1M2: the high-nibble channels are decoded as 16 n; their scales carry 1/16 (exact).
+        const uint32_t vs01_hi = kE1M2 ? hmul2(vs01, 0x2C002C00u) : vs01;
+        const uint32_t vs89_hi = kE1M2 ? hmul2(vs89, 0x2C002C00u) : vs89;
         const uint2 va = *reinterpret_cast<const uint2*>(st + kOffVc + (r0 + rv[0]) * 64 + 8 * g);
         const uint2 vb = *reinterpret_cast<const uint2*>(st + kOffVc + (r0 + rv[1]) * 64 + 8 * g);
         const uint2 vc = *reinterpret_cast<const uint2*>(st + kOffVc + (r0 + rv[2]) * 64 + 8 * g);
@@ -427,8 +442,8 @@ __global__ void __launch_bounds__(kThreads, NVFP4_ATTN_MIN_CTAS) attn_partial_ke
           }
 #pragma unroll
           for (int k = 0; k < 4; ++k) {
-            const uint32_t a[4] = {hmul2(f_lo_ab[k], vs01), hmul2(f_hi_ab[k], vs01), hmul2(f_lo_cd[k], vs89),
-                                   hmul2(f_hi_cd[k], vs89)};
+            const uint32_t a[4] = {hmul2(f_lo_ab[k], vs01), hmul2(f_hi_ab[k], vs01_hi), hmul2(f_lo_cd[k], vs89),
+                                   hmul2(f_hi_cd[k], vs89_hi)};
             mma16816(o[4 * half + k], a, pb0, pb1);
           }
         }
